@@ -1,0 +1,216 @@
+/*
+ * starkv.h -- C ABI of the STaR-KV compression stage on one GB300 (sm_103a).
+ *
+ * STaR-KV (Spatio-Temporal Adaptive Re-weighting) compresses the KV cache of a
+ * GUI vision-language model per layer (Algorithm 1, App. A.2):
+ *   1. score the last w window queries against every past key over the GQA
+ *      groups, pool along tokens and average inside each group  (Sec. 3.3);
+ *   2. re-weight by a per-group prior from the online spatial mutual
+ *      information of each group's scores with the screen-patch grid (Sec. 3.4);
+ *   3. discount stale visual tokens by the temporal stability of their
+ *      governing group (Sec. 3.5);
+ *   4. reshape by an entropy-derived temperature (Sec. 3.6);
+ *   5. keep the global top-B historical tokens plus the recent window and
+ *      gather them into a new contiguous cache (Sec. 3.7).
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - Pointers inside starkv_seq are DEVICE pointers (cudaMalloc / torch CUDA
+ *   memory), except for starkv_step_host, where they are HOST pointers.
+ *   The caller owns every input and output buffer; the library owns only the
+ *   state created by starkv_init_state.
+ * - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *   Calls are asynchronous and stream-ordered; none synchronises the stream.
+ * - `workspace` is caller-owned device scratch of at least
+ *   starkv_workspace_bytes(...) bytes, 256-byte aligned.  Its contents are
+ *   undefined on entry and on exit.  Concurrent calls must not share it.
+ * - Layouts (all row-major, contiguous):
+ *     k, v        bf16  [n_layers][G][L][d]
+ *     q           bf16  [n_layers][H][w][d]   post-RoPE queries of the last w tokens
+ *     meta        u32   [n_layers][L]  or [L] shared (meta_layer_stride = 0)
+ *     S           f32   [n_layers][G][L_p]     group score map, L_p = L - w
+ *     score       f32   [n_layers][L_p]        fused score s_t
+ *     idx         i32   [n_layers][B]          kept historical positions, ascending
+ *     k_out,v_out bf16  [n_layers][G][B + w][d]
+ *     meta_out    u32   [n_layers][B + w]
+ *     stats       f32   [n_layers][STARKV_STATS_STRIDE(G)]
+ *   Token metadata word: bit 31 = visual, bits 20..30 = frame id f(t),
+ *   bits 10..19 = patch row r_t, bits 0..9 = patch column c_t (Sec. 3.1).
+ *   Text tokens only need bit 31 clear.
+ * - Errors: a call that returns non-OK has launched nothing unless the code is
+ *   STARKV_ERR_CUDA (a launch or copy failed part-way).  Invalid arguments are
+ *   caught on the host before any launch.  Device-side checks (metadata out of
+ *   range, a bounded wait that ran out) latch a code in the state's device
+ *   error word, which starkv_check_device_error reads.  starkv_last_error
+ *   returns a thread-local message for the last non-OK status.
+ * - Supported shapes: d = 128; w >= 1; H % G == 0; (H / G) * w <= 256;
+ *   G <= 8; L >= w (L_p = L - w >= 0; L_p = 0 keeps only the window);
+ *   0 <= B <= L_p; L < 2^24; 1 <= R, C <= 1024; R * C <= 16384;
+ *   2 <= mi_bins <= 16; mi_bins * mi_grid^2 <= 4096; odd pool_kernel <= 31;
+ *   frame ids 0..2047.  Other shapes return STARKV_ERR_UNSUPPORTED.
+ *   k, v, q, k_out and v_out must be 16-byte aligned.
+ */
+#ifndef STARKV_H
+#define STARKV_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  STARKV_OK = 0,
+  STARKV_ERR_INVALID_ARG = 1,  /* a pointer, size or index is invalid          */
+  STARKV_ERR_UNSUPPORTED = 2,  /* valid but outside the supported shapes       */
+  STARKV_ERR_CUDA = 3,         /* a CUDA runtime call failed                   */
+  STARKV_ERR_TIMEOUT = 4,      /* a bounded device-side wait ran out           */
+  STARKV_ERR_NOMEM = 5,        /* state allocation failed                      */
+  STARKV_ERR_DEVICE = 6        /* a device-side input check failed             */
+} starkv_status;
+
+/* Hyper-parameters.  starkv_default_config fills the paper's defaults
+ * (App. A.1, Table 7 AgentNetBench / UI-TARS) and this library's readings of
+ * the values the paper leaves open (pool_kernel, mi_bins, mi_grid, eps, eps_h). */
+typedef struct {
+  int32_t n_layers;
+  int32_t n_heads;      /* H query heads                                           */
+  int32_t n_kv_heads;   /* G KV groups ("subspaces", Sec. 3.1)                     */
+  int32_t head_dim;     /* d, must be 128                                          */
+  int32_t window;       /* w: observation window = recent window W_rec (Sec. 3.1)  */
+  int32_t grid_rows;    /* R: patch rows of one screenshot                         */
+  int32_t grid_cols;    /* C: patch columns of one screenshot                      */
+  int32_t pool_kernel;  /* AvgPool1D kernel (odd), stride 1, zero padding (Sec 3.3)*/
+  int32_t mi_bins;      /* K equal-frequency rank bins (Sec. 3.4)                  */
+  int32_t mi_grid;      /* M: SpatialBin grid is M x M (Sec. 3.4)                  */
+  int32_t n_warmup;     /* lambda is 0 for the first n_warmup steps (App. A.1)     */
+  int32_t n_ramp;       /* then ramps linearly to lambda over n_ramp steps         */
+  int32_t max_seqs;     /* number of state slots (independent trajectories)        */
+  float lambda;         /* MI prior strength (Eq. final_score)                     */
+  float tau;            /* prior softmax temperature (Eq. 7)                       */
+  float rho_mi;         /* MI EMA decay (Eq. 6)                                    */
+  float rho_t;          /* temporal EMA decay (Eq. 8)                              */
+  float delta;          /* temporal decay rate (Eq. 9)                             */
+  float d_min;          /* minimum temporal factor D_min (Eq. 9)                   */
+  float t_min, t_max;   /* AEB temperature range (Sec. 3.6)                        */
+  float eps;            /* epsilon of the min-max prior (Eq. 7)                    */
+  float eps_h;          /* epsilon of the AEB entropy (Algorithm 1)                */
+} starkv_config;
+
+/* One sequence (trajectory) of a batch: inputs and caller-owned outputs.  For
+ * per-layer calls (score_layer / select / compact) the `layer` argument picks
+ * the [layer] slice of every [n_layers][...] buffer below. */
+typedef struct {
+  const void* k;                /* bf16 [n_layers][G][L][d]                         */
+  const void* v;                /* bf16 [n_layers][G][L][d]                         */
+  const void* q;                /* bf16 [n_layers][H][w][d]                         */
+  const uint32_t* meta;         /* u32  [n_layers][L] (or [L] if stride is 0)       */
+  int64_t meta_layer_stride;    /* elements between layers of meta: 0 or >= L       */
+  int32_t L;                    /* cache length, including the w recent tokens      */
+  int32_t cur_frame;            /* F: frame id of the current (newest) screenshot   */
+  int32_t budget;               /* B: kept historical tokens, 0 <= B <= L - w       */
+  int32_t slot;                 /* state slot in [0, max_seqs)                      */
+  void* k_out;                  /* bf16 [n_layers][G][B + w][d]       (compact)    */
+  void* v_out;                  /* bf16 [n_layers][G][B + w][d]       (compact)    */
+  uint32_t* meta_out;           /* u32  [n_layers][B + w]             (compact)    */
+  int32_t* idx;                 /* i32  [n_layers][B]      select writes, compact reads */
+  float* S;                     /* f32  [n_layers][G][L_p] score_layer writes, select
+                                   reads; may be NULL for starkv_step (workspace)   */
+  float* score;                 /* f32  [n_layers][L_p] fused s_t, optional (NULL)  */
+  float* stats;                 /* f32  [n_layers][STARKV_STATS_STRIDE(G)], optional */
+} starkv_seq;
+
+/* Per-layer diagnostics written to starkv_seq.stats (floats):
+ *   [0] H_hat  [1] T  [2] lambda_n  [3] n (steps seen before this one)
+ *   [4] sum_t s_bar_t  [5] visual tokens in L_p  [6] kept count  [7] 0
+ *   [8 + g]       MI_g of this step            (Eq. 5)
+ *   [8 + G + g]   MI_bar_g after the EMA       (Eq. 6)
+ *   [8 + 2G + g]  w_g                          (Eq. 7)
+ *   [8 + 3G + g]  phi_g                        (Eq. 8)                         */
+#define STARKV_STATS_STRIDE(G) (8 + 4 * (G))
+
+typedef struct starkv_state starkv_state;
+
+/* Fills `cfg` with the defaults for the UI-TARS-1.5-7B GQA shape (H = 28,
+ * G = 4, d = 128, w = 32, 52 x 52 patches, 28 layers, 1 slot). */
+void starkv_default_config(starkv_config* cfg);
+
+/* Allocates the device-resident per-(slot, layer) state: step counter n, MI EMA
+ * MI_bar[G] (Eq. 6), temporal EMA m_g[R*C] per group (Eq. 8), all zero (fresh).
+ * The state lives on the current CUDA device; use it only there.
+ * Errors: INVALID_ARG / UNSUPPORTED for a bad config, NOMEM, CUDA. */
+starkv_status starkv_init_state(const starkv_config* cfg, starkv_state** out, void* stream);
+
+/* Trajectory-level reset of one slot (App. A.4: states are reset per
+ * trajectory): zeroes n, MI_bar and m_g of every layer, stream-ordered. */
+starkv_status starkv_reset_seq(starkv_state* st, int32_t slot, void* stream);
+
+/* Frees the state (synchronises the device first).  NULL is accepted. */
+starkv_status starkv_destroy_state(starkv_state* st);
+
+/* Copies the config the state was created with. */
+starkv_status starkv_get_config(const starkv_state* st, starkv_config* out);
+
+/* Bytes of device workspace that starkv_score_layer, starkv_select,
+ * starkv_compact and starkv_step need for this batch (the maximum of the four).
+ * With host != 0: the bytes starkv_step_host needs (adds staging copies). */
+starkv_status starkv_workspace_bytes(const starkv_state* st, const starkv_seq* seqs, int32_t nseq,
+                                     int32_t host, size_t* bytes);
+
+/* Sec. 3.3, Eqs. (2)-(4) (Algorithm 1, first two steps): for layer `layer` of
+ * every sequence, writes S[g][t] = (G/H) * sum_{h in g} AvgPool1D(
+ * sum_{i<w} softmax_t(Q_{-i,h} K_past[g]^T / sqrt(d)))[t]  for t < L_p,
+ * softmax over K_past only.  Reads k, q; writes S.  Uses tcgen05 tensor cores
+ * (bf16 in, fp32 accumulate) in two passes (log-sum-exp, then normalised sums). */
+starkv_status starkv_score_layer(starkv_state* st, int32_t layer, const starkv_seq* seqs,
+                                 int32_t nseq, void* workspace, size_t workspace_bytes,
+                                 void* stream);
+
+/* Sec. 3.3 - 3.7 after the group score map (Algorithm 1 from s_bar to I): from
+ * S of layer `layer`: s_bar, g*, online MI per group (Eq. 5) -> EMA (Eq. 6) ->
+ * prior w (Eq. 7) -> beta; phi_g and the m_g update (Eq. 8) -> D_t (Eq. 9);
+ * H_hat and T (Sec. 3.6); s_t = max(s_bar beta D, 0)^(1/T); global top-B with
+ * ties to the lower index -> idx ascending.  Writes idx, and score / stats when
+ * non-NULL.  Advances this layer's state by one step (n += 1 and both EMAs). */
+starkv_status starkv_select(starkv_state* st, int32_t layer, const starkv_seq* seqs,
+                            int32_t nseq, void* workspace, size_t workspace_bytes, void* stream);
+
+/* Sec. 3.7, Eq. (11): K' = [K_past[I]; K_rec], V' = [V_past[I]; V_rec] and the
+ * same gather of meta, for layer `layer`, from idx.  Bit copies. */
+starkv_status starkv_compact(starkv_state* st, int32_t layer, const starkv_seq* seqs,
+                             int32_t nseq, void* workspace, size_t workspace_bytes, void* stream);
+
+/* Whole compression step of every layer of every sequence (Algorithm 1 for all
+ * layers): score, select, compact.  S may be NULL (workspace is used).
+ * Equivalent to calling the three per-layer calls for each layer in order. */
+starkv_status starkv_step(starkv_state* st, const starkv_seq* seqs, int32_t nseq,
+                          void* workspace, size_t workspace_bytes, void* stream);
+
+/* starkv_step with every pointer in `seqs` a HOST pointer (page-locked memory
+ * gives asynchronous copies): copies k, v, q, meta to device staging inside
+ * `workspace` (size from starkv_workspace_bytes(..., host = 1, ...)), runs the
+ * step, and copies k_out, v_out, meta_out, idx (and score / stats / S when
+ * non-NULL) back.  Stream-ordered: the host outputs are valid after the stream
+ * is synchronised. */
+starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t nseq,
+                               void* workspace, size_t workspace_bytes, void* stream);
+
+/* Reads and clears the state's device error word (synchronises `stream`).
+ * Returns STARKV_OK, STARKV_ERR_DEVICE or STARKV_ERR_TIMEOUT. */
+starkv_status starkv_check_device_error(starkv_state* st, void* stream);
+
+/* Limit, in nanoseconds, of every bounded device-side wait of this state's
+ * kernels (default 1e9).  A wait that runs out stops its kernel early and
+ * latches STARKV_ERR_TIMEOUT in the device error word.  A debugging and test
+ * knob: 0 makes the first wait that does not succeed at once run out. */
+starkv_status starkv_set_wait_limit(starkv_state* st, uint64_t limit_ns);
+
+/* Thread-local message describing the last non-OK status on this thread. */
+const char* starkv_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* STARKV_H */

@@ -1,0 +1,600 @@
+// C ABI of the STaR-KV compression stage (include/starkv.h): argument
+// validation, device state, workspace planning, TMA descriptors and launch
+// sequencing.  All arithmetic of the method runs in the kernels of score.cu,
+// select.cu and compact.cu.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "compact.cuh"
+#include "score.cuh"
+#include "select.cuh"
+
+using namespace starkv;
+
+struct starkv_state {
+  starkv_config cfg;
+  DevState dev;
+  void* mem = nullptr;
+  size_t mem_bytes = 0;
+  int device = 0;
+  int num_sms = 0;
+  uint64_t wait_ns = 1000000000ull;
+};
+
+namespace {
+
+thread_local std::string g_last_error;
+
+starkv_status set_error(starkv_status s, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+starkv_status set_error(starkv_status s, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return s;
+}
+
+#define CUDA_TRY(expr)                                                                        \
+  do {                                                                                        \
+    cudaError_t e_ = (expr);                                                                  \
+    if (e_ != cudaSuccess)                                                                    \
+      return set_error(STARKV_ERR_CUDA, "%s failed: %s", #expr, cudaGetErrorString(e_));      \
+  } while (0)
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+cudaError_t g_encode_err = cudaSuccess;
+
+starkv_status get_encoder() {
+  std::call_once(g_encode_once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    g_encode_err = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                    cudaEnableDefault, &q);
+    if (g_encode_err == cudaSuccess && q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  if (!g_encode)
+    return set_error(STARKV_ERR_CUDA, "cuTensorMapEncodeTiled unavailable (%s)",
+                     cudaGetErrorString(g_encode_err));
+  return STARKV_OK;
+}
+
+// 3-D bf16 tensor map, 128-byte swizzle, box (64, box_rows, 1), zero fill out of bounds.
+starkv_status encode_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_t d1, uint64_t d2,
+                        uint32_t box_rows) {
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {d0 * 2, d0 * d1 * 2};
+  cuuint32_t box[3] = {64, box_rows, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  CUresult r = g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+                        box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return set_error(STARKV_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+  return STARKV_OK;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+starkv_status validate_config(const starkv_config& c) {
+  if (c.n_layers < 1 || c.n_heads < 1 || c.n_kv_heads < 1 || c.window < 1 || c.max_seqs < 1)
+    return set_error(STARKV_ERR_INVALID_ARG, "config: n_layers, n_heads, n_kv_heads, window, max_seqs must be >= 1");
+  if (c.head_dim != kHeadDim) return set_error(STARKV_ERR_UNSUPPORTED, "config: head_dim must be 128");
+  if (c.n_heads % c.n_kv_heads) return set_error(STARKV_ERR_UNSUPPORTED, "config: n_heads %% n_kv_heads != 0");
+  if (c.n_kv_heads > kMaxGroups) return set_error(STARKV_ERR_UNSUPPORTED, "config: n_kv_heads > 8");
+  if ((c.n_heads / c.n_kv_heads) * c.window > kMaxRows)
+    return set_error(STARKV_ERR_UNSUPPORTED, "config: (H/G)*w > 256");
+  if (c.grid_rows < 1 || c.grid_cols < 1 || c.grid_rows > 1024 || c.grid_cols > 1024 ||
+      c.grid_rows * c.grid_cols > kMaxGrid)
+    return set_error(STARKV_ERR_UNSUPPORTED, "config: patch grid out of range");
+  if (c.pool_kernel < 1 || c.pool_kernel > 31 || c.pool_kernel % 2 == 0)
+    return set_error(STARKV_ERR_UNSUPPORTED, "config: pool_kernel must be odd, 1..31");
+  if (c.mi_bins < 2 || c.mi_bins > 16 || c.mi_grid < 1 || c.mi_bins * c.mi_grid * c.mi_grid > kMaxHist)
+    return set_error(STARKV_ERR_UNSUPPORTED, "config: mi_bins / mi_grid out of range");
+  if (c.n_warmup < 0 || c.n_ramp < 0) return set_error(STARKV_ERR_INVALID_ARG, "config: negative schedule");
+  if (!(c.t_min > 0.f) || !(c.t_max > 0.f) || !(c.tau > 0.f))
+    return set_error(STARKV_ERR_INVALID_ARG, "config: t_min, t_max and tau must be > 0");
+  if (!(c.rho_mi >= 0.f && c.rho_mi <= 1.f) || !(c.rho_t >= 0.f && c.rho_t <= 1.f) ||
+      !(c.d_min >= 0.f && c.d_min <= 1.f) || !(c.eps >= 0.f) || !(c.eps_h >= 0.f) || !(c.delta >= 0.f))
+    return set_error(STARKV_ERR_INVALID_ARG, "config: a rate or epsilon is out of range");
+  return STARKV_OK;
+}
+
+enum Need : unsigned {
+  kNeedK = 1, kNeedQ = 2, kNeedV = 4, kNeedMeta = 8, kNeedS = 16, kNeedIdx = 32, kNeedOut = 64
+};
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+starkv_status validate_seqs(const starkv_state* st, const starkv_seq* seqs, int nseq, unsigned need) {
+  if (!st) return set_error(STARKV_ERR_INVALID_ARG, "state is NULL");
+  if (nseq < 0 || (nseq > 0 && !seqs)) return set_error(STARKV_ERR_INVALID_ARG, "bad sequence array");
+  const starkv_config& c = st->cfg;
+  std::vector<char> used(c.max_seqs, 0);
+  for (int i = 0; i < nseq; ++i) {
+    const starkv_seq& s = seqs[i];
+    if (s.slot < 0 || s.slot >= c.max_seqs) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: slot out of range", i);
+    if (used[s.slot]) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: slot %d used twice in one call", i, s.slot);
+    used[s.slot] = 1;
+    if (s.L < c.window) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: L < window", i);
+    if (s.L >= (1 << 24)) return set_error(STARKV_ERR_UNSUPPORTED, "seq %d: L >= 2^24", i);
+    const int lp = s.L - c.window;
+    if (s.budget < 0 || s.budget > lp) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: budget outside [0, L - w]", i);
+    if (s.cur_frame < 0 || s.cur_frame > 2047) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: cur_frame outside [0, 2047]", i);
+    if ((need & kNeedK) && (!s.k || !aligned16(s.k))) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: k NULL or not 16-byte aligned", i);
+    if ((need & kNeedQ) && (!s.q || !aligned16(s.q))) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: q NULL or not 16-byte aligned", i);
+    if ((need & kNeedV) && (!s.v || !aligned16(s.v))) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: v NULL or not 16-byte aligned", i);
+    if (need & kNeedMeta) {
+      if (!s.meta) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: meta is NULL", i);
+      if (s.meta_layer_stride != 0 && s.meta_layer_stride < s.L)
+        return set_error(STARKV_ERR_INVALID_ARG, "seq %d: meta_layer_stride must be 0 or >= L", i);
+    }
+    if ((need & kNeedS) && !s.S && lp > 0) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: S is NULL", i);
+    if ((need & kNeedIdx) && !s.idx && s.budget > 0) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: idx is NULL", i);
+    if (need & kNeedOut) {
+      if (!s.k_out || !s.v_out || !s.meta_out || !aligned16(s.k_out) || !aligned16(s.v_out))
+        return set_error(STARKV_ERR_INVALID_ARG, "seq %d: k_out / v_out / meta_out NULL or misaligned", i);
+    }
+  }
+  return STARKV_OK;
+}
+
+KParams make_kparams(const starkv_state* st) {
+  const starkv_config& c = st->cfg;
+  KParams k;
+  k.n_layers = c.n_layers; k.H = c.n_heads; k.G = c.n_kv_heads; k.w = c.window;
+  k.R = c.grid_rows; k.C = c.grid_cols; k.pool = c.pool_kernel; k.K = c.mi_bins; k.M = c.mi_grid;
+  k.n_warmup = c.n_warmup; k.n_ramp = c.n_ramp;
+  k.lambda = c.lambda; k.tau = c.tau; k.rho_mi = c.rho_mi; k.rho_t = c.rho_t; k.delta = c.delta;
+  k.d_min = c.d_min; k.t_min = c.t_min; k.t_max = c.t_max; k.eps = c.eps; k.eps_h = c.eps_h;
+  k.wait_ns = st->wait_ns;
+  return k;
+}
+
+// Workspace regions of one call over layers [layer0, layer0 + nlayers).
+struct WsPlan {
+  size_t partials = 0, s_raw = 0, total = 0;
+  std::vector<size_t> raw_off, S_off, score_off;  // per seq, SIZE_MAX = not in workspace
+};
+
+int tiles_of(int lp) { return (lp + kTileKeys - 1) / kTileKeys; }
+
+void plan_ws(const starkv_state* st, const starkv_seq* seqs, int nseq, int nlayers, bool ws_S,
+             bool ws_score, WsPlan* p) {
+  const starkv_config& c = st->cfg;
+  const int G = c.n_kv_heads;
+  size_t off = 0;
+  size_t tiles = 0;
+  for (int i = 0; i < nseq; ++i) tiles += static_cast<size_t>(nlayers) * G * tiles_of(seqs[i].L - c.window);
+  p->partials = off;
+  off += align256(tiles * kMaxRows * sizeof(float2));
+  p->raw_off.assign(nseq, SIZE_MAX);
+  p->S_off.assign(nseq, SIZE_MAX);
+  p->score_off.assign(nseq, SIZE_MAX);
+  for (int i = 0; i < nseq; ++i) {
+    const size_t lp = seqs[i].L - c.window;
+    p->raw_off[i] = off;
+    off += align256(static_cast<size_t>(nlayers) * G * lp * sizeof(float));
+    if (ws_S && !seqs[i].S) {
+      p->S_off[i] = off;
+      off += align256(static_cast<size_t>(c.n_layers) * G * lp * sizeof(float));
+    }
+    if (ws_score && !seqs[i].score) {
+      p->score_off[i] = off;
+      off += align256(static_cast<size_t>(c.n_layers) * lp * sizeof(float));
+    }
+  }
+  p->total = std::max<size_t>(off, 256);
+}
+
+SeqView make_view(const starkv_state* st, const starkv_seq& s, char* ws, const WsPlan& plan, int i) {
+  const starkv_config& c = st->cfg;
+  SeqView v;
+  v.k = static_cast<const __nv_bfloat16*>(s.k);
+  v.v = static_cast<const __nv_bfloat16*>(s.v);
+  v.meta = s.meta;
+  v.meta_layer_stride = s.meta_layer_stride;
+  v.L = s.L;
+  v.Lp = s.L - c.window;
+  v.cur_frame = s.cur_frame;
+  v.budget = s.budget;
+  v.slot = s.slot;
+  v.pad_ = 0;
+  v.k_out = static_cast<__nv_bfloat16*>(s.k_out);
+  v.v_out = static_cast<__nv_bfloat16*>(s.v_out);
+  v.meta_out = s.meta_out;
+  v.idx = s.idx;
+  v.S = plan.S_off[i] != SIZE_MAX ? reinterpret_cast<float*>(ws + plan.S_off[i]) : s.S;
+  v.s_raw = reinterpret_cast<float*>(ws + plan.raw_off[i]);
+  v.score = plan.score_off[i] != SIZE_MAX ? reinterpret_cast<float*>(ws + plan.score_off[i]) : s.score;
+  v.stats = s.stats;
+  return v;
+}
+
+// Both scoring passes for sequences [i0, i1) over layers [layer0, layer0 + nlayers).
+starkv_status run_score(starkv_state* st, const starkv_seq* seqs, int i0, int i1, int layer0, int nlayers,
+                        char* ws, const WsPlan& plan, size_t* partial_cursor, cudaStream_t stream) {
+  const starkv_config& c = st->cfg;
+  const int G = c.n_kv_heads, H = c.n_heads, w = c.window;
+  starkv_status s = get_encoder();
+  if (s != STARKV_OK) return s;
+  static thread_local ScoreParams p;   // ~13 KB: kept off the stack
+  memset(&p, 0, sizeof(p));
+  p.nseq = i1 - i0;
+  p.layer0 = layer0;
+  p.nlayers = nlayers;
+  p.G = G;
+  p.rows = (H / G) * w;
+  p.n2 = (p.rows + 15) & ~15;
+  p.n_mtiles = (p.rows + kTileKeys - 1) / kTileKeys;
+  p.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(kHeadDim)));
+  int64_t tiles = 0;
+  for (int i = i0; i < i1; ++i) {
+    const starkv_seq& q = seqs[i];
+    const int lp = q.L - w;
+    ScoreSeq& ss = p.seq[i - i0];
+    ss.Lp = lp;
+    ss.nt = tiles_of(lp);
+    ss.tile_base = tiles;
+    ss.s_raw = reinterpret_cast<float*>(ws + plan.raw_off[i]);
+    tiles += static_cast<int64_t>(nlayers) * G * ss.nt;
+    if (ss.nt == 0) continue;
+    if ((s = encode_3d(&p.tmk[i - i0], q.k, kHeadDim, q.L, static_cast<uint64_t>(c.n_layers) * G, kTileKeys)) != STARKV_OK) return s;
+    if ((s = encode_3d(&p.tmq1[i - i0], q.q, kHeadDim, static_cast<uint64_t>(H) * w, c.n_layers, kTileKeys)) != STARKV_OK) return s;
+    if ((s = encode_3d(&p.tmq2[i - i0], q.q, kHeadDim, static_cast<uint64_t>(H) * w, c.n_layers, p.n2)) != STARKV_OK) return s;
+  }
+  if (tiles == 0) return STARKV_OK;
+  p.total_tiles = tiles;
+  p.grid1 = static_cast<int>(std::min<int64_t>(tiles, st->num_sms));
+  p.partials = reinterpret_cast<float2*>(ws + plan.partials) + *partial_cursor * kMaxRows;
+  *partial_cursor += tiles;
+  p.err = st->dev.err;
+  p.wait_ns = st->wait_ns;
+  CUDA_TRY(score_launch(p, p.grid1, stream));
+  return STARKV_OK;
+}
+
+SeqBatch make_batch(const starkv_state* st, const starkv_seq* seqs, int i0, int i1, int layer0, int nlayers,
+                    char* ws, const WsPlan& plan) {
+  SeqBatch b;
+  memset(&b, 0, sizeof(b));
+  b.nseq = i1 - i0;
+  b.layer0 = layer0;
+  b.nlayers = nlayers;
+  for (int i = i0; i < i1; ++i) b.s[i - i0] = make_view(st, seqs[i], ws, plan, i);
+  return b;
+}
+
+starkv_status check_ws(const starkv_state* st, void* ws, size_t bytes, size_t need) {
+  (void)st;
+  if (need > 0 && (!ws || bytes < need))
+    return set_error(STARKV_ERR_INVALID_ARG, "workspace too small: %zu bytes given, %zu needed", bytes, need);
+  if (reinterpret_cast<uintptr_t>(ws) & 255) return set_error(STARKV_ERR_INVALID_ARG, "workspace not 256-byte aligned");
+  return STARKV_OK;
+}
+
+starkv_status check_device(const starkv_state* st) {
+  int dev = -1;
+  CUDA_TRY(cudaGetDevice(&dev));
+  if (dev != st->device)
+    return set_error(STARKV_ERR_INVALID_ARG, "state lives on device %d, current device is %d", st->device, dev);
+  return STARKV_OK;
+}
+
+// Stages of the step (per-layer calls use a one-layer range).
+enum Stage : unsigned { kScore = 1, kPool = 2, kStatsRaw = 4, kStatsPooled = 8, kSelect = 16, kCompact = 32 };
+
+starkv_status run_stages(starkv_state* st, const starkv_seq* seqs, int nseq, int layer0, int nlayers,
+                         unsigned stages, void* workspace, size_t ws_bytes, cudaStream_t stream) {
+  const starkv_config& c = st->cfg;
+  WsPlan plan;
+  const bool ws_S = (stages & kStatsRaw) != 0;
+  plan_ws(st, seqs, nseq, nlayers, ws_S, true, &plan);
+  starkv_status s = check_ws(st, workspace, ws_bytes, plan.total);
+  if (s != STARKV_OK) return s;
+  char* ws = static_cast<char*>(workspace);
+  const KParams kp = make_kparams(st);
+  size_t partial_cursor = 0;
+  for (int i0 = 0; i0 < nseq; i0 += kMaxBatch) {
+    const int i1 = std::min(nseq, i0 + kMaxBatch);
+    int lp_max = 0, rows_out_max = 0;
+    for (int i = i0; i < i1; ++i) {
+      lp_max = std::max(lp_max, seqs[i].L - c.window);
+      rows_out_max = std::max(rows_out_max, seqs[i].budget + c.window);
+    }
+    const SeqBatch b = make_batch(st, seqs, i0, i1, layer0, nlayers, ws, plan);
+    if (stages & kScore) {
+      s = run_score(st, seqs, i0, i1, layer0, nlayers, ws, plan, &partial_cursor, stream);
+      if (s != STARKV_OK) return s;
+    }
+    if (stages & kPool) CUDA_TRY(pool_launch(b, c.n_kv_heads, c.n_heads, c.pool_kernel, lp_max, stream));
+    if (stages & (kStatsRaw | kStatsPooled))
+      CUDA_TRY(group_stats_launch(b, kp, st->dev, (stages & kStatsRaw) != 0, stream));
+    if (stages & kSelect) CUDA_TRY(select_launch(b, kp, st->dev, stream));
+    if (stages & kCompact) CUDA_TRY(compact_launch(b, c.n_kv_heads, c.window, rows_out_max, st->num_sms, st->dev.err, stream));
+  }
+  return STARKV_OK;
+}
+
+size_t seq_bytes_in(const starkv_config& c, const starkv_seq& s) {
+  const size_t kv = static_cast<size_t>(c.n_layers) * c.n_kv_heads * s.L * kHeadDim * 2;
+  const size_t q = static_cast<size_t>(c.n_layers) * c.n_heads * c.window * kHeadDim * 2;
+  const size_t meta = (s.meta_layer_stride ? static_cast<size_t>(c.n_layers) * s.meta_layer_stride : s.L) * 4;
+  return align256(kv) * 2 + align256(q) + align256(meta);
+}
+
+size_t seq_bytes_out(const starkv_config& c, const starkv_seq& s) {
+  const size_t ro = s.budget + c.window, lp = s.L - c.window;
+  size_t b = align256(static_cast<size_t>(c.n_layers) * c.n_kv_heads * ro * kHeadDim * 2) * 2;
+  b += align256(static_cast<size_t>(c.n_layers) * ro * 4);
+  b += align256(static_cast<size_t>(c.n_layers) * s.budget * 4);
+  if (s.S) b += align256(static_cast<size_t>(c.n_layers) * c.n_kv_heads * lp * 4);
+  if (s.score) b += align256(static_cast<size_t>(c.n_layers) * lp * 4);
+  if (s.stats) b += align256(static_cast<size_t>(c.n_layers) * (8 + 4 * c.n_kv_heads) * 4);
+  return b;
+}
+
+}  // namespace
+
+extern "C" {
+
+void starkv_default_config(starkv_config* c) {
+  if (!c) return;
+  memset(c, 0, sizeof(*c));
+  c->n_layers = 28;
+  c->n_heads = 28;
+  c->n_kv_heads = 4;
+  c->head_dim = 128;
+  c->window = 32;
+  c->grid_rows = 52;
+  c->grid_cols = 52;
+  c->pool_kernel = 5;
+  c->mi_bins = 8;
+  c->mi_grid = 8;
+  c->n_warmup = 5;
+  c->n_ramp = 10;
+  c->max_seqs = 1;
+  c->lambda = 0.5f;
+  c->tau = 1.0f;
+  c->rho_mi = 0.9f;
+  c->rho_t = 0.9f;
+  c->delta = 0.2f;
+  c->d_min = 0.1f;
+  c->t_min = 0.95f;
+  c->t_max = 1.05f;
+  c->eps = 1e-6f;
+  c->eps_h = 1e-12f;
+}
+
+starkv_status starkv_init_state(const starkv_config* cfg, starkv_state** out, void* stream) {
+  if (!cfg || !out) return set_error(STARKV_ERR_INVALID_ARG, "NULL config or output pointer");
+  *out = nullptr;
+  starkv_status s = validate_config(*cfg);
+  if (s != STARKV_OK) return s;
+  starkv_state* st = new (std::nothrow) starkv_state();
+  if (!st) return set_error(STARKV_ERR_NOMEM, "host allocation failed");
+  st->cfg = *cfg;
+  cudaError_t e = cudaGetDevice(&st->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&st->num_sms, cudaDevAttrMultiProcessorCount, st->device);
+  if (e == cudaSuccess) e = score_configure();
+  if (e == cudaSuccess) e = select_configure();
+  if (e != cudaSuccess) {
+    delete st;
+    return set_error(STARKV_ERR_CUDA, "device setup failed: %s", cudaGetErrorString(e));
+  }
+  const size_t SL = static_cast<size_t>(cfg->max_seqs) * cfg->n_layers;
+  const size_t G = cfg->n_kv_heads, RC = static_cast<size_t>(cfg->grid_rows) * cfg->grid_cols;
+  const size_t o_n = 0;
+  const size_t o_mibar = o_n + align256(SL * sizeof(int32_t));
+  const size_t o_micur = o_mibar + align256(SL * G * sizeof(double));
+  const size_t o_phi = o_micur + align256(SL * G * sizeof(double));
+  const size_t o_m = o_phi + align256(SL * G * sizeof(float));
+  const size_t o_err = o_m + align256(SL * G * RC * sizeof(float));
+  st->mem_bytes = o_err + 256;
+  e = cudaMalloc(&st->mem, st->mem_bytes);
+  if (e != cudaSuccess) {
+    delete st;
+    return set_error(STARKV_ERR_NOMEM, "state allocation of %zu bytes failed: %s", st->mem_bytes, cudaGetErrorString(e));
+  }
+  char* m = static_cast<char*>(st->mem);
+  st->dev.n = reinterpret_cast<int32_t*>(m + o_n);
+  st->dev.mi_bar = reinterpret_cast<double*>(m + o_mibar);
+  st->dev.mi_cur = reinterpret_cast<double*>(m + o_micur);
+  st->dev.phi_cur = reinterpret_cast<float*>(m + o_phi);
+  st->dev.m = reinterpret_cast<float*>(m + o_m);
+  st->dev.err = reinterpret_cast<uint32_t*>(m + o_err);
+  e = cudaMemsetAsync(st->mem, 0, st->mem_bytes, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) {
+    cudaFree(st->mem);
+    delete st;
+    return set_error(STARKV_ERR_CUDA, "state clear failed: %s", cudaGetErrorString(e));
+  }
+  *out = st;
+  return STARKV_OK;
+}
+
+starkv_status starkv_reset_seq(starkv_state* st, int32_t slot, void* stream) {
+  if (!st) return set_error(STARKV_ERR_INVALID_ARG, "state is NULL");
+  const starkv_config& c = st->cfg;
+  if (slot < 0 || slot >= c.max_seqs) return set_error(STARKV_ERR_INVALID_ARG, "slot out of range");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  const size_t L = c.n_layers, G = c.n_kv_heads, RC = static_cast<size_t>(c.grid_rows) * c.grid_cols;
+  CUDA_TRY(cudaMemsetAsync(st->dev.n + slot * L, 0, L * sizeof(int32_t), s));
+  CUDA_TRY(cudaMemsetAsync(st->dev.mi_bar + slot * L * G, 0, L * G * sizeof(double), s));
+  CUDA_TRY(cudaMemsetAsync(st->dev.m + slot * L * G * RC, 0, L * G * RC * sizeof(float), s));
+  return STARKV_OK;
+}
+
+starkv_status starkv_destroy_state(starkv_state* st) {
+  if (!st) return STARKV_OK;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e == cudaSuccess) e = cudaFree(st->mem);
+  delete st;
+  if (e != cudaSuccess) return set_error(STARKV_ERR_CUDA, "destroy failed: %s", cudaGetErrorString(e));
+  return STARKV_OK;
+}
+
+starkv_status starkv_get_config(const starkv_state* st, starkv_config* out) {
+  if (!st || !out) return set_error(STARKV_ERR_INVALID_ARG, "NULL argument");
+  *out = st->cfg;
+  return STARKV_OK;
+}
+
+starkv_status starkv_set_wait_limit(starkv_state* st, uint64_t limit_ns) {
+  if (!st) return set_error(STARKV_ERR_INVALID_ARG, "state is NULL");
+  st->wait_ns = limit_ns;
+  return STARKV_OK;
+}
+
+starkv_status starkv_workspace_bytes(const starkv_state* st, const starkv_seq* seqs, int32_t nseq, int32_t host,
+                                     size_t* bytes) {
+  if (!bytes) return set_error(STARKV_ERR_INVALID_ARG, "bytes is NULL");
+  starkv_status s = validate_seqs(st, seqs, nseq, 0);
+  if (s != STARKV_OK) return s;
+  WsPlan a, b;
+  plan_ws(st, seqs, nseq, st->cfg.n_layers, true, true, &a);
+  plan_ws(st, seqs, nseq, 1, false, true, &b);
+  size_t total = std::max(a.total, b.total);
+  if (host) {
+    std::vector<starkv_seq> dev(seqs, seqs + nseq);
+    size_t staged = 0;
+    for (int i = 0; i < nseq; ++i) {
+      staged += seq_bytes_in(st->cfg, seqs[i]) + seq_bytes_out(st->cfg, seqs[i]);
+      dev[i].S = nullptr;  // step keeps S in the workspace unless asked for it
+    }
+    WsPlan c;
+    plan_ws(st, dev.data(), nseq, st->cfg.n_layers, true, true, &c);
+    total = staged + c.total;
+  }
+  *bytes = total;
+  return STARKV_OK;
+}
+
+starkv_status starkv_score_layer(starkv_state* st, int32_t layer, const starkv_seq* seqs, int32_t nseq,
+                                 void* workspace, size_t workspace_bytes, void* stream) {
+  starkv_status s = validate_seqs(st, seqs, nseq, kNeedK | kNeedQ | kNeedS);
+  if (s != STARKV_OK) return s;
+  if (layer < 0 || layer >= st->cfg.n_layers) return set_error(STARKV_ERR_INVALID_ARG, "layer out of range");
+  if ((s = check_device(st)) != STARKV_OK) return s;
+  return run_stages(st, seqs, nseq, layer, 1, kScore | kPool, workspace, workspace_bytes,
+                    static_cast<cudaStream_t>(stream));
+}
+
+starkv_status starkv_select(starkv_state* st, int32_t layer, const starkv_seq* seqs, int32_t nseq,
+                            void* workspace, size_t workspace_bytes, void* stream) {
+  starkv_status s = validate_seqs(st, seqs, nseq, kNeedMeta | kNeedS | kNeedIdx);
+  if (s != STARKV_OK) return s;
+  if (layer < 0 || layer >= st->cfg.n_layers) return set_error(STARKV_ERR_INVALID_ARG, "layer out of range");
+  if ((s = check_device(st)) != STARKV_OK) return s;
+  return run_stages(st, seqs, nseq, layer, 1, kStatsPooled | kSelect, workspace, workspace_bytes,
+                    static_cast<cudaStream_t>(stream));
+}
+
+starkv_status starkv_compact(starkv_state* st, int32_t layer, const starkv_seq* seqs, int32_t nseq,
+                             void* workspace, size_t workspace_bytes, void* stream) {
+  starkv_status s = validate_seqs(st, seqs, nseq, kNeedK | kNeedV | kNeedMeta | kNeedIdx | kNeedOut);
+  if (s != STARKV_OK) return s;
+  if (layer < 0 || layer >= st->cfg.n_layers) return set_error(STARKV_ERR_INVALID_ARG, "layer out of range");
+  if ((s = check_device(st)) != STARKV_OK) return s;
+  return run_stages(st, seqs, nseq, layer, 1, kCompact, workspace, workspace_bytes,
+                    static_cast<cudaStream_t>(stream));
+}
+
+starkv_status starkv_step(starkv_state* st, const starkv_seq* seqs, int32_t nseq, void* workspace,
+                          size_t workspace_bytes, void* stream) {
+  starkv_status s = validate_seqs(st, seqs, nseq, kNeedK | kNeedQ | kNeedV | kNeedMeta | kNeedIdx | kNeedOut);
+  if (s != STARKV_OK) return s;
+  if ((s = check_device(st)) != STARKV_OK) return s;
+  return run_stages(st, seqs, nseq, 0, st->cfg.n_layers, kScore | kStatsRaw | kSelect | kCompact, workspace,
+                    workspace_bytes, static_cast<cudaStream_t>(stream));
+}
+
+starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t nseq, void* workspace,
+                               size_t workspace_bytes, void* stream) {
+  starkv_status s = validate_seqs(st, seqs, nseq, kNeedK | kNeedQ | kNeedV | kNeedMeta | kNeedIdx | kNeedOut);
+  if (s != STARKV_OK) return s;
+  if ((s = check_device(st)) != STARKV_OK) return s;
+  size_t need = 0;
+  if ((s = starkv_workspace_bytes(st, seqs, nseq, 1, &need)) != STARKV_OK) return s;
+  if ((s = check_ws(st, workspace, workspace_bytes, need)) != STARKV_OK) return s;
+  const starkv_config& c = st->cfg;
+  cudaStream_t strm = static_cast<cudaStream_t>(stream);
+  char* cur = static_cast<char*>(workspace);
+  auto take = [&](size_t bytes) {
+    char* p = cur;
+    cur += align256(bytes);
+    return p;
+  };
+  std::vector<starkv_seq> dev(seqs, seqs + nseq);
+  for (int i = 0; i < nseq; ++i) {
+    const starkv_seq& h = seqs[i];
+    starkv_seq& d = dev[i];
+    const size_t kv = static_cast<size_t>(c.n_layers) * c.n_kv_heads * h.L * kHeadDim * 2;
+    const size_t qb = static_cast<size_t>(c.n_layers) * c.n_heads * c.window * kHeadDim * 2;
+    const size_t mb = (h.meta_layer_stride ? static_cast<size_t>(c.n_layers) * h.meta_layer_stride : h.L) * 4;
+    d.k = take(kv);
+    d.v = take(kv);
+    d.q = take(qb);
+    d.meta = reinterpret_cast<const uint32_t*>(take(mb));
+    CUDA_TRY(cudaMemcpyAsync(const_cast<void*>(d.k), h.k, kv, cudaMemcpyHostToDevice, strm));
+    CUDA_TRY(cudaMemcpyAsync(const_cast<void*>(d.v), h.v, kv, cudaMemcpyHostToDevice, strm));
+    CUDA_TRY(cudaMemcpyAsync(const_cast<void*>(d.q), h.q, qb, cudaMemcpyHostToDevice, strm));
+    CUDA_TRY(cudaMemcpyAsync(const_cast<uint32_t*>(d.meta), h.meta, mb, cudaMemcpyHostToDevice, strm));
+    const size_t ro = h.budget + c.window, lp = h.L - c.window;
+    d.k_out = take(static_cast<size_t>(c.n_layers) * c.n_kv_heads * ro * kHeadDim * 2);
+    d.v_out = take(static_cast<size_t>(c.n_layers) * c.n_kv_heads * ro * kHeadDim * 2);
+    d.meta_out = reinterpret_cast<uint32_t*>(take(static_cast<size_t>(c.n_layers) * ro * 4));
+    d.idx = reinterpret_cast<int32_t*>(take(static_cast<size_t>(c.n_layers) * h.budget * 4));
+    d.S = h.S ? reinterpret_cast<float*>(take(static_cast<size_t>(c.n_layers) * c.n_kv_heads * lp * 4)) : nullptr;
+    d.score = h.score ? reinterpret_cast<float*>(take(static_cast<size_t>(c.n_layers) * lp * 4)) : nullptr;
+    d.stats = h.stats ? reinterpret_cast<float*>(take(static_cast<size_t>(c.n_layers) * (8 + 4 * c.n_kv_heads) * 4)) : nullptr;
+  }
+  const size_t used = static_cast<size_t>(cur - static_cast<char*>(workspace));
+  s = starkv_step(st, dev.data(), nseq, cur, workspace_bytes - used, stream);
+  if (s != STARKV_OK) return s;
+  for (int i = 0; i < nseq; ++i) {
+    const starkv_seq& h = seqs[i];
+    const starkv_seq& d = dev[i];
+    const size_t ro = h.budget + c.window, lp = h.L - c.window;
+    CUDA_TRY(cudaMemcpyAsync(h.k_out, d.k_out, static_cast<size_t>(c.n_layers) * c.n_kv_heads * ro * kHeadDim * 2, cudaMemcpyDeviceToHost, strm));
+    CUDA_TRY(cudaMemcpyAsync(h.v_out, d.v_out, static_cast<size_t>(c.n_layers) * c.n_kv_heads * ro * kHeadDim * 2, cudaMemcpyDeviceToHost, strm));
+    CUDA_TRY(cudaMemcpyAsync(h.meta_out, d.meta_out, static_cast<size_t>(c.n_layers) * ro * 4, cudaMemcpyDeviceToHost, strm));
+    if (h.budget > 0)
+      CUDA_TRY(cudaMemcpyAsync(h.idx, d.idx, static_cast<size_t>(c.n_layers) * h.budget * 4, cudaMemcpyDeviceToHost, strm));
+    if (h.S && lp > 0)
+      CUDA_TRY(cudaMemcpyAsync(h.S, d.S, static_cast<size_t>(c.n_layers) * c.n_kv_heads * lp * 4, cudaMemcpyDeviceToHost, strm));
+    if (h.score && lp > 0)
+      CUDA_TRY(cudaMemcpyAsync(h.score, d.score, static_cast<size_t>(c.n_layers) * lp * 4, cudaMemcpyDeviceToHost, strm));
+    if (h.stats)
+      CUDA_TRY(cudaMemcpyAsync(h.stats, d.stats, static_cast<size_t>(c.n_layers) * (8 + 4 * c.n_kv_heads) * 4, cudaMemcpyDeviceToHost, strm));
+  }
+  return STARKV_OK;
+}
+
+starkv_status starkv_check_device_error(starkv_state* st, void* stream) {
+  if (!st) return set_error(STARKV_ERR_INVALID_ARG, "state is NULL");
+  uint32_t h = 0;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  CUDA_TRY(cudaMemcpyAsync(&h, st->dev.err, sizeof(h), cudaMemcpyDeviceToHost, s));
+  CUDA_TRY(cudaStreamSynchronize(s));
+  CUDA_TRY(cudaMemsetAsync(st->dev.err, 0, sizeof(uint32_t), s));
+  if (h & kErrTimeout) return set_error(STARKV_ERR_TIMEOUT, "a bounded device wait ran out");
+  if (h & kErrMeta) return set_error(STARKV_ERR_DEVICE, "token metadata outside the patch grid");
+  if (h & kErrIndex) return set_error(STARKV_ERR_DEVICE, "an index outside the cache reached the gather");
+  return STARKV_OK;
+}
+
+const char* starkv_last_error(void) { return g_last_error.c_str(); }
+
+}  // extern "C"

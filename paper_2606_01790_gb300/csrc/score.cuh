@@ -1,0 +1,39 @@
+// Launch interface of the scoring kernels (score.cu).
+#pragma once
+
+#include "common.cuh"
+
+namespace starkv {
+
+constexpr int kScoreThreads = 384;   // 12 warps: TMA, MMA, 2 idle, 8 epilogue
+
+struct ScoreSeq {
+  int Lp;              // scored (historical) keys
+  int nt;              // ceil(Lp / 128) key tiles per (layer, group) row
+  int64_t tile_base;   // flat index of this sequence's first tile in the launch
+  float* s_raw;        // [nlayers][G][Lp] unpooled group sums
+};
+
+struct ScoreParams {
+  CUtensorMap tmk[kMaxBatch];    // K: dims (d, L, n_layers*G), box (64, 128, 1), 128B swizzle
+  CUtensorMap tmq1[kMaxBatch];   // Q: dims (d, H*w, n_layers), box (64, 128, 1)
+  CUtensorMap tmq2[kMaxBatch];   // Q: dims (d, H*w, n_layers), box (64, n2, 1)
+  ScoreSeq seq[kMaxBatch];
+  int nseq, layer0, nlayers, G;
+  int rows;            // (H / G) * w window rows per group
+  int n2;              // rows rounded up to 16 (pass-2 MMA N)
+  int n_mtiles;        // ceil(rows / 128) (pass-1 M tiles)
+  int grid1;           // pass-1 grid size (defines the partial-slot partition)
+  int64_t total_tiles;
+  float scale2;        // log2(e) / sqrt(d)
+  float2* partials;    // [total_tiles][kMaxRows] (max2, sum) at each piece's first tile
+  uint32_t* err;
+  uint64_t wait_ns;
+};
+
+size_t score_smem_bytes();
+cudaError_t score_configure();
+cudaError_t score_launch(const ScoreParams& p, int grid, cudaStream_t stream);
+cudaError_t pool_launch(const SeqBatch& b, int G, int H, int pool, int lp_max, cudaStream_t stream);
+
+}  // namespace starkv

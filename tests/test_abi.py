@@ -1,0 +1,74 @@
+"""The C-ABI library loads and exports every entry point include/starkv.h
+declares; host-side checks that need no GPU.  CPU only."""
+import ctypes
+import re
+from pathlib import Path
+
+import pytest
+
+from paper_2606_01790_gb300 import build as B
+from paper_2606_01790_gb300 import starkv as sk
+
+ROOT = Path(__file__).resolve().parents[1]
+
+
+@pytest.fixture(scope="module")
+def library():
+    B.build()
+    return sk.lib()
+
+
+def declared_functions():
+    text = (ROOT / "include" / "starkv.h").read_text()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(starkv_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_expected_calls():
+    names = declared_functions()
+    for required in ("starkv_init_state", "starkv_score_layer", "starkv_select", "starkv_compact",
+                     "starkv_step"):
+        assert required in names
+    assert set(names) == set(sk.ABI_FUNCTIONS)
+
+
+def test_library_exports_every_declared_symbol(library):
+    for name in declared_functions():
+        assert hasattr(library, name), name
+        assert ctypes.cast(getattr(library, name), ctypes.c_void_p).value
+
+
+def test_struct_layouts_match_header():
+    assert ctypes.sizeof(sk.CConfig) == 13 * 4 + 10 * 4
+    assert ctypes.sizeof(sk.CSeq) == 4 * 8 + 8 + 4 * 4 + 7 * 8
+
+
+def test_default_config_matches_paper_defaults(library):
+    c = sk.Config.default()
+    assert (c.n_heads, c.n_kv_heads, c.head_dim, c.window) == (28, 4, 128, 32)
+    assert abs(c.lambda_ - 0.5) < 1e-7 and abs(c.delta - 0.2) < 1e-7 and abs(c.d_min - 0.1) < 1e-7
+    assert (c.n_warmup, c.n_ramp) == (5, 10)
+    assert abs(c.t_min - 0.95) < 1e-7 and abs(c.t_max - 1.05) < 1e-7
+
+
+@pytest.mark.parametrize("bad", [dict(head_dim=64), dict(n_heads=30), dict(window=64),
+                                 dict(pool_kernel=4), dict(mi_bins=1), dict(t_min=0.0),
+                                 dict(n_kv_heads=0), dict(grid_rows=2000)])
+def test_invalid_config_rejected_before_any_device_call(library, bad):
+    cfg = sk.Config(**bad)
+    with pytest.raises(sk.StarkvError) as e:
+        sk.State(cfg, stream=0)
+    assert e.value.status in (sk.ERR_INVALID_ARG, sk.ERR_UNSUPPORTED)
+
+
+def test_meta_packing_roundtrip():
+    import numpy as np
+    vis = np.array([0, 1, 1, 1]); fr = np.array([0, 3, 2047, 0])
+    row = np.array([0, 51, 1023, 7]); col = np.array([0, 0, 9, 1023])
+    w = sk.pack_meta(vis, fr, row, col)
+    assert w[0] == 0 and (w[1:] >> 31).tolist() == [1, 1, 1]
+    v2, f2, r2, c2 = sk.unpack_meta(w)
+    assert v2.tolist() == vis.tolist() and f2[1:].tolist() == fr[1:].tolist()
+    assert r2[1:].tolist() == row[1:].tolist() and c2[1:].tolist() == col[1:].tolist()
+    with pytest.raises(ValueError):
+        sk.pack_meta([1], [4096], [0], [0])
