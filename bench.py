@@ -1,0 +1,416 @@
+#!/usr/bin/env python3
+"""Benchmark of the STaR-KV compression step on GB300.
+
+One step = Algorithm 1 for every layer of the workload: window-query scoring
+(two tcgen05 passes), online MI / temporal / entropy calibration, global top-B
+and the KV gather, through the C ABI (``starkv_step``).  Default workload: 28
+layers of the 5-screenshot UI-TARS-1.5-7B shape (28 q heads / 4 KV heads,
+d = 128, w = 32, 5 x 2704 visual + 512 text tokens, B = 20% of visual).
+
+Prints ONE JSON line (rank 0).  ``value`` is cache tokens scored per second
+(sum over layers and sequences of L_past per step / step time), inputs resident
+in HBM; ``e2e`` is the same metric through ``starkv_step_host`` with pinned
+host buffers, copies inside the timed region.  ``--impl reference`` times the
+fp64 CPU oracle on the same workload instead.
+
+Multi-GPU (torchrun): each rank compresses its own independent trajectory
+(weak scaling, no collective on the data path); timing is max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+from pathlib import Path
+
+ROOT = Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+METRIC = "KV compression latency/step (ms) & cache tokens scored/s; % of HBM/TC roofline"
+UNIT = "tokens/s"
+
+
+def _peaks():
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        d = json.loads(p.read_text())
+        return dict(hbm=float(d["hbm_gbs"]), tc=float(d["bf16_tflops"]),
+                    tc_sus=float(d.get("bf16_tflops_sustained", d["bf16_tflops"])), src="measured")
+    return dict(hbm=6800.0, tc=1900.0, tc_sus=1700.0, src="fallback")
+
+
+# ----------------------------------------------------------------------------- work accounting
+
+def work_per_step(wl, seqs):
+    """Algorithmic bytes and flops of one step, per kernel kind and in total.
+
+    Per scored token and layer: K read once (G * d * 2 B) and 2 * H * w * d
+    flop of Q K^T; per (layer, seq): window queries H * w * d * 2 B; the group
+    score map written and read (2 * G * 4 B per token); per kept row: K and V
+    read and written (4 * G * d * 2 B)."""
+    H, G, w, d, nl = wl.n_heads, wl.n_kv_heads, wl.window, wl.head_dim, wl.n_layers
+    tok = sum(s["L"] - w for s in seqs) * nl
+    kept = sum(s["B"] + w for s in seqs) * nl
+    qk_flops = 2.0 * H * w * d * tok
+    k_bytes = G * d * 2.0 * tok + H * w * d * 2.0 * nl * len(seqs)
+    s_bytes = 2 * G * 4.0 * tok
+    gather = 4.0 * G * d * 2 * kept + 2 * 4.0 * kept
+    return dict(tokens=tok, qk_flops=qk_flops, k_bytes=k_bytes, s_bytes=s_bytes, gather_bytes=gather,
+                step_bytes=k_bytes + s_bytes + gather)
+
+
+def kernel_work(kind, work):
+    """(bound, algorithmic units per step, unit) of one kernel kind."""
+    if kind in ("score_lse", "score_accum"):
+        return "tensor", work["qk_flops"] / 1e12, "TFLOP/s"
+    if kind == "compact":
+        return "hbm", work["gather_bytes"] / 1e9, "GB/s"
+    return "hbm", work["s_bytes"] / 1e9, "GB/s"
+
+
+def kernel_src_hash(kind):
+    files = {"score_lse": "score.cu", "score_accum": "score.cu", "pool": "score.cu",
+             "group_stats": "select.cu", "select": "select.cu", "compact": "compact.cu"}[kind]
+    h = hashlib.sha256()
+    for f in (files, "ptx.cuh", "common.cuh"):
+        h.update((ROOT / "paper_2606_01790_gb300" / "csrc" / f).read_bytes())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kind, workload):
+    """DRAM bytes per launch from a committed ncu summary, if it was taken on
+    the current source of the kernel; else None."""
+    p = ROOT / "profiles" / "traffic.json"
+    if not p.exists():
+        return None
+    d = json.loads(p.read_text()).get(f"{kind}@{workload}")
+    if not d or d.get("src_sha") != kernel_src_hash(kind):
+        return None
+    return d.get("dram_bytes_per_launch")
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.samples = []
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(device_index)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+            return
+        self.t = threading.Thread(target=self._read, daemon=True)
+        self.t.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), [x.strip() for x in line.split(",")]))
+
+    def stop(self):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0, t1):
+        rows = [s for (t, s) in self.samples if t0 <= t <= t1]
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4)
+                          if len(r) > 5 + i and r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows),
+                "power_w_max": max((num(r[3]) or 0.0) for r in rows)}
+
+
+# ----------------------------------------------------------------------------- oracle (CPU)
+
+def oracle_worker(args):
+    """Times the fp64 oracle on the workload; prints one JSON line.
+
+    Budget mode (``--repeat 0``): layers 0, 1, ... of sequence 0 until
+    ``--budget-s`` seconds of oracle work have run.  Repeat mode: layer 0,
+    ``--repeat`` times (the reference arm's steps)."""
+    from oracle import starkv_oracle as O
+    from paper_2606_01790_gb300 import synthetic as syn
+    wl = syn.WORKLOADS[args.workload]
+    p = O.Params()
+    spent, tokens = 0.0, 0
+    per_call = []
+    layers = [0] * args.repeat if args.repeat > 0 else list(range(min(wl.n_layers, args.max_layers)))
+    cache = {}
+    for layer in layers:
+        if layer not in cache:
+            cache[layer] = syn.make_sequence(wl, seq=0, layers=[layer])
+        si = cache[layer]
+        lay = si.layout[0]
+        st = O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols)
+        q, k, v = si.q[0].double().numpy(), si.k[0].double().numpy(), si.v[0].double().numpy()
+        t = time.perf_counter()
+        O.step_layer(q, k, v, lay.is_visual, lay.frame, lay.row, lay.col, si.cur_frame, si.budget,
+                     wl.window, wl.grid_rows, wl.grid_cols, st, p)
+        dt = time.perf_counter() - t
+        per_call.append(dt)
+        spent += dt
+        tokens += si.L - wl.window
+        if args.repeat == 0 and spent >= args.budget_s:
+            break
+    print(json.dumps(dict(tokens=tokens, seconds=spent, calls=len(per_call), per_call=per_call,
+                          l_past=syn.make_sequence(wl, seq=0, layers=[0]).L - wl.window)))
+
+
+def run_oracle_subprocess(workload, budget_s=15.0, max_layers=28, repeat=0):
+    threads = str(os.cpu_count() or 1)
+    env = dict(os.environ, OPENBLAS_NUM_THREADS=threads, OMP_NUM_THREADS=threads,
+               MKL_NUM_THREADS=threads, CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, str(ROOT / "bench.py"), "--oracle-worker", "--workload", workload,
+                        "--budget-s", str(budget_s), "--max-layers", str(max_layers),
+                        "--repeat", str(repeat)],
+                       capture_output=True, text=True, env=env, timeout=3600)
+    if r.returncode != 0:
+        raise RuntimeError(f"oracle worker failed:\n{r.stderr[-2000:]}")
+    d = json.loads(r.stdout.strip().splitlines()[-1])
+    d["cores"] = int(threads)
+    return d
+
+
+def reference_arm(args):
+    """--impl reference: the fp64 oracle as it stands, one layer of the
+    workload per step, on the host cores (rank 0 only)."""
+    if int(os.environ.get("RANK", "0")) != 0:
+        return
+    from paper_2606_01790_gb300 import synthetic as syn
+    wl = syn.WORKLOADS[args.workload]
+    d = run_oracle_subprocess(args.workload, repeat=args.warmup + args.steps)
+    times = d["per_call"][args.warmup:]
+    total = sum(times)
+    value = d["l_past"] * len(times) / total
+    sample = (f"layer 0 of {wl.n_layers} per step (L_past = {d['l_past']} tokens scored per step), "
+              f"numpy BLAS on {d['cores']} threads")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * total / len(times), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": args.workload},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": d["cores"], "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def gpu_arm(args):
+    import numpy as np
+    import torch
+    import __graft_entry__
+    from paper_2606_01790_gb300 import starkv as sk
+    from paper_2606_01790_gb300 import synthetic as syn
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    __graft_entry__.build()
+
+    wl = syn.WORKLOADS[args.workload]
+    seeds = [rank * 1000 + i for i in range(wl.n_seqs)]
+    sis = [syn.make_sequence(wl, seq=i, seed=s) for i, s in enumerate(seeds)]
+    cfg = sk.Config(n_layers=wl.n_layers, n_heads=wl.n_heads, n_kv_heads=wl.n_kv_heads,
+                    head_dim=wl.head_dim, window=wl.window, grid_rows=wl.grid_rows,
+                    grid_cols=wl.grid_cols, max_seqs=len(sis))
+    st = sk.init_state(cfg)
+    G, w, d, nl = wl.n_kv_heads, wl.window, wl.head_dim, wl.n_layers
+
+    def make_seq(si, slot, device, pin=False):
+        L, B = si.L, si.budget
+        words = sk.pack_meta(si.layout[0].is_visual, si.layout[0].frame, si.layout[0].row, si.layout[0].col)
+        alloc = (lambda shape, dt: torch.empty(shape, dtype=dt, pin_memory=True)) if pin else \
+            (lambda shape, dt: torch.empty(shape, dtype=dt, device=device))
+        def put(t):
+            if pin:
+                o = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+                o.copy_(t)
+                return o
+            return t.to(device)
+        return sk.Seq(k=put(si.k), v=put(si.v), q=put(si.q), meta=put(sk.meta_tensor(words)),
+                      meta_layer_stride=0, L=L, cur_frame=si.cur_frame, budget=B, slot=slot,
+                      k_out=alloc((nl, G, B + w, d), torch.bfloat16),
+                      v_out=alloc((nl, G, B + w, d), torch.bfloat16),
+                      meta_out=alloc((nl, B + w), torch.int32), idx=alloc((nl, B), torch.int32))
+
+    seqs = [make_seq(si, i, dev) for i, si in enumerate(sis)]
+    ws = sk.workspace(st, seqs, device=dev)
+    stream = torch.cuda.current_stream(dev)
+    work = work_per_step(wl, [dict(L=si.L, B=si.budget) for si in sis])
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+
+    clocks = ClockSampler(local)
+    for _ in range(args.warmup):
+        sk.step(st, seqs, ws)
+    torch.cuda.synchronize(dev)
+    sk.check_device_error(st)
+    # soak: untimed steps so that clocks settle and are sampled under load
+    t_soak = time.time()
+    while time.time() - t_soak < args.soak_s:
+        for _ in range(10):
+            sk.step(st, seqs, ws)
+        torch.cuda.synchronize(dev)
+    sk.kernel_times(st)  # reset counters
+    sk.set_timing(st, True)
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        sk.step(st, seqs, ws)
+    e1.record(stream)
+    barrier()
+    t_end = time.time()
+    sk.set_timing(st, False)
+    ms = e0.elapsed_time(e1)
+    kt = sk.kernel_times(st)
+    sk.check_device_error(st)
+    clocks.stop()
+    ms_t = torch.tensor([ms], dtype=torch.float64, device=dev)
+    if dist is not None:
+        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
+    ms_max = float(ms_t.item())
+    ms_step = ms_max / args.steps
+    value = work["tokens"] * world * args.steps / (ms_max / 1e3)
+    launches = sum(v[0] for v in kt.values())
+
+    # roofline of the dominant kernel
+    peaks = _peaks()
+    kernels = {}
+    for kind, (n, tms) in kt.items():
+        if n == 0:
+            continue
+        kernels[kind] = {"launches": n, "avg_us": 1e3 * tms / n, "share": tms / max(1e-9, sum(v[1] for v in kt.values()))}
+    dom = max(kernels, key=lambda k: kernels[k]["avg_us"] * kernels[k]["launches"])
+    bound, units_per_step, unit = kernel_work(dom, work)
+    per_launch = units_per_step * args.steps / kernels[dom]["launches"]
+    achieved = per_launch / (kernels[dom]["avg_us"] * 1e-6)
+    peak = peaks["tc_sus"] if bound == "tensor" else peaks["hbm"]
+    traffic = recorded_traffic(dom, args.workload)
+    roofline = {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
+                "traffic": traffic, "kernel": dom,
+                "peak_src": f"{peaks['src']} ({'bf16 sustained' if bound == 'tensor' else 'HBM copy'})"}
+    step_roof_us = max(work["step_bytes"] / (peaks["hbm"] * 1e9), work["qk_flops"] / (peaks["tc"] * 1e12)) * 1e6
+    step_roofline = {"roofline_us": step_roof_us, "measured_us": 1e3 * ms_step,
+                     "frac": step_roof_us / (1e3 * ms_step), "alg_bytes": work["step_bytes"],
+                     "alg_flops": work["qk_flops"], "peak_src": peaks["src"]}
+
+    # e2e through the public host-buffer call
+    e2e = None
+    if not args.no_e2e:
+        hseqs = [make_seq(si, i, None, pin=True) for i, si in enumerate(sis)]
+        hws = sk.workspace(st, hseqs, host=True, device=dev)
+        h2d = sum(s.k.numel() * 2 + s.v.numel() * 2 + s.q.numel() * 2 + s.meta.numel() * 4 for s in hseqs)
+        d2h = sum(s.k_out.numel() * 2 + s.v_out.numel() * 2 + s.meta_out.numel() * 4 + s.idx.numel() * 4
+                  for s in hseqs)
+        for _ in range(2):
+            sk.step_host(st, hseqs, hws)
+        barrier()
+        n_e2e = max(1, min(args.steps, 20))
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n_e2e):
+            sk.step_host(st, hseqs, hws)
+        b.record(stream)
+        barrier()
+        e_ms = torch.tensor([a.elapsed_time(b)], dtype=torch.float64, device=dev)
+        if dist is not None:
+            dist.all_reduce(e_ms, op=dist.ReduceOp.MAX)
+        e2e = {"value": work["tokens"] * world * n_e2e / (float(e_ms.item()) / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n_e2e,
+               "ms_per_step": float(e_ms.item()) / n_e2e}
+        sk.check_device_error(st)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        o = run_oracle_subprocess(args.workload, budget_s=args.cpu_budget_s, max_layers=wl.n_layers)
+        cpu = {"value": o["tokens"] / o["seconds"], "unit": UNIT, "cores": o["cores"], "kind": "oracle",
+               "sample": f"{o['calls']} of {wl.n_layers} layers of sequence 0 "
+                         f"({o['tokens']} tokens scored in {o['seconds']:.1f} s, "
+                         f"numpy BLAS on {o['cores']} threads)"}
+
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": args.workload, "layers": nl, "seqs_per_gpu": len(sis),
+                       "L": [si.L for si in sis], "w": w, "B": [si.budget for si in sis],
+                       "H": wl.n_heads, "G": G, "d": d,
+                       "l2": f"inputs {2 * sum(s.k.numel() for s in seqs) * 2 / 1e9:.2f} GB per step "
+                             "> 129 MB L2 (no flush)",
+                       "parallelism": f"replicas x{world}"},
+            "roofline": roofline, "step_roofline": step_roofline, "kernels": kernels,
+            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
+            "clocks": clocks.summary(t_soak, t_end),
+        }))
+    if dist is not None:
+        dist.destroy_process_group()
+    st.close()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["starkv", "reference"], default="starkv")
+    ap.add_argument("--workload", default="uitars_5shot_28l")
+    ap.add_argument("--soak-s", type=float, default=2.0)
+    ap.add_argument("--cpu-budget-s", type=float, default=15.0)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--oracle-worker", action="store_true", help=argparse.SUPPRESS)
+    ap.add_argument("--budget-s", type=float, default=15.0, help=argparse.SUPPRESS)
+    ap.add_argument("--max-layers", type=int, default=28, help=argparse.SUPPRESS)
+    ap.add_argument("--repeat", type=int, default=0, help=argparse.SUPPRESS)
+    args = ap.parse_args()
+    if args.oracle_worker:
+        oracle_worker(args)
+    elif args.impl == "reference":
+        reference_arm(args)
+    else:
+        gpu_arm(args)
+
+
+if __name__ == "__main__":
+    main()

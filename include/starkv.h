@@ -206,6 +206,27 @@ starkv_status starkv_check_device_error(starkv_state* st, void* stream);
  * knob: 0 makes the first wait that does not succeed at once run out. */
 starkv_status starkv_set_wait_limit(starkv_state* st, uint64_t limit_ns);
 
+/* Kernels of the library, for starkv_kernel_times. */
+enum {
+  STARKV_KERNEL_SCORE_LSE = 0,    /* scoring pass 1: per-row log-sum-exp (Sec. 3.3)        */
+  STARKV_KERNEL_SCORE_ACCUM = 1,  /* scoring pass 2: normalised group sums (Eqs. 2-4)      */
+  STARKV_KERNEL_POOL = 2,         /* AvgPool1D + group mean (Eqs. 3-4), per-layer calls    */
+  STARKV_KERNEL_GROUP_STATS = 3,  /* MI_g, phi_g, m_g per group (Eqs. 5, 8)                */
+  STARKV_KERNEL_SELECT = 4,       /* prior, temperature, fused score, top-B (Sec. 3.4-3.7) */
+  STARKV_KERNEL_COMPACT = 5,      /* KV gather (Eq. 11)                                    */
+  STARKV_NUM_KERNELS = 6
+};
+
+/* Kernel timing, a profiling aid.  While `on` is non-zero every kernel launch
+ * made for this state is bracketed by a CUDA event pair on its stream. */
+starkv_status starkv_set_timing(starkv_state* st, int32_t on);
+
+/* Per kernel kind (arrays of STARKV_NUM_KERNELS): launches made and, while
+ * timing was on, their summed device time in milliseconds, since the last
+ * call.  Waits for the recorded events.  Launch counts are kept with timing
+ * off too (total_ms then stays 0).  Either array may be NULL. */
+starkv_status starkv_kernel_times(starkv_state* st, int64_t* launches, float* total_ms);
+
 /* Thread-local message describing the last non-OK status on this thread. */
 const char* starkv_last_error(void);
 

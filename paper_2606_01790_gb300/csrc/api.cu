@@ -28,6 +28,15 @@ struct starkv_state {
   int device = 0;
   int num_sms = 0;
   uint64_t wait_ns = 1000000000ull;
+  // kernel timing (starkv_set_timing / starkv_kernel_times)
+  bool timing = false;
+  int64_t launches[STARKV_NUM_KERNELS] = {};
+  struct Rec {
+    int kind;
+    cudaEvent_t a, b;
+  };
+  std::vector<Rec> recs;
+  std::vector<cudaEvent_t> pool;
 };
 
 namespace {
@@ -86,6 +95,33 @@ starkv_status encode_3d(CUtensorMap* map, const void* base, uint64_t d0, uint64_
 }
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
+
+cudaEvent_t take_event(starkv_state* st) {
+  if (!st->pool.empty()) {
+    cudaEvent_t e = st->pool.back();
+    st->pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Launches one kernel kind through `fn`, counting it and, when timing is on,
+// bracketing it with an event pair on `stream`.
+template <typename F>
+cudaError_t launch(starkv_state* st, int kind, cudaStream_t stream, F&& fn) {
+  st->launches[kind] += 1;
+  if (!st->timing) return fn();
+  starkv_state::Rec r{kind, take_event(st), take_event(st)};
+  cudaError_t e = cudaEventRecord(r.a, stream);
+  if (e != cudaSuccess) return e;
+  e = fn();
+  if (e != cudaSuccess) return e;
+  e = cudaEventRecord(r.b, stream);
+  st->recs.push_back(r);
+  return e;
+}
 
 starkv_status validate_config(const starkv_config& c) {
   if (c.n_layers < 1 || c.n_heads < 1 || c.n_kv_heads < 1 || c.window < 1 || c.max_seqs < 1)
@@ -261,7 +297,8 @@ starkv_status run_score(starkv_state* st, const starkv_seq* seqs, int i0, int i1
   *partial_cursor += tiles;
   p.err = st->dev.err;
   p.wait_ns = st->wait_ns;
-  CUDA_TRY(score_launch(p, p.grid1, stream));
+  CUDA_TRY(launch(st, STARKV_KERNEL_SCORE_LSE, stream, [&] { return score_lse_launch(p, p.grid1, stream); }));
+  CUDA_TRY(launch(st, STARKV_KERNEL_SCORE_ACCUM, stream, [&] { return score_accum_launch(p, p.grid1, stream); }));
   return STARKV_OK;
 }
 
@@ -318,11 +355,20 @@ starkv_status run_stages(starkv_state* st, const starkv_seq* seqs, int nseq, int
       s = run_score(st, seqs, i0, i1, layer0, nlayers, ws, plan, &partial_cursor, stream);
       if (s != STARKV_OK) return s;
     }
-    if (stages & kPool) CUDA_TRY(pool_launch(b, c.n_kv_heads, c.n_heads, c.pool_kernel, lp_max, stream));
+    if ((stages & kPool) && lp_max > 0)
+      CUDA_TRY(launch(st, STARKV_KERNEL_POOL, stream, [&] {
+        return pool_launch(b, c.n_kv_heads, c.n_heads, c.pool_kernel, lp_max, stream);
+      }));
     if (stages & (kStatsRaw | kStatsPooled))
-      CUDA_TRY(group_stats_launch(b, kp, st->dev, (stages & kStatsRaw) != 0, stream));
-    if (stages & kSelect) CUDA_TRY(select_launch(b, kp, st->dev, stream));
-    if (stages & kCompact) CUDA_TRY(compact_launch(b, c.n_kv_heads, c.window, rows_out_max, st->num_sms, st->dev.err, stream));
+      CUDA_TRY(launch(st, STARKV_KERNEL_GROUP_STATS, stream, [&] {
+        return group_stats_launch(b, kp, st->dev, (stages & kStatsRaw) != 0, stream);
+      }));
+    if (stages & kSelect)
+      CUDA_TRY(launch(st, STARKV_KERNEL_SELECT, stream, [&] { return select_launch(b, kp, st->dev, stream); }));
+    if ((stages & kCompact) && rows_out_max > 0)
+      CUDA_TRY(launch(st, STARKV_KERNEL_COMPACT, stream, [&] {
+        return compact_launch(b, c.n_kv_heads, c.window, rows_out_max, st->num_sms, st->dev.err, stream);
+      }));
   }
   return STARKV_OK;
 }
@@ -439,6 +485,11 @@ starkv_status starkv_reset_seq(starkv_state* st, int32_t slot, void* stream) {
 starkv_status starkv_destroy_state(starkv_state* st) {
   if (!st) return STARKV_OK;
   cudaError_t e = cudaDeviceSynchronize();
+  for (auto& r : st->recs) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  for (auto ev : st->pool) cudaEventDestroy(ev);
   if (e == cudaSuccess) e = cudaFree(st->mem);
   delete st;
   if (e != cudaSuccess) return set_error(STARKV_ERR_CUDA, "destroy failed: %s", cudaGetErrorString(e));
@@ -593,6 +644,35 @@ starkv_status starkv_check_device_error(starkv_state* st, void* stream) {
   if (h & kErrMeta) return set_error(STARKV_ERR_DEVICE, "token metadata outside the patch grid");
   if (h & kErrIndex) return set_error(STARKV_ERR_DEVICE, "an index outside the cache reached the gather");
   return STARKV_OK;
+}
+
+starkv_status starkv_set_timing(starkv_state* st, int32_t on) {
+  if (!st) return set_error(STARKV_ERR_INVALID_ARG, "state is NULL");
+  st->timing = on != 0;
+  return STARKV_OK;
+}
+
+starkv_status starkv_kernel_times(starkv_state* st, int64_t* launches, float* total_ms) {
+  if (!st) return set_error(STARKV_ERR_INVALID_ARG, "state is NULL");
+  float ms[STARKV_NUM_KERNELS] = {};
+  starkv_status status = STARKV_OK;
+  for (auto& r : st->recs) {
+    float t = 0.f;
+    cudaError_t e = cudaEventSynchronize(r.b);
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&t, r.a, r.b);
+    if (e != cudaSuccess && status == STARKV_OK)
+      status = set_error(STARKV_ERR_CUDA, "event timing failed: %s", cudaGetErrorString(e));
+    ms[r.kind] += t;
+    st->pool.push_back(r.a);
+    st->pool.push_back(r.b);
+  }
+  st->recs.clear();
+  for (int k = 0; k < STARKV_NUM_KERNELS; ++k) {
+    if (launches) launches[k] = st->launches[k];
+    if (total_ms) total_ms[k] = ms[k];
+    st->launches[k] = 0;
+  }
+  return status;
 }
 
 const char* starkv_last_error(void) { return g_last_error.c_str(); }

@@ -456,12 +456,13 @@ cudaError_t score_configure() {
   return cudaFuncSetAttribute(k_score_accum, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
-cudaError_t score_launch(const ScoreParams& p, int grid, cudaStream_t stream) {
-  const size_t bytes = score_smem_bytes();
-  k_score_lse<<<grid, kScoreThreads, bytes, stream>>>(p);
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  k_score_accum<<<grid, kScoreThreads, bytes, stream>>>(p);
+cudaError_t score_lse_launch(const ScoreParams& p, int grid, cudaStream_t stream) {
+  k_score_lse<<<grid, kScoreThreads, score_smem_bytes(), stream>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t score_accum_launch(const ScoreParams& p, int grid, cudaStream_t stream) {
+  k_score_accum<<<grid, kScoreThreads, score_smem_bytes(), stream>>>(p);
   return cudaGetLastError();
 }
 

@@ -33,7 +33,8 @@ struct ScoreParams {
 
 size_t score_smem_bytes();
 cudaError_t score_configure();
-cudaError_t score_launch(const ScoreParams& p, int grid, cudaStream_t stream);
+cudaError_t score_lse_launch(const ScoreParams& p, int grid, cudaStream_t stream);
+cudaError_t score_accum_launch(const ScoreParams& p, int grid, cudaStream_t stream);
 cudaError_t pool_launch(const SeqBatch& b, int G, int H, int pool, int lp_max, cudaStream_t stream);
 
 }  // namespace starkv

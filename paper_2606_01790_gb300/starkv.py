@@ -24,8 +24,10 @@ ABI_FUNCTIONS = [
     "starkv_default_config", "starkv_init_state", "starkv_reset_seq", "starkv_destroy_state",
     "starkv_get_config", "starkv_workspace_bytes", "starkv_score_layer", "starkv_select",
     "starkv_compact", "starkv_step", "starkv_step_host", "starkv_check_device_error",
-    "starkv_set_wait_limit", "starkv_last_error",
+    "starkv_set_wait_limit", "starkv_set_timing", "starkv_kernel_times", "starkv_last_error",
 ]
+
+KERNELS = ["score_lse", "score_accum", "pool", "group_stats", "select", "compact"]
 
 
 class StarkvError(RuntimeError):
@@ -77,6 +79,8 @@ def lib() -> C.CDLL:
                                              C.POINTER(C.c_size_t)]
         L.starkv_check_device_error.argtypes = [st, C.c_void_p]
         L.starkv_set_wait_limit.argtypes = [st, C.c_uint64]
+        L.starkv_set_timing.argtypes = [st, C.c_int32]
+        L.starkv_kernel_times.argtypes = [st, C.POINTER(C.c_int64), C.POINTER(C.c_float)]
         L.starkv_last_error.argtypes = []
         L.starkv_last_error.restype = C.c_char_p
         for name in ABI_FUNCTIONS:
@@ -295,3 +299,16 @@ def check_device_error(st: State, stream=None) -> None:
 
 def device_error_status(st: State, stream=None) -> int:
     return lib().starkv_check_device_error(st.handle, _stream(stream))
+
+
+def set_timing(st: State, on: bool) -> None:
+    _check(lib().starkv_set_timing(st.handle, int(on)))
+
+
+def kernel_times(st: State):
+    """{kernel: (launches, total_ms)} since the previous read."""
+    n = len(KERNELS)
+    launches = (C.c_int64 * n)()
+    ms = (C.c_float * n)()
+    _check(lib().starkv_kernel_times(st.handle, launches, ms))
+    return {k: (int(launches[i]), float(ms[i])) for i, k in enumerate(KERNELS)}

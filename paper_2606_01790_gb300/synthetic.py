@@ -309,7 +309,7 @@ def make_sequence(wl: Workload, seq: int = 0, seed: int = 0,
     _parallel(one, list(range(nl)))
     n_vis = sh.n_shots * wl.visual_per_shot
     l_past = lay.L - wl.window
-    return SeqInput(q=q_out, k=k_out, v=v_out, layout=[lay] * nl, cur_frame=sh.n_shots - 1,
+    return SeqInput(q=q_out, k=k_out, v=v_out, layout=[lay] * nl, cur_frame=max(sh.n_shots - 1, 0),
                     budget=budget(sh.budget_pct, n_vis, l_past), n_visual_history=n_vis)
 
 
