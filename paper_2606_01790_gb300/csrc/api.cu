@@ -337,7 +337,8 @@ starkv_status run_stages(starkv_state* st, const starkv_seq* seqs, int nseq, int
   const starkv_config& c = st->cfg;
   WsPlan plan;
   const bool ws_S = (stages & kStatsRaw) != 0;
-  plan_ws(st, seqs, nseq, nlayers, ws_S, true, &plan);
+  const bool ws_score = (stages & kSelect) != 0;
+  plan_ws(st, seqs, nseq, nlayers, ws_S, ws_score, &plan);
   starkv_status s = check_ws(st, workspace, ws_bytes, plan.total);
   if (s != STARKV_OK) return s;
   char* ws = static_cast<char*>(workspace);
@@ -513,10 +514,11 @@ starkv_status starkv_workspace_bytes(const starkv_state* st, const starkv_seq* s
   if (!bytes) return set_error(STARKV_ERR_INVALID_ARG, "bytes is NULL");
   starkv_status s = validate_seqs(st, seqs, nseq, 0);
   if (s != STARKV_OK) return s;
-  WsPlan a, b;
-  plan_ws(st, seqs, nseq, st->cfg.n_layers, true, true, &a);
-  plan_ws(st, seqs, nseq, 1, false, true, &b);
-  size_t total = std::max(a.total, b.total);
+  WsPlan a, b, c1;
+  plan_ws(st, seqs, nseq, st->cfg.n_layers, true, true, &a);   // starkv_step
+  plan_ws(st, seqs, nseq, 1, false, false, &b);                 // starkv_score_layer, starkv_compact
+  plan_ws(st, seqs, nseq, 1, false, true, &c1);                 // starkv_select
+  size_t total = std::max(a.total, std::max(b.total, c1.total));
   if (host) {
     std::vector<starkv_seq> dev(seqs, seqs + nseq);
     size_t staged = 0;
