@@ -167,6 +167,26 @@ starkv_status starkv_score_layer(starkv_state* st, int32_t layer, const starkv_s
                                  int32_t nseq, void* workspace, size_t workspace_bytes,
                                  void* stream);
 
+/* starkv_score_layer for callers that cannot allocate device memory: for
+ * example code running where cudaMalloc is forbidden or unavailable, such as a
+ * host that hands out only pre-registered buffers, or a plugin inside another
+ * runtime that owns every device allocation.  The paper has no counterpart;
+ * this is a deployment aid.  Same arguments and results as starkv_score_layer,
+ * minus the workspace: the scratch (pass-1 partials and unpooled sums) is one
+ * static device array of 16 MiB per device, which every GPU that loads this
+ * library holds until the process exits.  The call allocates no device memory
+ * (no cudaMalloc / cudaFree).  Its first call on a device looks up the array's
+ * device address (cudaGetSymbolAddress) with that device current, so make that
+ * first call before any stream capture.  Every call on a device shares the one
+ * array and leaves its last contents there (nothing in it has to start at
+ * zero): calls that may overlap on the GPU (different streams, or threads
+ * without ordering) race on it and must not be issued.  A batch whose scratch
+ * would exceed 16 MiB is rejected with STARKV_ERR_UNSUPPORTED before any
+ * launch (about 1.1 MB per sequence at the 5-screenshot UI-TARS shape); kernel
+ * timing must be off (it creates CUDA events). */
+starkv_status starkv_score_layer_noalloc(starkv_state* st, int32_t layer, const starkv_seq* seqs,
+                                         int32_t nseq, void* stream);
+
 /* Sec. 3.3 - 3.7 after the group score map (Algorithm 1 from s_bar to I): from
  * S of layer `layer`: s_bar, g*, online MI per group (Eq. 5) -> EMA (Eq. 6) ->
  * prior w (Eq. 7) -> beta; phi_g and the m_g update (Eq. 8) -> D_t (Eq. 9);

@@ -680,3 +680,54 @@ starkv_status starkv_kernel_times(starkv_state* st, int64_t* launches, float* to
 const char* starkv_last_error(void) { return g_last_error.c_str(); }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// starkv_score_layer_noalloc: the scoring call for callers that cannot
+// allocate device memory (see include/starkv.h).  Its scratch is one static
+// device array shared by every call on a device; the array's device address is
+// looked up once per device with that device current.
+
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;   // 16 MiB per device
+__device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+
+}  // namespace
+
+extern "C" starkv_status starkv_score_layer_noalloc(starkv_state* st, int32_t layer, const starkv_seq* seqs,
+                                                    int32_t nseq, void* stream) {
+  starkv_status s = validate_seqs(st, seqs, nseq, kNeedK | kNeedQ | kNeedS);
+  if (s != STARKV_OK) return s;
+  if (layer < 0 || layer >= st->cfg.n_layers) return set_error(STARKV_ERR_INVALID_ARG, "layer out of range");
+  if (st->timing)
+    return set_error(STARKV_ERR_INVALID_ARG, "kernel timing creates CUDA events: turn it off for this call");
+  if ((s = check_device(st)) != STARKV_OK) return s;
+  if (st->device < 0 || st->device >= kNoAllocMaxDevices)
+    return set_error(STARKV_ERR_UNSUPPORTED, "device index %d is beyond the %d this call tracks", st->device,
+                     kNoAllocMaxDevices);
+  WsPlan plan;
+  plan_ws(st, seqs, nseq, 1, false, false, &plan);
+  if (plan.total > kNoAllocScratchBytes)
+    return set_error(STARKV_ERR_UNSUPPORTED,
+                     "this call needs %zu bytes of scratch; the static scratch holds %zu bytes: "
+                     "split the batch or use starkv_score_layer with a workspace",
+                     plan.total, kNoAllocScratchBytes);
+  void* scratch = nullptr;
+  {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[st->device]) {
+      void* p = nullptr;
+      const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+      if (e != cudaSuccess || !p)
+        return set_error(STARKV_ERR_CUDA, "cudaGetSymbolAddress of the static scratch failed: %s",
+                         cudaGetErrorString(e));
+      g_noalloc_ptr[st->device] = p;
+    }
+    scratch = g_noalloc_ptr[st->device];
+  }
+  return run_stages(st, seqs, nseq, layer, 1, kScore | kPool, scratch, kNoAllocScratchBytes,
+                    static_cast<cudaStream_t>(stream));
+}

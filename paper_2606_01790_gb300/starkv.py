@@ -25,6 +25,7 @@ ABI_FUNCTIONS = [
     "starkv_get_config", "starkv_workspace_bytes", "starkv_score_layer", "starkv_select",
     "starkv_compact", "starkv_step", "starkv_step_host", "starkv_check_device_error",
     "starkv_set_wait_limit", "starkv_set_timing", "starkv_kernel_times", "starkv_last_error",
+    "starkv_score_layer_noalloc",
 ]
 
 KERNELS = ["score_lse", "score_accum", "pool", "group_stats", "select", "compact"]
@@ -69,6 +70,7 @@ def lib() -> C.CDLL:
         for name in ("starkv_step", "starkv_step_host"):
             getattr(L, name).argtypes = [st, C.POINTER(CSeq), C.c_int32, C.c_void_p, C.c_size_t,
                                          C.c_void_p]
+        L.starkv_score_layer_noalloc.argtypes = [st, C.c_int32, C.POINTER(CSeq), C.c_int32, C.c_void_p]
         L.starkv_default_config.argtypes = [C.POINTER(CConfig)]
         L.starkv_default_config.restype = None
         L.starkv_init_state.argtypes = [C.POINTER(CConfig), C.POINTER(C.c_void_p), C.c_void_p]
@@ -272,6 +274,13 @@ def _call_layer(fn, st: State, layer: int, seqs: Sequence[Seq], ws: torch.Tensor
 
 def score_layer(st: State, layer: int, seqs: Sequence[Seq], ws: torch.Tensor, stream=None) -> None:
     _call_layer(lib().starkv_score_layer, st, layer, seqs, ws, stream)
+
+
+def score_layer_noalloc(st: State, layer: int, seqs: Sequence[Seq], stream=None) -> None:
+    """``starkv_score_layer`` without a workspace: for callers that cannot
+    allocate device memory; the library's static 16 MiB scratch is used."""
+    arr = _seq_array(seqs)
+    _check(lib().starkv_score_layer_noalloc(st.handle, layer, arr, len(seqs), _stream(stream)))
 
 
 def select(st: State, layer: int, seqs: Sequence[Seq], ws: torch.Tensor, stream=None) -> None:
