@@ -76,7 +76,7 @@ def kernel_work(kind, work):
 
 def kernel_src_hash(kind):
     files = {"score_lse": "score.cu", "score_accum": "score.cu", "pool": "score.cu",
-             "group_stats": "select.cu", "select": "select.cu", "compact": "compact.cu"}[kind]
+             "calibrate": "select.cu", "compact": "compact.cu"}[kind]
     h = hashlib.sha256()
     for f in (files, "ptx.cuh", "common.cuh"):
         h.update((ROOT / "paper_2606_01790_gb300" / "csrc" / f).read_bytes())

@@ -231,10 +231,10 @@ enum {
   STARKV_KERNEL_SCORE_LSE = 0,    /* scoring pass 1: per-row log-sum-exp (Sec. 3.3)        */
   STARKV_KERNEL_SCORE_ACCUM = 1,  /* scoring pass 2: normalised group sums (Eqs. 2-4)      */
   STARKV_KERNEL_POOL = 2,         /* AvgPool1D + group mean (Eqs. 3-4), per-layer calls    */
-  STARKV_KERNEL_GROUP_STATS = 3,  /* MI_g, phi_g, m_g per group (Eqs. 5, 8)                */
-  STARKV_KERNEL_SELECT = 4,       /* prior, temperature, fused score, top-B (Sec. 3.4-3.7) */
-  STARKV_KERNEL_COMPACT = 5,      /* KV gather (Eq. 11)                                    */
-  STARKV_NUM_KERNELS = 6
+  STARKV_KERNEL_CALIBRATE = 3,    /* MI, phi, prior, temperature, fused score, top-B
+                                     (Sec. 3.4-3.7): one cluster of G CTAs per layer       */
+  STARKV_KERNEL_COMPACT = 4,      /* KV gather (Eq. 11)                                    */
+  STARKV_NUM_KERNELS = 5
 };
 
 /* Kernel timing, a profiling aid.  While `on` is non-zero every kernel launch

@@ -201,15 +201,18 @@ KParams make_kparams(const starkv_state* st) {
 // Workspace regions of one call over layers [layer0, layer0 + nlayers).
 struct WsPlan {
   size_t partials = 0, s_raw = 0, total = 0;
-  std::vector<size_t> raw_off, S_off, score_off;  // per seq, SIZE_MAX = not in workspace
+  std::vector<size_t> raw_off, S_off, score_off, vis_off;  // per seq, SIZE_MAX = not in workspace
 };
 
 int tiles_of(int lp) { return (lp + kTileKeys - 1) / kTileKeys; }
 
+// ws_score: the calibration kernel runs (fused score region; key/cell region
+// of the rows longer than its shared-memory capacity).
 void plan_ws(const starkv_state* st, const starkv_seq* seqs, int nseq, int nlayers, bool ws_S,
              bool ws_score, WsPlan* p) {
   const starkv_config& c = st->cfg;
   const int G = c.n_kv_heads;
+  const int cap = calibrate_capacity(c.mi_bins, c.mi_grid, c.grid_rows, c.grid_cols);
   size_t off = 0;
   size_t tiles = 0;
   for (int i = 0; i < nseq; ++i) tiles += static_cast<size_t>(nlayers) * G * tiles_of(seqs[i].L - c.window);
@@ -218,8 +221,13 @@ void plan_ws(const starkv_state* st, const starkv_seq* seqs, int nseq, int nlaye
   p->raw_off.assign(nseq, SIZE_MAX);
   p->S_off.assign(nseq, SIZE_MAX);
   p->score_off.assign(nseq, SIZE_MAX);
+  p->vis_off.assign(nseq, SIZE_MAX);
   for (int i = 0; i < nseq; ++i) {
     const size_t lp = seqs[i].L - c.window;
+    if (ws_score && lp > static_cast<size_t>(cap)) {
+      p->vis_off[i] = off;
+      off += align256(static_cast<size_t>(nlayers) * G * lp * 2 * sizeof(uint32_t));
+    }
     p->raw_off[i] = off;
     off += align256(static_cast<size_t>(nlayers) * G * lp * sizeof(float));
     if (ws_S && !seqs[i].S) {
@@ -255,6 +263,7 @@ SeqView make_view(const starkv_state* st, const starkv_seq& s, char* ws, const W
   v.s_raw = reinterpret_cast<float*>(ws + plan.raw_off[i]);
   v.score = plan.score_off[i] != SIZE_MAX ? reinterpret_cast<float*>(ws + plan.score_off[i]) : s.score;
   v.stats = s.stats;
+  v.vis = plan.vis_off[i] != SIZE_MAX ? reinterpret_cast<uint32_t*>(ws + plan.vis_off[i]) : nullptr;
   return v;
 }
 
@@ -360,12 +369,10 @@ starkv_status run_stages(starkv_state* st, const starkv_seq* seqs, int nseq, int
       CUDA_TRY(launch(st, STARKV_KERNEL_POOL, stream, [&] {
         return pool_launch(b, c.n_kv_heads, c.n_heads, c.pool_kernel, lp_max, stream);
       }));
-    if (stages & (kStatsRaw | kStatsPooled))
-      CUDA_TRY(launch(st, STARKV_KERNEL_GROUP_STATS, stream, [&] {
-        return group_stats_launch(b, kp, st->dev, (stages & kStatsRaw) != 0, stream);
-      }));
     if (stages & kSelect)
-      CUDA_TRY(launch(st, STARKV_KERNEL_SELECT, stream, [&] { return select_launch(b, kp, st->dev, stream); }));
+      CUDA_TRY(launch(st, STARKV_KERNEL_CALIBRATE, stream, [&] {
+        return calibrate_launch(b, kp, st->dev, (stages & kStatsRaw) != 0, lp_max, stream);
+      }));
     if ((stages & kCompact) && rows_out_max > 0)
       CUDA_TRY(launch(st, STARKV_KERNEL_COMPACT, stream, [&] {
         return compact_launch(b, c.n_kv_heads, c.window, rows_out_max, st->num_sms, st->dev.err, stream);

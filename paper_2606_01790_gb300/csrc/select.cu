@@ -1,28 +1,37 @@
-// Calibration and selection of Sec. 3.4 - 3.7 (Algorithm 1 from s_bar to I).
+// Calibration and selection of Sec. 3.4 - 3.7 (Algorithm 1 from s_bar to I):
+// one thread-block cluster of G CTAs per (sequence, layer).
 //
-// k_group_stats, one CTA per (seq, layer, group g):
-//   (optionally) AvgPool1D + group mean of the unpooled sums -> S[g, :]   (Eqs. 3-4)
-//   RankBin: K equal-frequency bins of S[g, visual] by an exact multi-target
-//            radix select (4 x 8-bit digit passes) on order-preserving keys,
-//            ties broken by position with a block-wide ordered count;
-//   SpatialBin + joint histogram (shared-memory atomics) -> plug-in MI_g  (Eq. 5)
-//   phi_g = cos(current-frame row on the patch grid, m_g); m_g EMA update (Eq. 8)
-// k_select, one CTA per (seq, layer):
-//   MI EMA -> min-max -> softmax prior w (Eqs. 6-7), lambda schedule;
-//   s_bar, g*, entropy H and temperature T (Sec. 3.6);
-//   s_t = max(s_bar beta D, 0)^(1/T) (Eq. final_score, Eq. 9);
-//   global top-B with ties to the lower index by radix select on
-//   order-preserving keys + ordered stream compaction -> ascending indices.
+// Phase 1, CTA g of the cluster works on group g:
+//   (step path) AvgPool1D + group mean of the unpooled sums -> S[g, :] (Eqs. 3-4);
+//   RankBin: the K - 1 equal-frequency boundaries of S[g, visual tokens] by an
+//     exact multi-target radix select (12 + 10 + 10-bit digits) on
+//     order-preserving keys, equal keys ordered by position;
+//   SpatialBin + joint histogram -> plug-in MI_g                        (Eq. 5);
+//   phi_g = cos(current-frame row on the patch grid, m_g); m_g update    (Eq. 8).
+// Phase 2, CTA r of the cluster works on tokens [r Lp / G, (r + 1) Lp / G):
+//   MI EMA, min-max and softmax prior, lambda schedule                  (Eqs. 6-7);
+//   s_bar, g*, Z = sum s_bar and the entropy H (Sec. 3.6), the per-CTA
+//     partial sums exchanged through distributed shared memory;
+//   s_t = max(s_bar beta D, 0)^(1/T)                     (Eq. final_score, Eq. 9);
+//   global top-B with ties to the lower index (Sec. 3.7): one radix select
+//     whose digit histograms are summed over the cluster, then an ordered
+//     compaction whose offsets come from the lower-ranked CTAs.
+#include <algorithm>
+
 #include "common.cuh"
+#include "ptx.cuh"
 #include "select.cuh"
 
 namespace starkv {
 
 namespace {
 
-constexpr int kStatsThreads = 512;
-constexpr int kSelectThreads = 1024;
-constexpr int kMaxTargets = 15;   // K - 1 with K <= 16
+constexpr int kCalThreads = 1024;
+constexpr int kMaxTargets = 15;      // K - 1 with K <= 16
+constexpr int kBins0 = 4096;         // first radix digit: key bits 31..20
+constexpr int kBins1 = 1024;         // second and third digits: bits 19..10 and 9..0
+constexpr uint16_t kNoCell = 0xFFFF; // not a (valid) visual token
+constexpr size_t kSmemMax = 227 * 1024;
 
 // Order-preserving map float -> uint32 (a < b  <=>  key(a) < key(b) for non-NaN).
 __device__ __forceinline__ uint32_t order_key(float x) {
@@ -37,55 +46,20 @@ __device__ __forceinline__ T warp_sum(T v) {
   return v;
 }
 
-// Block-wide sum (all threads get the result).  `red` holds >= 32 T.
+// Sum over the 1024 threads, in a fixed order; every thread gets the result.
 template <typename T>
 __device__ T block_sum(T v, T* red) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   v = warp_sum(v);
   __syncthreads();
   if (lane == 0) red[warp] = v;
   __syncthreads();
-  T t = lane < nw ? red[lane] : T(0);
-  t = warp_sum(t);
-  return t;
+  return warp_sum(red[lane]);
 }
 
-// Warp-cooperative search in a 256-bin histogram: the digit whose bin holds
-// rank `rank` (0-based) and the count of keys in lower bins.
-__device__ __forceinline__ void find_digit(const int* hist, int rank, int* digit, int* below) {
-  const int lane = threadIdx.x & 31;
-  int local[8];
-  int sum = 0;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    local[i] = hist[lane * 8 + i];
-    sum += local[i];
-  }
-  int incl = sum;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += y;
-  }
-  const int excl = incl - sum;
-  const unsigned hit = __ballot_sync(0xffffffffu, rank >= excl && rank < incl);
-  const int src = __ffs(hit) - 1;
-  if (lane == src) {
-    int c = excl;
-    for (int i = 0; i < 8; ++i) {
-      if (rank < c + local[i]) {
-        *digit = lane * 8 + i;
-        *below = c;
-        break;
-      }
-      c += local[i];
-    }
-  }
-}
-
-// Exclusive scan of one int per thread over the block; `tmp` holds >= 32 ints.
-__device__ int block_exclusive_scan(int v, int* tmp, int* total) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+// Exclusive scan of one int per thread over the block; `tmp` holds >= 33 ints.
+__device__ int block_excl_scan(int v, int* tmp, int* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   int incl = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -96,396 +70,617 @@ __device__ int block_exclusive_scan(int v, int* tmp, int* total) {
   if (lane == 31) tmp[warp] = incl;
   __syncthreads();
   if (warp == 0) {
-    int w = lane < nw ? tmp[lane] : 0;
+    const int w = tmp[lane];
     int wi = w;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int y = __shfl_up_sync(0xffffffffu, wi, o);
       if (lane >= o) wi += y;
     }
-    if (lane < nw) tmp[lane] = wi - w;
-    if (lane == nw - 1) tmp[32] = wi;
+    tmp[lane] = wi - w;
+    if (lane == 31) tmp[32] = wi;
   }
   __syncthreads();
   if (total) *total = tmp[32];
   return tmp[warp] + incl - v;
 }
 
-struct StatsShared {
-  int hist[kMaxTargets][256];
-  uint32_t prefix[kMaxTargets];
-  int rem[kMaxTargets];
-  int less[kMaxTargets];
-  int reach[kMaxTargets];
-  int eqbase[kMaxTargets];
-  int digit[kMaxTargets];
-  int below[kMaxTargets];
-  int tmp[33];
-  double dred[32];
-  int joint[kMaxHist];
+// One warp: the bin of a 1024-bin histogram that holds rank `rank` (0-based)
+// and the count of keys in lower bins; written by the lane that finds it.
+__device__ void warp_find_1024(const int* hist, int rank, int* digit, int* below) {
+  const int lane = threadIdx.x & 31;
+  const int4* h4 = reinterpret_cast<const int4*>(hist + lane * 32);
+  int v[32];
+  int sum = 0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int4 q = h4[i];
+    v[4 * i] = q.x;
+    v[4 * i + 1] = q.y;
+    v[4 * i + 2] = q.z;
+    v[4 * i + 3] = q.w;
+    sum += (q.x + q.y) + (q.z + q.w);
+  }
+  int incl = sum;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += y;
+  }
+  const int excl = incl - sum;
+  if (rank >= excl && rank < incl) {
+    int c = excl, d = 0;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      if (d == i && rank >= c + v[i]) {
+        c += v[i];
+        d = i + 1;
+      }
+    *digit = lane * 32 + d;
+    *below = c;
+  }
+}
+
+// Warp-aggregated shared-memory histogram increment; every lane calls it.
+__device__ __forceinline__ void hist_add(int* hist, bool valid, uint32_t bin) {
+  const uint32_t key = valid ? bin : 0xFFFFFFFFu;
+  const unsigned peers = __match_any_sync(0xffffffffu, key);
+  if (valid && (__ffs(peers) - 1) == static_cast<int>(threadIdx.x & 31)) atomicAdd(&hist[bin], __popc(peers));
+}
+
+struct CalShared {
+  uint32_t prefix[kMaxTargets];   // RankBin boundary keys, built digit by digit
+  int rem[kMaxTargets];           // rank of the boundary among the keys sharing its prefix
+  int reach[kMaxTargets];         // boundary rank < N
+  int dig[kMaxTargets], below[kMaxTargets];
+  int eqcnt[kMaxTargets];         // keys equal to the boundary key
+  int nb[16];                     // rank-bin marginals
+  int scan[33];
+  float fred[32];
+  int ired[32];
+  double mib_old[kMaxGroups];     // MI EMA before this step
+  float w[kMaxGroups], ph[kMaxGroups];
+  float lam;
+  int n_old;
+  int any_tie;
+  // read by the other CTAs of the cluster
+  float mi, phi;                  // this CTA's group (phase 1)
+  float zpart, hpart;             // this CTA's token range (phase 2)
+  int vpart, nlt, neq;
+  // top-B radix select
+  uint32_t tprefix;
+  int trank;
 };
+
+constexpr size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
+constexpr size_t kCalSharedBytes = align16(sizeof(CalShared));
+
+__host__ __device__ __forceinline__ int hist_ints(int K) {
+  const int a = 2 * kBins0, b = (K - 1) * kBins1;
+  return a > b ? a : b;
+}
+
+size_t fixed_bytes(int K, int M, int R, int C) {
+  return kCalSharedBytes + static_cast<size_t>(hist_ints(K)) * 4 + align16(static_cast<size_t>(K) * M * M * 4) +
+         align16(static_cast<size_t>(R) * C * 4);
+}
 
 }  // namespace
 
 template <bool FROM_RAW>
-__global__ void __launch_bounds__(kStatsThreads) k_group_stats(const __grid_constant__ SeqBatch b,
-                                                               const __grid_constant__ KParams kp,
-                                                               DevState st) {
+__global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_constant__ SeqBatch b,
+                                                              const __grid_constant__ KParams kp, DevState st,
+                                                              int capl) {
   extern __shared__ __align__(16) uint8_t smem_raw[];
-  StatsShared& sh = *reinterpret_cast<StatsShared*>(smem_raw);
-  float* cur = reinterpret_cast<float*>(smem_raw + sizeof(StatsShared));  // [R*C]
+  CalShared& sh = *reinterpret_cast<CalShared*>(smem_raw);
+  const int G = kp.G, K = kp.K, M = kp.M, R = kp.R, C = kp.C, MM = M * M, RC = R * C, nt = K - 1;
+  int* hist = reinterpret_cast<int*>(smem_raw + kCalSharedBytes);
+  int* joint = hist + hist_ints(K);
+  float* cur = reinterpret_cast<float*>(joint + ((K * MM + 3) & ~3));
+  uint32_t* skeys = reinterpret_cast<uint32_t*>(cur + ((RC + 3) & ~3));
+  uint16_t* scells = reinterpret_cast<uint16_t*>(skeys + capl);
 
   const SeqView& sv = b.s[blockIdx.z];
-  const int g = blockIdx.x, ll = blockIdx.y, layer = b.layer0 + ll;
-  const int Lp = sv.Lp, G = kp.G, K = kp.K, M = kp.M, R = kp.R, C = kp.C;
-  const int tid = threadIdx.x, nth = blockDim.x;
-  const int warp = tid >> 5, lane = tid & 31;
-  float* S = sv.S + (static_cast<int64_t>(layer) * G + g) * Lp;
+  const int g = blockIdx.x;              // == rank in the cluster (the cluster spans grid x)
+  const int ll = blockIdx.y, layer = b.layer0 + ll;
+  const int Lp = sv.Lp;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const uint32_t* meta = sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride;
   const int sl = sv.slot * kp.n_layers + layer;
+  float* S = sv.S + (static_cast<int64_t>(layer) * G + g) * Lp;
+  const bool in_smem = Lp <= capl;
+  uint32_t* keys = in_smem ? skeys : sv.vis + static_cast<int64_t>(ll * G + g) * Lp * 2;
+  uint16_t* cells = in_smem ? scells : reinterpret_cast<uint16_t*>(keys + Lp);
 
-  // ---- Eqs. (3)-(4): pool along tokens and average the group's heads
-  if (FROM_RAW) {
-    const float* raw = sv.s_raw + static_cast<int64_t>(ll * G + g) * Lp;
-    const float scale = static_cast<float>(G) / static_cast<float>(kp.H) / static_cast<float>(kp.pool);
-    const int half = kp.pool >> 1;
-    for (int t = tid; t < Lp; t += nth) {
-      float acc = 0.f;
-      for (int j = -half; j <= half; ++j) {
-        const int u = t + j;
-        if (u >= 0 && u < Lp) acc += raw[u];
-      }
-      S[t] = acc * scale;
-    }
+  if (tid < G) sh.mib_old[tid] = st.mi_bar[sl * G + tid];
+  if (tid == 0) {
+    sh.n_old = st.n[sl];
+    sh.any_tie = 0;
   }
-  // ---- count visual tokens, validate their patch coordinates
+  for (int i = tid; i < kBins0; i += kCalThreads) hist[i] = 0;
+  for (int i = tid; i < K * MM; i += kCalThreads) joint[i] = 0;
+  for (int i = tid; i < RC; i += kCalThreads) cur[i] = 0.f;
+  __syncthreads();
+
+  // ================= phase 1: group g =================
+  // ---- one pass over the row: pooling (Eqs. 3-4), keys and cells of the
+  // visual tokens, the first radix digit, the current frame on the grid
+  const float pscale = static_cast<float>(G) / static_cast<float>(kp.H) / static_cast<float>(kp.pool);
+  const int half = kp.pool >> 1;
+  const float* raw = FROM_RAW ? sv.s_raw + static_cast<int64_t>(ll * G + g) * Lp : nullptr;
   int nv = 0;
-  for (int t = tid; t < Lp; t += nth) {
-    const uint32_t mt = meta[t];
-    if (meta_visual(mt)) {
-      ++nv;
-      if (meta_row(mt) >= R || meta_col(mt) >= C) atomicOr(st.err, kErrMeta);
+  for (int base = 0; base < Lp; base += 2 * kCalThreads) {
+    float s[2];
+    uint32_t mt[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int t = base + k * kCalThreads + tid;
+      s[k] = 0.f;
+      mt[k] = 0;
+      if (t < Lp) {
+        mt[k] = meta[t];
+        if (FROM_RAW) {
+          float acc = 0.f;
+          for (int j = -half; j <= half; ++j) {
+            const int u = t + j;
+            if (u >= 0 && u < Lp) acc += raw[u];
+          }
+          s[k] = acc * pscale;
+        } else {
+          s[k] = S[t];
+        }
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int t = base + k * kCalThreads + tid;
+      bool vis = false;
+      uint32_t key = 0;
+      if (t < Lp) {
+        if (FROM_RAW) S[t] = s[k];
+        uint16_t cell = kNoCell;
+        if (meta_visual(mt[k])) {
+          const int r = meta_row(mt[k]), c = meta_col(mt[k]);
+          if (r < R && c < C) {
+            vis = true;
+            key = order_key(s[k]);
+            cell = static_cast<uint16_t>((r * M / R) * M + (c * M / C));
+            if (meta_frame(mt[k]) == sv.cur_frame) atomicAdd(&cur[r * C + c], s[k]);
+          } else {
+            atomicOr(st.err, kErrMeta);
+          }
+        }
+        keys[t] = key;
+        cells[t] = cell;
+      }
+      nv += vis;
+      hist_add(hist, vis, key >> 20);
     }
   }
-  for (int i = tid; i < K * M * M; i += nth) sh.joint[i] = 0;
-  for (int i = tid; i < R * C; i += nth) cur[i] = 0.f;
-  nv = static_cast<int>(block_sum<double>(static_cast<double>(nv), sh.dred) + 0.5);
-  const int N = nv;
-  const int nt = K - 1;
+  const int N = block_sum<int>(nv, sh.ired);
   if (tid < nt) {
-    const int b1 = tid + 1;
-    const int Rb = static_cast<int>((static_cast<int64_t>(b1) * N + K - 1) / K);  // ceil(bN/K)
+    const int Rb = static_cast<int>((static_cast<int64_t>(tid + 1) * N + K - 1) / K);  // ceil(bN/K)
     sh.reach[tid] = Rb < N;
     sh.rem[tid] = Rb;
     sh.prefix[tid] = 0;
-    sh.less[tid] = 0;
+    sh.dig[tid] = 0;
+    sh.below[tid] = 0;
+    sh.eqcnt[tid] = 0;
   }
   __syncthreads();
 
-  double mi = 0.0;
+  float mi = 0.f;
   if (N > 0) {
-    // ---- Sec. 3.4 RankBin: the key at each boundary rank, 4 radix passes
-    for (int pass = 0; pass < 4; ++pass) {
-      const int shift = 24 - 8 * pass;
-      const int nh = pass == 0 ? 1 : nt;   // pass 0: one histogram serves every target
-      for (int i = tid; i < nh * 256; i += nth) (&sh.hist[0][0])[i] = 0;
-      __syncthreads();
-      for (int t = tid; t < Lp; t += nth) {
-        if (!meta_visual(meta[t])) continue;
-        const uint32_t u = order_key(S[t]);
-        if (pass == 0) {
-          atomicAdd(&sh.hist[0][u >> 24], 1);
-        } else {
-          for (int j = 0; j < nt; ++j)
-            if (sh.reach[j] && ((u ^ sh.prefix[j]) >> (shift + 8)) == 0)
-              atomicAdd(&sh.hist[j][(u >> shift) & 255], 1);
-        }
-      }
-      __syncthreads();
-      if (warp < nt && sh.reach[warp]) {
-        find_digit(pass == 0 ? sh.hist[0] : sh.hist[warp], sh.rem[warp], &sh.digit[warp], &sh.below[warp]);
-        __syncwarp();
-        if (lane == 0) {
-          sh.prefix[warp] |= static_cast<uint32_t>(sh.digit[warp]) << shift;
-          sh.rem[warp] -= sh.below[warp];
-          sh.less[warp] += sh.below[warp];
-        }
-      }
-      __syncthreads();
-    }
-    // ---- ties: rank among equal keys in index order (contiguous chunks per thread)
-    const int cs = ceil_div(Lp, nth);
-    const int t0 = min(Lp, tid * cs), t1 = min(Lp, t0 + cs);
-    int eq_local[kMaxTargets];
-    for (int j = 0; j < nt; ++j) eq_local[j] = 0;
-    for (int t = t0; t < t1; ++t) {
-      if (!meta_visual(meta[t])) continue;
-      const uint32_t u = order_key(S[t]);
-      for (int j = 0; j < nt; ++j) eq_local[j] += (sh.reach[j] && u == sh.prefix[j]);
-    }
-    for (int j = 0; j < nt; ++j) eq_local[j] = block_exclusive_scan(eq_local[j], sh.tmp, nullptr);
-    // ---- bins, spatial cells, joint histogram
-    const int MM = M * M;
-    for (int t = t0; t < t1; ++t) {
-      const uint32_t mt = meta[t];
-      if (!meta_visual(mt)) continue;
-      const uint32_t u = order_key(S[t]);
-      int bin = 0;
+    // ---- Sec. 3.4 RankBin, digit 1: one 4096-bin histogram serves every boundary
+    {
+      const int4 h = reinterpret_cast<const int4*>(hist)[tid];
+      const int sum = (h.x + h.y) + (h.z + h.w);
+      const int excl = block_excl_scan(sum, sh.scan, nullptr);
       for (int j = 0; j < nt; ++j) {
-        if (!sh.reach[j]) continue;
-        const uint32_t v = sh.prefix[j];
-        if (u > v || (u == v && eq_local[j] >= sh.rem[j])) ++bin;
-        eq_local[j] += (u == v);
+        const int r = sh.rem[j];
+        if (sh.reach[j] && r >= excl && r < excl + sum) {
+          int c = excl, d = 0;
+          if (r >= c + h.x) { c += h.x; d = 1; }
+          if (d == 1 && r >= c + h.y) { c += h.y; d = 2; }
+          if (d == 2 && r >= c + h.z) { c += h.z; d = 3; }
+          sh.dig[j] = tid * 4 + d;
+          sh.below[j] = c;
+        }
       }
-      const int r = meta_row(mt), c = meta_col(mt);
-      if (r < R && c < C) atomicAdd(&sh.joint[bin * MM + (r * M / R) * M + (c * M / C)], 1);
+      __syncthreads();
+      if (tid < nt && sh.reach[tid]) {
+        sh.prefix[tid] = static_cast<uint32_t>(sh.dig[tid]) << 20;
+        sh.rem[tid] -= sh.below[tid];
+      }
+      __syncthreads();
+    }
+    // ---- digits 2 and 3: one 1024-bin histogram per boundary over the keys
+    // that share the boundary's higher digits
+    for (int pass = 1; pass <= 2; ++pass) {
+      const int shift = pass == 1 ? 10 : 0;
+      for (int i = tid; i < nt * kBins1; i += kCalThreads) hist[i] = 0;
+      __syncthreads();
+      for (int t = tid; t < Lp; t += kCalThreads) {
+        if (cells[t] == kNoCell) continue;
+        const uint32_t u = keys[t];
+        for (int j = 0; j < nt; ++j)
+          if (sh.reach[j] && ((u ^ sh.prefix[j]) >> (shift + 10)) == 0)
+            atomicAdd(&hist[j * kBins1 + ((u >> shift) & 1023)], 1);
+      }
+      __syncthreads();
+      if (warp < nt && sh.reach[warp]) warp_find_1024(hist + warp * kBins1, sh.rem[warp], &sh.dig[warp], &sh.below[warp]);
+      __syncthreads();
+      if (tid < nt && sh.reach[tid]) {
+        sh.prefix[tid] |= static_cast<uint32_t>(sh.dig[tid]) << shift;
+        sh.rem[tid] -= sh.below[tid];
+        if (pass == 2) {
+          const int e = hist[tid * kBins1 + sh.dig[tid]];
+          sh.eqcnt[tid] = e;
+          if (e > 1) atomicOr(&sh.any_tie, 1);
+        }
+      }
+      __syncthreads();
+    }
+    // ---- rank bin of every visual token: the number of boundaries at or
+    // below it; joint (bin, cell) histogram
+    if (!sh.any_tie) {
+      for (int t = tid; t < Lp; t += kCalThreads) {
+        const int cell = cells[t];
+        if (cell == kNoCell) continue;
+        const uint32_t u = keys[t];
+        int bin = 0;
+        for (int j = 0; j < nt; ++j) bin += (sh.reach[j] && u >= sh.prefix[j]);
+        atomicAdd(&joint[bin * MM + cell], 1);
+      }
+    } else {
+      // equal keys at a boundary: their order is their position, so each
+      // thread walks one contiguous span and counts the equal keys before it
+      const int cs = ceil_div(Lp, kCalThreads);
+      const int t0 = min(Lp, tid * cs), t1 = min(Lp, t0 + cs);
+      int eqb[kMaxTargets];
+#pragma unroll
+      for (int j = 0; j < kMaxTargets; ++j) {
+        if (j >= nt) break;
+        int cnt = 0;
+        for (int t = t0; t < t1; ++t) cnt += (cells[t] != kNoCell && keys[t] == sh.prefix[j]);
+        eqb[j] = block_excl_scan(cnt, sh.scan, nullptr);
+      }
+      for (int t = t0; t < t1; ++t) {
+        const int cell = cells[t];
+        if (cell == kNoCell) continue;
+        const uint32_t u = keys[t];
+        int bin = 0;
+#pragma unroll
+        for (int j = 0; j < kMaxTargets; ++j) {
+          if (j >= nt) break;
+          if (!sh.reach[j]) continue;
+          const uint32_t P = sh.prefix[j];
+          if (u > P) {
+            ++bin;
+          } else if (u == P) {
+            if (eqb[j] >= sh.rem[j]) ++bin;
+            ++eqb[j];
+          }
+        }
+        atomicAdd(&joint[bin * MM + cell], 1);
+      }
     }
     __syncthreads();
-    // ---- Eq. (5): plug-in MI from the joint histogram (fp64)
-    const double invN = 1.0 / static_cast<double>(N);
-    for (int e = tid; e < K * MM; e += nth) {
-      const int n = sh.joint[e];
+    // ---- Eq. (5): plug-in MI (nats) from the joint histogram
+    int* nc = hist;   // cell marginals
+    for (int c = tid; c < MM; c += kCalThreads) {
+      int s = 0;
+      for (int bb = 0; bb < K; ++bb) s += joint[bb * MM + c];
+      nc[c] = s;
+    }
+    if (warp < K) {
+      int s = 0;
+      for (int i = lane; i < MM; i += 32) s += joint[warp * MM + i];
+      s = warp_sum(s);
+      if (lane == 0) sh.nb[warp] = s;
+    }
+    __syncthreads();
+    const float fN = static_cast<float>(N);
+    float acc = 0.f;
+    for (int e = tid; e < K * MM; e += kCalThreads) {
+      const int n = joint[e];
       if (n == 0) continue;
-      const int bb = e / MM, cc = e - bb * MM;
-      int nb = 0, nc = 0;
-      for (int i = 0; i < MM; ++i) nb += sh.joint[bb * MM + i];
-      for (int i = 0; i < K; ++i) nc += sh.joint[i * MM + cc];
-      mi += n * invN * log(static_cast<double>(n) * N / (static_cast<double>(nb) * nc));
+      const int bb = e / MM, c = e - bb * MM;
+      const float fn = static_cast<float>(n);
+      acc += fn * logf(fn * fN / (static_cast<float>(sh.nb[bb]) * static_cast<float>(nc[c])));
     }
+    mi = block_sum<float>(acc, sh.fred) / fN;
   }
-  mi = block_sum<double>(mi, sh.dred);
 
-  // ---- Sec. 3.5: current-frame row on the patch grid, phi_g, m_g update
-  for (int t = tid; t < Lp; t += nth) {
-    const uint32_t mt = meta[t];
-    if (meta_visual(mt) && meta_frame(mt) == sv.cur_frame) {
-      const int r = meta_row(mt), c = meta_col(mt);
-      if (r < R && c < C) atomicAdd(&cur[r * C + c], S[t]);
-    }
+  // ---- Sec. 3.5: phi_g = cos(current row, m_g); m_g EMA update (Eq. 8)
+  float* mrow = st.m + static_cast<int64_t>(sl * G + g) * RC;
+  float dot = 0.f, ncur = 0.f, nm = 0.f;
+  for (int i = tid; i < RC; i += kCalThreads) {
+    const float a = cur[i], bm = mrow[i];
+    dot = fmaf(a, bm, dot);
+    ncur = fmaf(a, a, ncur);
+    nm = fmaf(bm, bm, nm);
   }
-  __syncthreads();
-  float* m = st.m + static_cast<int64_t>(sl * G + g) * (R * C);
-  double dot = 0.0, ncur = 0.0, nm = 0.0;
-  for (int i = tid; i < R * C; i += nth) {
-    const double a = cur[i], bm = m[i];
-    dot += a * bm;
-    ncur += a * a;
-    nm += bm * bm;
-  }
-  dot = block_sum<double>(dot, sh.dred);
-  ncur = block_sum<double>(ncur, sh.dred);
-  nm = block_sum<double>(nm, sh.dred);
+  dot = block_sum<float>(dot, sh.fred);
+  ncur = block_sum<float>(ncur, sh.fred);
+  nm = block_sum<float>(nm, sh.fred);
   float phi = 0.f;
-  if (ncur > 0.0) {
-    if (nm > 0.0) {
-      phi = static_cast<float>(dot / (sqrt(ncur) * sqrt(nm)));
+  if (ncur > 0.f) {
+    if (nm > 0.f) {
+      phi = dot / (sqrtf(ncur) * sqrtf(nm));
       const float rt = kp.rho_t;
-      for (int i = tid; i < R * C; i += nth) m[i] = rt * m[i] + (1.f - rt) * cur[i];
+      for (int i = tid; i < RC; i += kCalThreads) mrow[i] = rt * mrow[i] + (1.f - rt) * cur[i];
     } else {
-      for (int i = tid; i < R * C; i += nth) m[i] = cur[i];
+      for (int i = tid; i < RC; i += kCalThreads) mrow[i] = cur[i];
     }
   }
   if (tid == 0) {
+    sh.mi = mi;
+    sh.phi = phi;
     st.mi_cur[sl * G + g] = mi;
     st.phi_cur[sl * G + g] = phi;
   }
-}
+  for (int i = tid; i < kBins0; i += kCalThreads) hist[i] = 0;   // top-B digit 1 (below)
+  cluster_sync();   // every group's S row, MI_g and phi_g are complete
 
-__global__ void __launch_bounds__(kSelectThreads) k_select(const __grid_constant__ SeqBatch b,
-                                                           const __grid_constant__ KParams kp,
-                                                           DevState st) {
-  __shared__ int hist[256];
-  __shared__ int tmp[33];
-  __shared__ double dred[32];
-  __shared__ float w_s[kMaxGroups], phi_s[kMaxGroups];
-  __shared__ float lam_s;
-  __shared__ int digit_s, below_s;
-
-  const SeqView& sv = b.s[blockIdx.y];
-  const int ll = blockIdx.x, layer = b.layer0 + ll;
-  const int Lp = sv.Lp, G = kp.G;
-  const int tid = threadIdx.x, nth = blockDim.x, warp = tid >> 5;
-  const float* S = sv.S + static_cast<int64_t>(layer) * G * Lp;
-  const uint32_t* meta = sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride;
-  float* score = sv.score + static_cast<int64_t>(layer) * Lp;
-  const int sl = sv.slot * kp.n_layers + layer;
+  // ================= phase 2: tokens [ta, tb) =================
   float* stats = sv.stats ? sv.stats + static_cast<int64_t>(layer) * (8 + 4 * G) : nullptr;
-
-  // ---- Eqs. (6)-(7): MI EMA, min-max, softmax prior; lambda schedule
+  // ---- Eqs. (6)-(7): MI EMA, min-max, softmax prior; lambda schedule (the
+  // same arithmetic in every CTA; CTA 0 stores the new state)
   if (tid == 0) {
-    const int n = st.n[sl];
-    double mib[kMaxGroups];
+    const int n = sh.n_old;
+    double mib[kMaxGroups], mic[kMaxGroups];
     double lo = 1e300, hi = -1e300;
-    for (int g = 0; g < G; ++g) {
-      const double cur = st.mi_cur[sl * G + g];
-      const double prev = st.mi_bar[sl * G + g];
-      mib[g] = n == 0 ? cur : kp.rho_mi * prev + (1.0 - kp.rho_mi) * cur;
-      st.mi_bar[sl * G + g] = mib[g];
-      lo = fmin(lo, mib[g]);
-      hi = fmax(hi, mib[g]);
+    for (int gg = 0; gg < G; ++gg) {
+      mic[gg] = static_cast<double>(dsmem_ld_f32(dsmem_map(&sh.mi, gg)));
+      sh.ph[gg] = dsmem_ld_f32(dsmem_map(&sh.phi, gg));
+      mib[gg] = n == 0 ? mic[gg] : kp.rho_mi * sh.mib_old[gg] + (1.0 - kp.rho_mi) * mic[gg];
+      lo = fmin(lo, mib[gg]);
+      hi = fmax(hi, mib[gg]);
     }
     double e[kMaxGroups], zmax = -1e300, zs = 0.0;
-    for (int g = 0; g < G; ++g) {
-      e[g] = ((mib[g] - lo) / ((hi - lo) + kp.eps)) / kp.tau;
-      zmax = fmax(zmax, e[g]);
+    for (int gg = 0; gg < G; ++gg) {
+      e[gg] = ((mib[gg] - lo) / ((hi - lo) + kp.eps)) / kp.tau;
+      zmax = fmax(zmax, e[gg]);
     }
-    for (int g = 0; g < G; ++g) {
-      e[g] = exp(e[g] - zmax);
-      zs += e[g];
+    for (int gg = 0; gg < G; ++gg) {
+      e[gg] = exp(e[gg] - zmax);
+      zs += e[gg];
     }
-    for (int g = 0; g < G; ++g) {
-      w_s[g] = static_cast<float>(e[g] / zs);
-      phi_s[g] = st.phi_cur[sl * G + g];
-    }
+    for (int gg = 0; gg < G; ++gg) sh.w[gg] = static_cast<float>(e[gg] / zs);
     float lam = 0.f;
     if (n >= kp.n_warmup)
       lam = kp.n_ramp <= 0 ? kp.lambda
                            : kp.lambda * fminf(1.f, static_cast<float>(n - kp.n_warmup) / kp.n_ramp);
-    lam_s = lam;
-    if (stats) {
-      stats[2] = lam;
-      stats[3] = static_cast<float>(n);
-      stats[6] = static_cast<float>(sv.budget);
-      stats[7] = 0.f;
-      for (int g = 0; g < G; ++g) {
-        stats[8 + g] = static_cast<float>(st.mi_cur[sl * G + g]);
-        stats[8 + G + g] = static_cast<float>(mib[g]);
-        stats[8 + 2 * G + g] = w_s[g];
-        stats[8 + 3 * G + g] = phi_s[g];
+    sh.lam = lam;
+    if (g == 0) {
+      for (int gg = 0; gg < G; ++gg) st.mi_bar[sl * G + gg] = mib[gg];
+      st.n[sl] = n + 1;
+      if (stats) {
+        stats[2] = lam;
+        stats[3] = static_cast<float>(n);
+        stats[6] = static_cast<float>(sv.budget);
+        stats[7] = 0.f;
+        for (int gg = 0; gg < G; ++gg) {
+          stats[8 + gg] = static_cast<float>(mic[gg]);
+          stats[8 + G + gg] = static_cast<float>(mib[gg]);
+          stats[8 + 2 * G + gg] = sh.w[gg];
+          stats[8 + 3 * G + gg] = sh.ph[gg];
+        }
       }
     }
-    st.n[sl] = n + 1;
   }
-  __syncthreads();
-
-  // ---- Eq. (4): s_bar; Sec. 3.6: Z = sum s_bar
+  const int ta = static_cast<int>(static_cast<int64_t>(g) * Lp / G);
+  const int tb = static_cast<int>(static_cast<int64_t>(g + 1) * Lp / G);
+  const int nr = tb - ta;
+  const float* S0 = sv.S + static_cast<int64_t>(layer) * G * Lp;
   const float invG = 1.f / static_cast<float>(G);
-  double z = 0.0;
-  int nv = 0;
-  for (int t = tid; t < Lp; t += nth) {
-    float acc = 0.f;
-    for (int g = 0; g < G; ++g) acc += S[static_cast<int64_t>(g) * Lp + t];
-    const float sbar = acc * invG;
-    score[t] = sbar;
-    z += sbar;
-    nv += meta_visual(meta[t]);
-  }
-  z = block_sum<double>(z, dred);
-  const double nvd = block_sum<double>(static_cast<double>(nv), dred);
-  // ---- Sec. 3.6: H = -sum p log(p + eps) / log L_p, T
-  const float invz = static_cast<float>(1.0 / (z + kp.eps_h));
-  double hs = 0.0;
-  for (int t = tid; t < Lp; t += nth) {
-    const float p = score[t] * invz;
-    hs += static_cast<double>(p * logf(p + kp.eps_h));
-  }
-  hs = block_sum<double>(hs, dred);
-  const double Hn = Lp > 1 ? -hs / log(static_cast<double>(Lp)) : 0.0;
-  const float T = static_cast<float>(kp.t_min + (kp.t_max - kp.t_min) * Hn);
-  const float invT = 1.f / T;
-  if (tid == 0 && stats) {
-    stats[0] = static_cast<float>(Hn);
-    stats[1] = T;
-    stats[4] = static_cast<float>(z);
-    stats[5] = static_cast<float>(nvd);
-  }
-  // ---- Eq. (final_score) with Eq. (9): fused score
-  const float lam = lam_s;
-  for (int t = tid; t < Lp; t += nth) {
-    float best = S[t];
-    int gs = 0;
-    for (int g = 1; g < G; ++g) {
-      const float v = S[static_cast<int64_t>(g) * Lp + t];
+  // s_bar (Eq. 4) of token t and its governing group g* (lowest on ties)
+  auto sbar_of = [&](int t, int& gs) {
+    float best = S0[t], acc = best;
+    gs = 0;
+    for (int gg = 1; gg < G; ++gg) {
+      const float v = S0[static_cast<int64_t>(gg) * Lp + t];
+      acc += v;
       if (v > best) {
         best = v;
-        gs = g;
+        gs = gg;
       }
     }
-    const float sbar = score[t];
-    const float beta = (1.f - lam) + lam * static_cast<float>(G) * w_s[gs];
-    float d = 1.f;
-    const uint32_t mt = meta[t];
-    if (meta_visual(mt)) {
-      const float df = static_cast<float>(sv.cur_frame - meta_frame(mt));
-      d = kp.d_min + (1.f - kp.d_min) * expf(-kp.delta * df * phi_s[gs]);
-    }
-    score[t] = powf(fmaxf(sbar * beta * d, 0.f), invT);
+    return acc * invG;
+  };
+  // ---- Sec. 3.6: Z = sum s_bar over the cluster
+  float z = 0.f;
+  int nvr = 0;
+  for (int t = ta + tid; t < tb; t += kCalThreads) {
+    int gs;
+    z += sbar_of(t, gs);
+    nvr += meta_visual(meta[t]);
   }
-  __syncthreads();
+  z = block_sum<float>(z, sh.fred);
+  nvr = block_sum<int>(nvr, sh.ired);
+  if (tid == 0) {
+    sh.zpart = z;
+    sh.vpart = nvr;
+  }
+  cluster_sync();
+  float Z = 0.f;
+  int nvis = 0;
+  for (int r = 0; r < G; ++r) {
+    Z += dsmem_ld_f32(dsmem_map(&sh.zpart, r));
+    nvis += dsmem_ld_s32(dsmem_map(&sh.vpart, r));
+  }
+  // ---- entropy H = -sum p log(p + eps) / log L_p, temperature T
+  const float invz = 1.f / (Z + kp.eps_h);
+  float hs = 0.f;
+  for (int t = ta + tid; t < tb; t += kCalThreads) {
+    int gs;
+    const float p = sbar_of(t, gs) * invz;
+    hs += p * logf(p + kp.eps_h);
+  }
+  hs = block_sum<float>(hs, sh.fred);
+  if (tid == 0) sh.hpart = hs;
+  cluster_sync();
+  float Hs = 0.f;
+  for (int r = 0; r < G; ++r) Hs += dsmem_ld_f32(dsmem_map(&sh.hpart, r));
+  const float Hn = Lp > 1 ? -Hs / logf(static_cast<float>(Lp)) : 0.f;
+  const float T = kp.t_min + (kp.t_max - kp.t_min) * Hn;
+  const float invT = 1.f / T;
+  if (tid == 0 && g == 0 && stats) {
+    stats[0] = Hn;
+    stats[1] = T;
+    stats[4] = Z;
+    stats[5] = static_cast<float>(nvis);
+  }
+  // ---- Eq. (final_score) with Eq. (9): fused score, its descending key and
+  // the first digit of the top-B select
+  const float lam = sh.lam;
+  float* score = sv.score + static_cast<int64_t>(layer) * Lp;
+  for (int base = ta; base < tb; base += kCalThreads) {
+    const int t = base + tid;
+    uint32_t key = 0;
+    if (t < tb) {
+      int gs;
+      const float sb = sbar_of(t, gs);
+      const float beta = (1.f - lam) + lam * static_cast<float>(G) * sh.w[gs];
+      float d = 1.f;
+      const uint32_t mt = meta[t];
+      if (meta_visual(mt)) {
+        const float df = static_cast<float>(sv.cur_frame - meta_frame(mt));
+        d = kp.d_min + (1.f - kp.d_min) * expf(-kp.delta * df * sh.ph[gs]);
+      }
+      const float s = powf(fmaxf(sb * beta * d, 0.f), invT);
+      score[t] = s;
+      key = ~order_key(s);   // descending score = ascending key
+      keys[t - ta] = key;
+    }
+    hist_add(hist, t < tb, key >> 20);
+  }
 
   // ---- Sec. 3.7: global top-B, ties to the lower index
-  const int B = sv.budget;
-  if (B <= 0) return;
-  int32_t* idx = sv.idx + static_cast<int64_t>(layer) * B;
-  // descending order of s = ascending order of ~key(s)
-  uint32_t prefix = 0;
-  int rank = B - 1, less = 0;
-  for (int pass = 0; pass < 4; ++pass) {
-    const int shift = 24 - 8 * pass;
-    for (int i = tid; i < 256; i += nth) hist[i] = 0;
-    __syncthreads();
-    for (int t = tid; t < Lp; t += nth) {
-      const uint32_t u = ~order_key(score[t]);
-      if (pass == 0 || ((u ^ prefix) >> (shift + 8)) == 0) atomicAdd(&hist[(u >> shift) & 255], 1);
+  const int B = sv.budget;   // the same in every CTA of the cluster
+  if (B > 0) {
+    cluster_sync();
+    // digit 1 over the cluster: 4 bins per thread
+    {
+      int4 h = make_int4(0, 0, 0, 0);
+      for (int r = 0; r < G; ++r) {
+        const int4 q = dsmem_ld_v4(dsmem_map(hist + 4 * tid, r));
+        h.x += q.x;
+        h.y += q.y;
+        h.z += q.z;
+        h.w += q.w;
+      }
+      const int sum = (h.x + h.y) + (h.z + h.w);
+      const int excl = block_excl_scan(sum, sh.scan, nullptr);
+      const int rank = B - 1;
+      if (rank >= excl && rank < excl + sum) {
+        int c = excl, d = 0;
+        if (rank >= c + h.x) { c += h.x; d = 1; }
+        if (d == 1 && rank >= c + h.y) { c += h.y; d = 2; }
+        if (d == 2 && rank >= c + h.z) { c += h.z; d = 3; }
+        sh.tprefix = static_cast<uint32_t>(tid * 4 + d) << 20;
+        sh.trank = rank - c;
+      }
     }
     __syncthreads();
-    if (warp == 0) find_digit(hist, rank, &digit_s, &below_s);
-    __syncthreads();
-    prefix |= static_cast<uint32_t>(digit_s) << shift;
-    rank -= below_s;
-    less += below_s;
-    __syncthreads();
-  }
-  // selected: u < prefix, or u == prefix among the first rank + 1 equal keys
-  const int cs = ceil_div(Lp, nth);
-  const int t0 = min(Lp, tid * cs), t1 = min(Lp, t0 + cs);
-  int nlt = 0, neq = 0;
-  for (int t = t0; t < t1; ++t) {
-    const uint32_t u = ~order_key(score[t]);
-    nlt += u < prefix;
-    neq += u == prefix;
-  }
-  int lt_before = block_exclusive_scan(nlt, tmp, nullptr);
-  int eq_before = block_exclusive_scan(neq, tmp, nullptr);
-  for (int t = t0; t < t1; ++t) {
-    const uint32_t u = ~order_key(score[t]);
-    int pos = -1;
-    if (u < prefix) {
-      pos = lt_before + min(eq_before, rank + 1);
-      ++lt_before;
-    } else if (u == prefix) {
-      if (eq_before <= rank) pos = lt_before + eq_before;
-      ++eq_before;
+    // digits 2 and 3: histogram B (past the digit-1 bins), then histogram A
+    // again (every CTA has read the peers' digit-1 bins before the barrier)
+    for (int pass = 1; pass <= 2; ++pass) {
+      const int shift = pass == 1 ? 10 : 0;
+      int* hp = pass == 1 ? hist + kBins0 : hist;
+      const uint32_t P = sh.tprefix;
+      const int rk = sh.trank;
+      hp[tid] = 0;
+      __syncthreads();
+      for (int i = tid; i < nr; i += kCalThreads) {
+        const uint32_t u = keys[i];
+        if (((u ^ P) >> (shift + 10)) == 0) atomicAdd(&hp[(u >> shift) & 1023], 1);
+      }
+      cluster_sync();
+      int v = 0;
+      for (int r = 0; r < G; ++r) v += dsmem_ld_s32(dsmem_map(hp + tid, r));
+      const int excl = block_excl_scan(v, sh.scan, nullptr);
+      if (rk >= excl && rk < excl + v) {
+        sh.tprefix = P | (static_cast<uint32_t>(tid) << shift);
+        sh.trank = rk - excl;
+      }
+      __syncthreads();
     }
-    if (pos >= B) atomicOr(st.err, kErrIndex);   // cannot happen for a correct select
-    else if (pos >= 0) idx[pos] = t;
+    // kept: key < P, or key == P and among the first rk + 1 equal keys in
+    // position order; contiguous spans per thread keep position order
+    const uint32_t P = sh.tprefix;
+    const int rk = sh.trank;
+    const int cs = ceil_div(nr, kCalThreads);
+    const int i0 = min(nr, tid * cs), i1 = min(nr, i0 + cs);
+    int nlt = 0, neq = 0;
+    for (int i = i0; i < i1; ++i) {
+      const uint32_t u = keys[i];
+      nlt += u < P;
+      neq += u == P;
+    }
+    int tot_lt, tot_eq;
+    int lt_b = block_excl_scan(nlt, sh.scan, &tot_lt);
+    int eq_b = block_excl_scan(neq, sh.scan, &tot_eq);
+    if (tid == 0) {
+      sh.nlt = tot_lt;
+      sh.neq = tot_eq;
+    }
+    cluster_sync();
+    for (int r = 0; r < g; ++r) {
+      lt_b += dsmem_ld_s32(dsmem_map(&sh.nlt, r));
+      eq_b += dsmem_ld_s32(dsmem_map(&sh.neq, r));
+    }
+    int32_t* idx = sv.idx + static_cast<int64_t>(layer) * B;
+    for (int i = i0; i < i1; ++i) {
+      const uint32_t u = keys[i];
+      int pos = -1;
+      if (u < P) {
+        pos = lt_b + min(eq_b, rk + 1);
+        ++lt_b;
+      } else if (u == P) {
+        if (eq_b <= rk) pos = lt_b + eq_b;
+        ++eq_b;
+      }
+      if (pos >= B) atomicOr(st.err, kErrIndex);   // cannot happen for a correct select
+      else if (pos >= 0) idx[pos] = ta + i;
+    }
   }
+  cluster_sync();   // the peers' shared memory stays valid until every remote read is done
 }
 
-size_t group_stats_smem_bytes(int R, int C) { return sizeof(StatsShared) + sizeof(float) * R * C; }
+int calibrate_capacity(int K, int M, int R, int C) {
+  const size_t fixed = fixed_bytes(K, M, R, C);
+  if (fixed >= kSmemMax) return 0;
+  return static_cast<int>(((kSmemMax - fixed) / 6) & ~size_t(15));
+}
 
 cudaError_t select_configure() {
-  const int bytes = static_cast<int>(group_stats_smem_bytes(128, 128));
-  cudaError_t e = cudaFuncSetAttribute(k_group_stats<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  const int bytes = static_cast<int>(kSmemMax);
+  cudaError_t e = cudaFuncSetAttribute(k_calibrate<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(k_group_stats<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  return cudaFuncSetAttribute(k_calibrate<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
-cudaError_t group_stats_launch(const SeqBatch& b, const KParams& kp, const DevState& st, bool from_raw,
-                               cudaStream_t stream) {
-  dim3 grid(kp.G, b.nlayers, b.nseq);
-  const size_t bytes = group_stats_smem_bytes(kp.R, kp.C);
-  if (from_raw)
-    k_group_stats<true><<<grid, kStatsThreads, bytes, stream>>>(b, kp, st);
-  else
-    k_group_stats<false><<<grid, kStatsThreads, bytes, stream>>>(b, kp, st);
-  return cudaGetLastError();
-}
-
-cudaError_t select_launch(const SeqBatch& b, const KParams& kp, const DevState& st, cudaStream_t stream) {
-  dim3 grid(b.nlayers, b.nseq);
-  k_select<<<grid, kSelectThreads, 0, stream>>>(b, kp, st);
-  return cudaGetLastError();
+cudaError_t calibrate_launch(const SeqBatch& b, const KParams& kp, const DevState& st, bool from_raw, int lp_max,
+                             cudaStream_t stream) {
+  const int cap = calibrate_capacity(kp.K, kp.M, kp.R, kp.C);
+  const int capl = std::min(cap, (lp_max + 15) & ~15);
+  const size_t smem = fixed_bytes(kp.K, kp.M, kp.R, kp.C) + static_cast<size_t>(capl) * 6;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(kp.G, b.nlayers, b.nseq);
+  cfg.blockDim = dim3(kCalThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kp.G;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (from_raw) return cudaLaunchKernelEx(&cfg, k_calibrate<true>, b, kp, st, capl);
+  return cudaLaunchKernelEx(&cfg, k_calibrate<false>, b, kp, st, capl);
 }
 
 }  // namespace starkv

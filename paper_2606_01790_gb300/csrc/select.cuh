@@ -1,17 +1,18 @@
-// Launch interface of the calibration / selection kernels (select.cu).
+// Launch interface of the calibration / selection kernel (select.cu).
 #pragma once
 
 #include "common.cuh"
 
 namespace starkv {
 
-size_t group_stats_smem_bytes(int R, int C);
+// Tokens per (layer, group) row whose keys and cells the kernel keeps in
+// shared memory; longer rows use the workspace region SeqView::vis.
+int calibrate_capacity(int K, int M, int R, int C);
 cudaError_t select_configure();
-// MI_g, phi_g and the m_g update per (seq, layer, group); with from_raw the
-// kernel first pools the unpooled sums into S.
-cudaError_t group_stats_launch(const SeqBatch& b, const KParams& kp, const DevState& st, bool from_raw,
-                               cudaStream_t stream);
-// Prior, temperature, fused score and top-B per (seq, layer).
-cudaError_t select_launch(const SeqBatch& b, const KParams& kp, const DevState& st, cudaStream_t stream);
+// MI, temporal factor, prior, temperature, fused score and top-B of every
+// (seq, layer) of the batch: one cluster of G CTAs each.  With from_raw the
+// kernel first pools the unpooled group sums into S.
+cudaError_t calibrate_launch(const SeqBatch& b, const KParams& kp, const DevState& st, bool from_raw, int lp_max,
+                             cudaStream_t stream);
 
 }  // namespace starkv

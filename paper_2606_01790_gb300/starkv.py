@@ -28,7 +28,7 @@ ABI_FUNCTIONS = [
     "starkv_score_layer_noalloc",
 ]
 
-KERNELS = ["score_lse", "score_accum", "pool", "group_stats", "select", "compact"]
+KERNELS = ["score_lse", "score_accum", "pool", "calibrate", "compact"]
 
 
 class StarkvError(RuntimeError):
