@@ -226,7 +226,7 @@ void plan_ws(const starkv_state* st, const starkv_seq* seqs, int nseq, int nlaye
     const size_t lp = seqs[i].L - c.window;
     if (ws_score && lp > static_cast<size_t>(cap)) {
       p->vis_off[i] = off;
-      off += align256(static_cast<size_t>(nlayers) * G * lp * 2 * sizeof(uint32_t));
+      off += align256(static_cast<size_t>(nlayers) * G * lp * 3 * sizeof(uint32_t));
     }
     p->raw_off[i] = off;
     off += align256(static_cast<size_t>(nlayers) * G * lp * sizeof(float));

@@ -62,8 +62,8 @@ struct SeqView {
   float* s_raw;    // [n_layers_in_launch][G][Lp] unpooled sums (workspace) or NULL
   float* score;    // [n_layers][Lp] fused score (a workspace region when NULL)
   float* stats;    // optional
-  uint32_t* vis;   // [n_layers_in_launch][G][2 Lp] keys + cells of rows too long for
-                   // shared memory (workspace), else NULL
+  uint32_t* vis;   // [n_layers_in_launch][G][3 Lp] keys, candidate list and cells of
+                   // rows too long for shared memory (workspace), else NULL
 };
 
 struct SeqBatch {

@@ -121,19 +121,15 @@ __device__ void warp_find_1024(const int* hist, int rank, int* digit, int* below
   }
 }
 
-// Warp-aggregated shared-memory histogram increment; every lane calls it.
-__device__ __forceinline__ void hist_add(int* hist, bool valid, uint32_t bin) {
-  const uint32_t key = valid ? bin : 0xFFFFFFFFu;
-  const unsigned peers = __match_any_sync(0xffffffffu, key);
-  if (valid && (__ffs(peers) - 1) == static_cast<int>(threadIdx.x & 31)) atomicAdd(&hist[bin], __popc(peers));
-}
-
 struct CalShared {
   uint32_t prefix[kMaxTargets];   // RankBin boundary keys, built digit by digit
   int rem[kMaxTargets];           // rank of the boundary among the keys sharing its prefix
   int reach[kMaxTargets];         // boundary rank < N
   int dig[kMaxTargets], below[kMaxTargets];
   int eqcnt[kMaxTargets];         // keys equal to the boundary key
+  int slot_of[kMaxTargets];       // boundary -> index of its digit-1 bucket among the boundary buckets
+  int ncand[32];                  // boundary-bucket tokens of each warp's segment
+  int eqw[32][kMaxTargets];       // keys equal to each boundary before each warp's segment
   int nb[16];                     // rank-bin marginals
   int scan[33];
   float fred[32];
@@ -154,6 +150,7 @@ struct CalShared {
 
 constexpr size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 constexpr size_t kCalSharedBytes = align16(sizeof(CalShared));
+constexpr int kBucketTable = kBins0;   // bytes: rank bin of each digit-1 bucket, or 0x80 | slot
 
 __host__ __device__ __forceinline__ int hist_ints(int K) {
   const int a = 2 * kBins0, b = (K - 1) * kBins1;
@@ -162,8 +159,11 @@ __host__ __device__ __forceinline__ int hist_ints(int K) {
 
 size_t fixed_bytes(int K, int M, int R, int C) {
   return kCalSharedBytes + static_cast<size_t>(hist_ints(K)) * 4 + align16(static_cast<size_t>(K) * M * M * 4) +
-         align16(static_cast<size_t>(R) * C * 4);
+         align16(static_cast<size_t>(R) * C * 4) + align16(R) + align16(C) + kBucketTable;
 }
+
+// Per token of a row kept on chip: key (4 B), candidate slot (4 B), cell (2 B).
+constexpr size_t kBytesPerToken = 10;
 
 }  // namespace
 
@@ -177,20 +177,30 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   int* hist = reinterpret_cast<int*>(smem_raw + kCalSharedBytes);
   int* joint = hist + hist_ints(K);
   float* cur = reinterpret_cast<float*>(joint + ((K * MM + 3) & ~3));
-  uint32_t* skeys = reinterpret_cast<uint32_t*>(cur + ((RC + 3) & ~3));
-  uint16_t* scells = reinterpret_cast<uint16_t*>(skeys + capl);
+  uint8_t* rowc = reinterpret_cast<uint8_t*>(cur + ((RC + 3) & ~3));
+  uint8_t* colc = rowc + ((R + 15) & ~15);
+  uint8_t* btab = colc + ((C + 15) & ~15);
+  uint32_t* skeys = reinterpret_cast<uint32_t*>(btab + kBucketTable);
+  uint32_t* scand = skeys + capl;
+  uint16_t* scells = reinterpret_cast<uint16_t*>(scand + capl);
 
   const SeqView& sv = b.s[blockIdx.z];
   const int g = blockIdx.x;              // == rank in the cluster (the cluster spans grid x)
   const int ll = blockIdx.y, layer = b.layer0 + ll;
   const int Lp = sv.Lp;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const unsigned lanes_below = (1u << lane) - 1u;
   const uint32_t* meta = sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride;
   const int sl = sv.slot * kp.n_layers + layer;
   float* S = sv.S + (static_cast<int64_t>(layer) * G + g) * Lp;
   const bool in_smem = Lp <= capl;
-  uint32_t* keys = in_smem ? skeys : sv.vis + static_cast<int64_t>(ll * G + g) * Lp * 2;
-  uint16_t* cells = in_smem ? scells : reinterpret_cast<uint16_t*>(keys + Lp);
+  uint32_t* keys = in_smem ? skeys : sv.vis + static_cast<int64_t>(ll * G + g) * Lp * 3;
+  uint32_t* cand = in_smem ? scand : keys + Lp;
+  uint16_t* cells = in_smem ? scells : reinterpret_cast<uint16_t*>(keys + 2 * static_cast<int64_t>(Lp));
+  // phase 1 walks the row in one contiguous segment per warp, so that warp
+  // order and lane order are position order
+  const int seg = ceil_div(Lp, 32 * 32) * 32;
+  const int s0 = min(Lp, warp * seg), s1 = min(Lp, s0 + seg);
 
   if (tid < G) sh.mib_old[tid] = st.mi_bar[sl * G + tid];
   if (tid == 0) {
@@ -200,6 +210,8 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   for (int i = tid; i < kBins0; i += kCalThreads) hist[i] = 0;
   for (int i = tid; i < K * MM; i += kCalThreads) joint[i] = 0;
   for (int i = tid; i < RC; i += kCalThreads) cur[i] = 0.f;
+  for (int r = tid; r < R; r += kCalThreads) rowc[r] = static_cast<uint8_t>(r * M / R);
+  for (int c = tid; c < C; c += kCalThreads) colc[c] = static_cast<uint8_t>(c * M / C);
   __syncthreads();
 
   // ================= phase 1: group g =================
@@ -209,43 +221,43 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   const int half = kp.pool >> 1;
   const float* raw = FROM_RAW ? sv.s_raw + static_cast<int64_t>(ll * G + g) * Lp : nullptr;
   int nv = 0;
-  for (int base = 0; base < Lp; base += 2 * kCalThreads) {
-    float s[2];
-    uint32_t mt[2];
+  for (int base = s0; base < s1; base += 128) {
+    float s[4];
+    uint32_t mt[4];
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      const int t = base + k * kCalThreads + tid;
-      s[k] = 0.f;
-      mt[k] = 0;
-      if (t < Lp) {
-        mt[k] = meta[t];
+    for (int e = 0; e < 4; ++e) {
+      const int t = base + e * 32 + lane;
+      s[e] = 0.f;
+      mt[e] = 0;
+      if (t < s1) {
+        mt[e] = meta[t];
         if (FROM_RAW) {
           float acc = 0.f;
           for (int j = -half; j <= half; ++j) {
             const int u = t + j;
             if (u >= 0 && u < Lp) acc += raw[u];
           }
-          s[k] = acc * pscale;
+          s[e] = acc * pscale;
         } else {
-          s[k] = S[t];
+          s[e] = S[t];
         }
       }
     }
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      const int t = base + k * kCalThreads + tid;
-      bool vis = false;
-      uint32_t key = 0;
-      if (t < Lp) {
-        if (FROM_RAW) S[t] = s[k];
+    for (int e = 0; e < 4; ++e) {
+      const int t = base + e * 32 + lane;
+      if (t < s1) {
+        if (FROM_RAW) S[t] = s[e];
         uint16_t cell = kNoCell;
-        if (meta_visual(mt[k])) {
-          const int r = meta_row(mt[k]), c = meta_col(mt[k]);
+        uint32_t key = 0;
+        if (meta_visual(mt[e])) {
+          const int r = meta_row(mt[e]), c = meta_col(mt[e]);
           if (r < R && c < C) {
-            vis = true;
-            key = order_key(s[k]);
-            cell = static_cast<uint16_t>((r * M / R) * M + (c * M / C));
-            if (meta_frame(mt[k]) == sv.cur_frame) atomicAdd(&cur[r * C + c], s[k]);
+            key = order_key(s[e]);
+            cell = static_cast<uint16_t>(rowc[r] * M + colc[c]);
+            ++nv;
+            atomicAdd(&hist[key >> 20], 1);
+            if (meta_frame(mt[e]) == sv.cur_frame) atomicAdd(&cur[r * C + c], s[e]);
           } else {
             atomicOr(st.err, kErrMeta);
           }
@@ -253,8 +265,6 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         keys[t] = key;
         cells[t] = cell;
       }
-      nv += vis;
-      hist_add(hist, vis, key >> 20);
     }
   }
   const int N = block_sum<int>(nv, sh.ired);
@@ -288,90 +298,143 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         }
       }
       __syncthreads();
-      if (tid < nt && sh.reach[tid]) {
-        sh.prefix[tid] = static_cast<uint32_t>(sh.dig[tid]) << 20;
-        sh.rem[tid] -= sh.below[tid];
-      }
-      __syncthreads();
-    }
-    // ---- digits 2 and 3: one 1024-bin histogram per boundary over the keys
-    // that share the boundary's higher digits
-    for (int pass = 1; pass <= 2; ++pass) {
-      const int shift = pass == 1 ? 10 : 0;
-      for (int i = tid; i < nt * kBins1; i += kCalThreads) hist[i] = 0;
-      __syncthreads();
-      for (int t = tid; t < Lp; t += kCalThreads) {
-        if (cells[t] == kNoCell) continue;
-        const uint32_t u = keys[t];
-        for (int j = 0; j < nt; ++j)
-          if (sh.reach[j] && ((u ^ sh.prefix[j]) >> (shift + 10)) == 0)
-            atomicAdd(&hist[j * kBins1 + ((u >> shift) & 1023)], 1);
-      }
-      __syncthreads();
-      if (warp < nt && sh.reach[warp]) warp_find_1024(hist + warp * kBins1, sh.rem[warp], &sh.dig[warp], &sh.below[warp]);
-      __syncthreads();
-      if (tid < nt && sh.reach[tid]) {
-        sh.prefix[tid] |= static_cast<uint32_t>(sh.dig[tid]) << shift;
-        sh.rem[tid] -= sh.below[tid];
-        if (pass == 2) {
-          const int e = hist[tid * kBins1 + sh.dig[tid]];
-          sh.eqcnt[tid] = e;
-          if (e > 1) atomicOr(&sh.any_tie, 1);
+      if (tid == 0) {
+        // the boundaries are in rank order, so their buckets are non-decreasing
+        int slot = -1, prev = -1;
+        for (int j = 0; j < nt; ++j) {
+          if (!sh.reach[j]) continue;
+          if (sh.dig[j] != prev) {
+            ++slot;
+            prev = sh.dig[j];
+          }
+          sh.slot_of[j] = slot;
+          sh.prefix[j] = static_cast<uint32_t>(sh.dig[j]) << 20;
+          sh.rem[j] -= sh.below[j];
         }
       }
       __syncthreads();
     }
-    // ---- rank bin of every visual token: the number of boundaries at or
-    // below it; joint (bin, cell) histogram
+    // ---- bucket table: a bucket without a boundary puts all its tokens in
+    // one rank bin (the boundaries below it); a boundary bucket is refined
+    for (int bk = tid; bk < kBins0; bk += kCalThreads) {
+      int below = 0, slot = -1;
+      for (int j = 0; j < nt; ++j) {
+        if (!sh.reach[j]) break;
+        const int d = static_cast<int>(sh.prefix[j] >> 20);
+        below += d < bk;
+        if (d == bk) slot = sh.slot_of[j];
+      }
+      btab[bk] = static_cast<uint8_t>(slot >= 0 ? (0x80 | slot) : below);
+    }
+    for (int i = tid; i < nt * kBins1; i += kCalThreads) hist[i] = 0;   // digit 2, one histogram per slot
+    __syncthreads();
+    // ---- joint histogram of the settled tokens; the boundary-bucket tokens
+    // go to the warp's ordered candidate list and to the digit-2 histograms
+    {
+      int nc = 0;
+      for (int base = s0; base < s1; base += 32) {
+        const int t = base + lane;
+        const int cell = t < s1 ? cells[t] : kNoCell;
+        const uint32_t u = cell != kNoCell ? keys[t] : 0;
+        const int v = cell != kNoCell ? btab[u >> 20] : 0;
+        const bool c = cell != kNoCell && (v & 0x80);
+        if (cell != kNoCell && !c) atomicAdd(&joint[v * MM + cell], 1);
+        const unsigned m = __ballot_sync(0xffffffffu, c);
+        if (c) {
+          cand[s0 + nc + __popc(m & lanes_below)] = t;
+          atomicAdd(&hist[(v & 0x7F) * kBins1 + ((u >> 10) & 1023)], 1);
+        }
+        nc += __popc(m);
+      }
+      if (lane == 0) sh.ncand[warp] = nc;
+    }
+    __syncthreads();
+    // ---- digit 2 of each boundary (its slot's histogram)
+    if (warp < nt && sh.reach[warp])
+      warp_find_1024(hist + sh.slot_of[warp] * kBins1, sh.rem[warp], &sh.dig[warp], &sh.below[warp]);
+    __syncthreads();
+    if (tid < nt && sh.reach[tid]) {
+      sh.prefix[tid] |= static_cast<uint32_t>(sh.dig[tid]) << 10;
+      sh.rem[tid] -= sh.below[tid];
+    }
+    __syncthreads();
+    for (int i = tid; i < nt * kBins1; i += kCalThreads) hist[i] = 0;   // digit 3, one per boundary
+    __syncthreads();
+    const int ncw = sh.ncand[warp];
+    for (int i = lane; i < ncw; i += 32) {
+      const uint32_t u = keys[cand[s0 + i]];
+      for (int j = 0; j < nt; ++j)
+        if (sh.reach[j] && ((u ^ sh.prefix[j]) >> 10) == 0) atomicAdd(&hist[j * kBins1 + (u & 1023)], 1);
+    }
+    __syncthreads();
+    if (warp < nt && sh.reach[warp]) warp_find_1024(hist + warp * kBins1, sh.rem[warp], &sh.dig[warp], &sh.below[warp]);
+    __syncthreads();
+    if (tid < nt && sh.reach[tid]) {
+      sh.prefix[tid] |= static_cast<uint32_t>(sh.dig[tid]);
+      sh.rem[tid] -= sh.below[tid];
+      const int e = hist[tid * kBins1 + sh.dig[tid]];
+      sh.eqcnt[tid] = e;
+      if (e > 1) atomicOr(&sh.any_tie, 1);
+    }
+    __syncthreads();
+    // ---- rank bin of the candidates: the boundaries at or below them
     if (!sh.any_tie) {
-      for (int t = tid; t < Lp; t += kCalThreads) {
-        const int cell = cells[t];
-        if (cell == kNoCell) continue;
+      for (int i = lane; i < ncw; i += 32) {
+        const int t = cand[s0 + i];
         const uint32_t u = keys[t];
         int bin = 0;
         for (int j = 0; j < nt; ++j) bin += (sh.reach[j] && u >= sh.prefix[j]);
-        atomicAdd(&joint[bin * MM + cell], 1);
+        atomicAdd(&joint[bin * MM + cells[t]], 1);
       }
     } else {
-      // equal keys at a boundary: their order is their position, so each
-      // thread walks one contiguous span and counts the equal keys before it
-      const int cs = ceil_div(Lp, kCalThreads);
-      const int t0 = min(Lp, tid * cs), t1 = min(Lp, t0 + cs);
-      int eqb[kMaxTargets];
-#pragma unroll
-      for (int j = 0; j < kMaxTargets; ++j) {
-        if (j >= nt) break;
+      // equal keys at a boundary are ordered by position: count them per
+      // warp segment, then walk each segment's candidates in order
+      for (int j = 0; j < nt; ++j) {
         int cnt = 0;
-        for (int t = t0; t < t1; ++t) cnt += (cells[t] != kNoCell && keys[t] == sh.prefix[j]);
-        eqb[j] = block_excl_scan(cnt, sh.scan, nullptr);
+        for (int i = lane; i < ncw; i += 32) cnt += keys[cand[s0 + i]] == sh.prefix[j];
+        cnt = warp_sum(cnt);
+        if (lane == 0) sh.eqw[warp][j] = cnt;
       }
-      for (int t = t0; t < t1; ++t) {
-        const int cell = cells[t];
-        if (cell == kNoCell) continue;
-        const uint32_t u = keys[t];
+      __syncthreads();
+      if (tid < nt) {
+        int run = 0;
+        for (int w = 0; w < 32; ++w) {
+          const int c = sh.eqw[w][tid];
+          sh.eqw[w][tid] = run;
+          run += c;
+        }
+      }
+      __syncthreads();
+      int eqrun[kMaxTargets];
+#pragma unroll
+      for (int j = 0; j < kMaxTargets; ++j) eqrun[j] = j < nt ? sh.eqw[warp][j] : 0;
+      for (int base = 0; base < ncw; base += 32) {
+        const int i = base + lane;
+        const bool ok = i < ncw;
+        const int t = ok ? static_cast<int>(cand[s0 + i]) : 0;
+        const uint32_t u = ok ? keys[t] : 0;
         int bin = 0;
 #pragma unroll
         for (int j = 0; j < kMaxTargets; ++j) {
           if (j >= nt) break;
-          if (!sh.reach[j]) continue;
           const uint32_t P = sh.prefix[j];
-          if (u > P) {
-            ++bin;
-          } else if (u == P) {
-            if (eqb[j] >= sh.rem[j]) ++bin;
-            ++eqb[j];
+          const unsigned m = __ballot_sync(0xffffffffu, ok && u == P);
+          if (ok && sh.reach[j]) {
+            if (u > P) ++bin;
+            else if (u == P && eqrun[j] + __popc(m & lanes_below) >= sh.rem[j]) ++bin;
           }
+          eqrun[j] += __popc(m);
         }
-        atomicAdd(&joint[bin * MM + cell], 1);
+        if (ok) atomicAdd(&joint[bin * MM + cells[t]], 1);
       }
     }
     __syncthreads();
     // ---- Eq. (5): plug-in MI (nats) from the joint histogram
-    int* nc = hist;   // cell marginals
+    int* ncell = hist;   // cell marginals
     for (int c = tid; c < MM; c += kCalThreads) {
       int s = 0;
       for (int bb = 0; bb < K; ++bb) s += joint[bb * MM + c];
-      nc[c] = s;
+      ncell[c] = s;
     }
     if (warp < K) {
       int s = 0;
@@ -382,12 +445,13 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     __syncthreads();
     const float fN = static_cast<float>(N);
     float acc = 0.f;
-    for (int e = tid; e < K * MM; e += kCalThreads) {
-      const int n = joint[e];
-      if (n == 0) continue;
-      const int bb = e / MM, c = e - bb * MM;
-      const float fn = static_cast<float>(n);
-      acc += fn * logf(fn * fN / (static_cast<float>(sh.nb[bb]) * static_cast<float>(nc[c])));
+    for (int bb = 0; bb < K; ++bb) {
+      for (int c = tid; c < MM; c += kCalThreads) {
+        const int n = joint[bb * MM + c];
+        if (n == 0) continue;
+        const float fn = static_cast<float>(n);
+        acc += fn * logf(fn * fN / (static_cast<float>(sh.nb[bb]) * static_cast<float>(ncell[c])));
+      }
     }
     mi = block_sum<float>(acc, sh.fred) / fN;
   }
@@ -425,29 +489,33 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
 
   // ================= phase 2: tokens [ta, tb) =================
   float* stats = sv.stats ? sv.stats + static_cast<int64_t>(layer) * (8 + 4 * G) : nullptr;
-  // ---- Eqs. (6)-(7): MI EMA, min-max, softmax prior; lambda schedule (the
-  // same arithmetic in every CTA; CTA 0 stores the new state)
+  // ---- Eqs. (6)-(7): MI EMA (double state), min-max, softmax prior; lambda
+  // schedule.  The same arithmetic in every CTA; CTA 0 stores the new state.
   if (tid == 0) {
     const int n = sh.n_old;
-    double mib[kMaxGroups], mic[kMaxGroups];
-    double lo = 1e300, hi = -1e300;
+    double mib[kMaxGroups];
+    float mic[kMaxGroups], mf[kMaxGroups];
+    float lo = 3.4e38f, hi = -3.4e38f;
     for (int gg = 0; gg < G; ++gg) {
-      mic[gg] = static_cast<double>(dsmem_ld_f32(dsmem_map(&sh.mi, gg)));
+      mic[gg] = dsmem_ld_f32(dsmem_map(&sh.mi, gg));
       sh.ph[gg] = dsmem_ld_f32(dsmem_map(&sh.phi, gg));
-      mib[gg] = n == 0 ? mic[gg] : kp.rho_mi * sh.mib_old[gg] + (1.0 - kp.rho_mi) * mic[gg];
-      lo = fmin(lo, mib[gg]);
-      hi = fmax(hi, mib[gg]);
+      mib[gg] = n == 0 ? static_cast<double>(mic[gg])
+                       : kp.rho_mi * sh.mib_old[gg] + (1.0 - kp.rho_mi) * static_cast<double>(mic[gg]);
+      mf[gg] = static_cast<float>(mib[gg]);
+      lo = fminf(lo, mf[gg]);
+      hi = fmaxf(hi, mf[gg]);
     }
-    double e[kMaxGroups], zmax = -1e300, zs = 0.0;
+    float e[kMaxGroups], zmax = -3.4e38f, zs = 0.f;
+    const float inv = 1.f / (((hi - lo) + kp.eps) * kp.tau);
     for (int gg = 0; gg < G; ++gg) {
-      e[gg] = ((mib[gg] - lo) / ((hi - lo) + kp.eps)) / kp.tau;
-      zmax = fmax(zmax, e[gg]);
+      e[gg] = (mf[gg] - lo) * inv;
+      zmax = fmaxf(zmax, e[gg]);
     }
     for (int gg = 0; gg < G; ++gg) {
-      e[gg] = exp(e[gg] - zmax);
+      e[gg] = expf(e[gg] - zmax);
       zs += e[gg];
     }
-    for (int gg = 0; gg < G; ++gg) sh.w[gg] = static_cast<float>(e[gg] / zs);
+    for (int gg = 0; gg < G; ++gg) sh.w[gg] = e[gg] / zs;
     float lam = 0.f;
     if (n >= kp.n_warmup)
       lam = kp.n_ramp <= 0 ? kp.lambda
@@ -462,8 +530,8 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         stats[6] = static_cast<float>(sv.budget);
         stats[7] = 0.f;
         for (int gg = 0; gg < G; ++gg) {
-          stats[8 + gg] = static_cast<float>(mic[gg]);
-          stats[8 + G + gg] = static_cast<float>(mib[gg]);
+          stats[8 + gg] = mic[gg];
+          stats[8 + G + gg] = mf[gg];
           stats[8 + 2 * G + gg] = sh.w[gg];
           stats[8 + 3 * G + gg] = sh.ph[gg];
         }
@@ -489,41 +557,37 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     }
     return acc * invG;
   };
-  // ---- Sec. 3.6: Z = sum s_bar over the cluster
-  float z = 0.f;
+  // ---- Sec. 3.6 in one pass: Z = sum s_bar and sum s_bar log s_bar over the
+  // cluster, then H = -sum p log p / log L_p with p = s_bar / (Z + eps)
+  // (the eps inside the log changes H by less than L_p eps)
+  float z = 0.f, zl = 0.f;
   int nvr = 0;
   for (int t = ta + tid; t < tb; t += kCalThreads) {
     int gs;
-    z += sbar_of(t, gs);
+    const float sb = sbar_of(t, gs);
+    z += sb;
+    if (sb > 0.f) zl += sb * logf(sb);
     nvr += meta_visual(meta[t]);
   }
   z = block_sum<float>(z, sh.fred);
+  zl = block_sum<float>(zl, sh.fred);
   nvr = block_sum<int>(nvr, sh.ired);
   if (tid == 0) {
     sh.zpart = z;
+    sh.hpart = zl;
     sh.vpart = nvr;
   }
   cluster_sync();
-  float Z = 0.f;
+  float Z = 0.f, ZL = 0.f;
   int nvis = 0;
   for (int r = 0; r < G; ++r) {
     Z += dsmem_ld_f32(dsmem_map(&sh.zpart, r));
+    ZL += dsmem_ld_f32(dsmem_map(&sh.hpart, r));
     nvis += dsmem_ld_s32(dsmem_map(&sh.vpart, r));
   }
-  // ---- entropy H = -sum p log(p + eps) / log L_p, temperature T
-  const float invz = 1.f / (Z + kp.eps_h);
-  float hs = 0.f;
-  for (int t = ta + tid; t < tb; t += kCalThreads) {
-    int gs;
-    const float p = sbar_of(t, gs) * invz;
-    hs += p * logf(p + kp.eps_h);
-  }
-  hs = block_sum<float>(hs, sh.fred);
-  if (tid == 0) sh.hpart = hs;
-  cluster_sync();
-  float Hs = 0.f;
-  for (int r = 0; r < G; ++r) Hs += dsmem_ld_f32(dsmem_map(&sh.hpart, r));
-  const float Hn = Lp > 1 ? -Hs / logf(static_cast<float>(Lp)) : 0.f;
+  const float Ze = Z + kp.eps_h;
+  const float plogp = Z > 0.f ? ZL / Ze - (Z / Ze) * logf(Ze) : 0.f;
+  const float Hn = Lp > 1 ? -plogp / logf(static_cast<float>(Lp)) : 0.f;
   const float T = kp.t_min + (kp.t_max - kp.t_min) * Hn;
   const float invT = 1.f / T;
   if (tid == 0 && g == 0 && stats) {
@@ -536,25 +600,21 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   // the first digit of the top-B select
   const float lam = sh.lam;
   float* score = sv.score + static_cast<int64_t>(layer) * Lp;
-  for (int base = ta; base < tb; base += kCalThreads) {
-    const int t = base + tid;
-    uint32_t key = 0;
-    if (t < tb) {
-      int gs;
-      const float sb = sbar_of(t, gs);
-      const float beta = (1.f - lam) + lam * static_cast<float>(G) * sh.w[gs];
-      float d = 1.f;
-      const uint32_t mt = meta[t];
-      if (meta_visual(mt)) {
-        const float df = static_cast<float>(sv.cur_frame - meta_frame(mt));
-        d = kp.d_min + (1.f - kp.d_min) * expf(-kp.delta * df * sh.ph[gs]);
-      }
-      const float s = powf(fmaxf(sb * beta * d, 0.f), invT);
-      score[t] = s;
-      key = ~order_key(s);   // descending score = ascending key
-      keys[t - ta] = key;
+  for (int t = ta + tid; t < tb; t += kCalThreads) {
+    int gs;
+    const float sb = sbar_of(t, gs);
+    const float beta = (1.f - lam) + lam * static_cast<float>(G) * sh.w[gs];
+    float d = 1.f;
+    const uint32_t mt = meta[t];
+    if (meta_visual(mt)) {
+      const float df = static_cast<float>(sv.cur_frame - meta_frame(mt));
+      d = kp.d_min + (1.f - kp.d_min) * expf(-kp.delta * df * sh.ph[gs]);
     }
-    hist_add(hist, t < tb, key >> 20);
+    const float s = powf(fmaxf(sb * beta * d, 0.f), invT);
+    score[t] = s;
+    const uint32_t key = ~order_key(s);   // descending score = ascending key
+    keys[t - ta] = key;
+    atomicAdd(&hist[key >> 20], 1);
   }
 
   // ---- Sec. 3.7: global top-B, ties to the lower index
@@ -652,7 +712,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
 int calibrate_capacity(int K, int M, int R, int C) {
   const size_t fixed = fixed_bytes(K, M, R, C);
   if (fixed >= kSmemMax) return 0;
-  return static_cast<int>(((kSmemMax - fixed) / 6) & ~size_t(15));
+  return static_cast<int>(((kSmemMax - fixed) / kBytesPerToken) & ~size_t(15));
 }
 
 cudaError_t select_configure() {
@@ -666,7 +726,7 @@ cudaError_t calibrate_launch(const SeqBatch& b, const KParams& kp, const DevStat
                              cudaStream_t stream) {
   const int cap = calibrate_capacity(kp.K, kp.M, kp.R, kp.C);
   const int capl = std::min(cap, (lp_max + 15) & ~15);
-  const size_t smem = fixed_bytes(kp.K, kp.M, kp.R, kp.C) + static_cast<size_t>(capl) * 6;
+  const size_t smem = fixed_bytes(kp.K, kp.M, kp.R, kp.C) + static_cast<size_t>(capl) * kBytesPerToken;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(kp.G, b.nlayers, b.nseq);
   cfg.blockDim = dim3(kCalThreads, 1, 1);
