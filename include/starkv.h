@@ -182,7 +182,7 @@ starkv_status starkv_score_layer(starkv_state* st, int32_t layer, const starkv_s
  * zero): calls that may overlap on the GPU (different streams, or threads
  * without ordering) race on it and must not be issued.  A batch whose scratch
  * would exceed 16 MiB is rejected with STARKV_ERR_UNSUPPORTED before any
- * launch (about 1.1 MB per sequence at the 5-screenshot UI-TARS shape); kernel
+ * launch (about 1.8 MB per sequence at the 5-screenshot UI-TARS shape); kernel
  * timing must be off (it creates CUDA events). */
 starkv_status starkv_score_layer_noalloc(starkv_state* st, int32_t layer, const starkv_seq* seqs,
                                          int32_t nseq, void* stream);

@@ -18,6 +18,7 @@ constexpr int kMaxBatch = 32;       // sequences per launch (kernel-parameter ar
 constexpr int kMaxBins = 64;        // K rank bins
 constexpr int kMaxHist = 4096;      // K * M^2
 constexpr int kMaxGrid = 16384;     // R * C
+constexpr int kRawCopies = 4;       // unpooled group sums: one copy per pass-2 column quarter
 
 // device error word bits
 constexpr uint32_t kErrTimeout = 1u;
@@ -59,7 +60,7 @@ struct SeqView {
   uint32_t* meta_out;
   int32_t* idx;
   float* S;        // [n_layers][G][Lp] (a workspace region when the caller passed NULL)
-  float* s_raw;    // [n_layers_in_launch][G][Lp] unpooled sums (workspace) or NULL
+  float* s_raw;    // [n_layers_in_launch][G][kRawCopies][Lp] unpooled sums (workspace) or NULL
   float* score;    // [n_layers][Lp] fused score (a workspace region when NULL)
   float* stats;    // optional
   uint32_t* vis;   // [n_layers_in_launch][G][3 Lp] keys, candidate list and cells of

@@ -7,20 +7,24 @@
 // The softmax normaliser of a window row spans every past key, so the work is
 // done in two passes over the same key tiles:
 //   pass 1 (k_score_lse):   rows (query, head) on TMEM lanes, 128 keys per MMA
-//                           column block; each thread keeps an online
-//                           (max, sum-of-exp2) for its row over its key range
-//                           and writes one partial per (row, piece).
+//                           column block; each thread keeps a (reference,
+//                           sum of exp2) pair for its row over its keys and
+//                           one partial per (row, piece) is written.
 //   pass 2 (k_score_accum): keys on TMEM lanes (M = 128), the group's window
 //                           rows on columns (N <= 256); each thread sums
 //                           exp2(z * log2e/sqrt(d) - lse2[col]) over its
 //                           columns, so the per-key group sum needs no
-//                           cross-thread reduction.  The score matrix never
+//                           cross-lane reduction.  The score matrix never
 //                           leaves the chip.
 // Both passes split the flattened (seq, layer, group, key tile) space into one
 // contiguous range per CTA (persistent grid <= #SMs), so a CTA reloads the
 // group's queries only when its range crosses into a new (seq, layer, group)
-// row.  Warp roles: warp 0 TMA producer, warp 1 MMA issuer (+ TMEM owner),
-// warps 4..11 epilogue (two warpgroups).
+// row ("piece").  Warp roles: warp 0 TMA producer, warp 1 MMA issuer (+ TMEM
+// owner), warps 4..19 epilogue: four warpgroups that all work on every tile,
+// so the 32-bit exp2 stream (the bound of both passes) is spread over 16
+// warps.  Two 256-column TMEM accumulator stages let the MMA of tile i+1 run
+// under the epilogue of tile i; TMEM is read in 16-column loads with the next
+// load in flight under the arithmetic, which runs on packed fp32 pairs.
 #include "common.cuh"
 #include "ptx.cuh"
 #include "score.cuh"
@@ -33,6 +37,10 @@ constexpr int kStages = 4;                    // K-tile pipeline depth
 constexpr int kTileBytes = kTileKeys * 256;   // 128 keys x 128 bf16
 constexpr int kHalfBytes = kTileKeys * 128;   // one 64-column swizzled half
 constexpr int kTmemCols = 512;
+constexpr int kEpiWarp0 = 4;                  // first epilogue warp (warpgroup aligned)
+constexpr int kEpiWarps = 16;
+constexpr int kEpiThreads = 32 * kEpiWarps;
+constexpr uint32_t kFull = 0xffffffffu;
 
 struct TileCoord {
   int s, l, g, j;
@@ -53,12 +61,45 @@ __device__ __forceinline__ TileCoord decode(const ScoreParams& p, int64_t f) {
   return c;
 }
 
-// Flat index of the first tile of the (seq, layer, group) row holding `c`.
-__device__ __forceinline__ int64_t row_first(const ScoreParams& p, const TileCoord& c) {
-  return p.seq[c.s].tile_base + static_cast<int64_t>(c.l * p.G + c.g) * p.seq[c.s].nt;
-}
 
 __device__ __forceinline__ int64_t range_begin(int64_t T, int c, int P) { return T * c / P; }
+
+// Coordinates of consecutive flat tiles [f0, f1), advanced without divisions
+// (one decode at the start).  A piece is a run of tiles of one (seq, layer,
+// group) row inside the range.
+struct TileIter {
+  int s, l, g, j, nt;
+  int64_t f, fe;
+  __device__ void init(const ScoreParams& p, int64_t f0, int64_t f1) {
+    f = f0;
+    fe = f1;
+    s = l = g = j = nt = 0;
+    if (f >= fe) return;
+    const TileCoord c = decode(p, f0);
+    s = c.s;
+    l = c.l;
+    g = c.g;
+    j = c.j;
+    nt = p.seq[s].nt;
+  }
+  __device__ bool valid() const { return f < fe; }
+  __device__ bool first(int64_t fb) const { return f == fb || j == 0; }
+  __device__ bool last() const { return f + 1 == fe || j + 1 == nt; }
+  __device__ void next(const ScoreParams& p) {
+    ++f;
+    if (f >= fe) return;
+    if (++j < nt) return;
+    j = 0;
+    if (++g < p.G) return;
+    g = 0;
+    if (++l < p.nlayers) return;
+    l = 0;
+    do {
+      ++s;
+    } while (s + 1 < p.nseq && p.seq[s].nt == 0);
+    nt = p.seq[s].nt;
+  }
+};
 
 struct SmemCtl {
   uint64_t k_full[kStages];
@@ -88,7 +129,7 @@ __device__ __forceinline__ void ctl_init(SmemCtl* ctl) {
   }
   for (int i = 0; i < 2; ++i) {
     mbar_init(&ctl->t_full[i], 1);
-    mbar_init(&ctl->t_empty[i], 8);   // one arrival per epilogue warp
+    mbar_init(&ctl->t_empty[i], kEpiWarps);   // one arrival per epilogue warp
   }
   mbar_init(&ctl->q_full, 1);
   mbar_init(&ctl->q_empty, 1);
@@ -105,16 +146,13 @@ __device__ void producer_loop(const ScoreParams& p, SmemCtl* ctl, uint8_t* sQ, u
                               int64_t fb, int64_t fe) {
   const uint64_t pol_k = PASS == 1 ? policy_evict_last() : policy_evict_first();
   int it = 0, pc = 0;
-  int64_t cur_row = -1;
   int last_q_pc = -1;
   int last_it[kStages];
   for (int i = 0; i < kStages; ++i) last_it[i] = -1;
-  for (int64_t f = fb; f < fe; ++f) {
+  TileIter c;
+  for (c.init(p, fb, fe); c.valid(); c.next(p)) {
     if (ctl->abort) break;
-    const TileCoord c = decode(p, f);
-    const int64_t row = row_first(p, c);
-    if (row != cur_row) {
-      cur_row = row;
+    if (c.first(fb)) {
       if (!mbar_wait(&ctl->q_empty, (pc & 1) ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
       const int zq = p.layer0 + c.l;
       if (PASS == 1) {
@@ -157,14 +195,11 @@ __device__ void mma_loop(const ScoreParams& p, SmemCtl* ctl, const uint8_t* sQ, 
   const uint32_t idesc = PASS == 1 ? idesc_bf16(128, kTileKeys) : idesc_bf16(128, p.n2);
   const uint32_t q_addr = smem_u32(sQ), k_addr = smem_u32(sK);
   int it = 0, jt = 0, pc = 0;
-  int64_t cur_row = -1;
-  for (int64_t f = fb; f < fe; ++f) {
+  TileIter c;
+  for (c.init(p, fb, fe); c.valid(); c.next(p)) {
     if (ctl->abort) break;
-    const TileCoord c = decode(p, f);
-    const int64_t row = row_first(p, c);
-    const bool last = (f + 1 == fe) || row_first(p, decode(p, f + 1)) != row;
-    if (row != cur_row) {
-      cur_row = row;
+    const bool last = c.last();
+    if (c.first(fb)) {
       if (!mbar_wait(&ctl->q_full, pc & 1, p.wait_ns)) { fail(ctl, p.err); break; }
       ++pc;
     }
@@ -230,14 +265,105 @@ __device__ float combine_lse2(const ScoreParams& p, int64_t r0, int nt, int col)
   return mx + log2f(sum);
 }
 
+
+// Streams `n` 16-column chunks of this thread's TMEM lane from `base`, one
+// load in flight under the arithmetic of the previous chunk.
+template <typename F>
+__device__ __forceinline__ void stream16(uint32_t base, int n, F&& consume) {
+  uint32_t A[16], B[16];
+  tmem_ld16_async(base, A);
+  tmem_wait16(A);
+  for (int ch = 0;; ch += 2) {
+    const bool hb = ch + 1 < n;
+    if (hb) tmem_ld16_async(base + (ch + 1) * 16, B);
+    consume(A, ch);
+    if (!hb) break;
+    tmem_wait16(B);
+    const bool ha = ch + 2 < n;
+    if (ha) tmem_ld16_async(base + (ch + 2) * 16, A);
+    consume(B, ch + 1);
+    if (!ha) break;
+    tmem_wait16(A);
+  }
+}
+
+// Adds exp2(v * sc - m) over 16 logits (packed pairs); keys at or beyond
+// `lim` (relative to the first) are masked.
+__device__ __forceinline__ float exp2_sum16(const float (&v)[16], float sc, float m) {
+  const float2 sc2 = make_float2(sc, sc), nm2 = make_float2(-m, -m);
+  float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+#pragma unroll
+  for (int i = 0; i < 16; i += 4) {
+    const float2 t0 = ffma2(make_float2(v[i], v[i + 1]), sc2, nm2);
+    const float2 t1 = ffma2(make_float2(v[i + 2], v[i + 3]), sc2, nm2);
+    acc0 = fadd2(acc0, make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
+    acc1 = fadd2(acc1, make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
+  }
+  const float2 a = fadd2(acc0, acc1);
+  return a.x + a.y;
+}
+
+__device__ __forceinline__ float max16(const float (&v)[16]) {
+  const float c0 = fmax3(v[0], v[1], v[2]), c1 = fmax3(v[3], v[4], v[5]);
+  const float c2 = fmax3(v[6], v[7], v[8]), c3 = fmax3(v[9], v[10], v[11]);
+  const float c4 = fmax3(v[12], v[13], v[14]);
+  return fmax3(fmax3(c0, c1, c2), fmax3(c3, c4, v[15]), -INFINITY);
+}
+
+// One row's (reference m, sum s of exp2(z sc - m)) over 16 more logits.  The
+// reference is the first chunk's maximum and only moves when a chunk sum
+// exceeds 2^64 (a logit more than 64 above it, or overflow); then the chunk is
+// redone against its own maximum.  Terms far below the reference underflow to
+// zero, which is below fp32 resolution of the sum anyway.
+__device__ __forceinline__ void lse_update16(const uint32_t (&r)[16], int lim, float sc, float& m, float& s) {
+  float v[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+  if (lim < 16) {
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (i >= lim) v[i] = -INFINITY;
+  }
+  if (m == -INFINITY) {
+    m = max16(v) * sc;
+    if (m == -INFINITY) return;   // every key masked so far
+  }
+  float cs = exp2_sum16(v, sc, m);
+  if (!(cs < 1.8446744e19f)) {    // 2^64, or inf
+    const float mn = fmaxf(m, max16(v) * sc);
+    s *= ex2_approx(m - mn);
+    m = mn;
+    cs = exp2_sum16(v, sc, m);
+  }
+  s += cs;
+}
+
+// sum over 16 columns of exp2(z * sc + nl[col]), nl = -lse2 of the columns
+__device__ __forceinline__ void accum16(const uint32_t (&r)[16], const float4* nl, float sc, float2& a0,
+                                        float2& a1) {
+  const float2 sc2 = make_float2(sc, sc);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float4 l = nl[i];
+    const float2 t0 = ffma2(make_float2(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1])), sc2,
+                            make_float2(l.x, l.y));
+    const float2 t1 = ffma2(make_float2(__uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3])), sc2,
+                            make_float2(l.z, l.w));
+    a0 = fadd2(a0, make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
+    a1 = fadd2(a1, make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
+  }
+}
+
 }  // namespace
 
+// 20 warps share the register file: at most 96 registers a thread.
 __global__ void __launch_bounds__(kScoreThreads, 1) k_score_lse(const __grid_constant__ ScoreParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   uint8_t* sQ = smem;                          // [2 M-tiles][2 halves][128][128 B]
   uint8_t* sK = smem + 2 * kTileBytes;         // [kStages][2 halves][128][128 B]
   SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sK + kStages * kTileBytes);
+  float2* pbuf = reinterpret_cast<float2*>(reinterpret_cast<uint8_t*>(ctl) + 256);   // [4 wg][128]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) ctl_init(ctl);
@@ -257,71 +383,72 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_lse(const __grid_con
     if (lane == 0) producer_loop<1>(p, ctl, sQ, sK, fb, fe);
   } else if (warp == 1) {
     if (lane == 0) mma_loop<1>(p, ctl, sQ, sK, tmem, fb, fe);
-  } else if (warp >= 4) {
-    const int ew = warp - 4;
-    const int mt = ew >> 2;                 // M-tile of this epilogue warpgroup
+  } else if (warp >= kEpiWarp0) {
+    const int wg = (warp - kEpiWarp0) >> 2;  // epilogue warpgroup 0..3
     const int quad = warp & 3;              // TMEM lane quadrant
-    const int r = mt * kTileKeys + quad * 32 + lane;  // window row within the group
-    const bool active = mt < p.n_mtiles;
+    const int q = quad * 32 + lane;         // TMEM lane
+    // two M tiles: warpgroup (mt, half) owns 64 keys of M tile mt;
+    // one M tile: the four warpgroups own 32 keys each
+    const bool two = p.n_mtiles == 2;
+    const int mt = two ? (wg >> 1) : 0;
+    const int kofs = two ? (wg & 1) * 64 : wg * 32;
+    const int nch = two ? 4 : 2;
+    const int r = mt * kTileKeys + q;       // window row within the group
+    const bool active = mt * kTileKeys + quad * 32 < p.rows;
+    const uint32_t base0 = tmem + (static_cast<uint32_t>(quad * 32) << 16) + mt * kTileKeys + kofs;
     const float sc = p.scale2;
     float m = -INFINITY, s = 0.f;
     int jt = 0;
-    int64_t cur_row = -1, piece_start = 0;
-    for (int64_t f = fb; f < fe; ++f) {
-      // every decision below is warp-uniform: tcgen05.ld is a .sync.aligned op
-      if (__any_sync(0xffffffffu, ctl->abort != 0)) break;
-      const TileCoord c = decode(p, f);
-      const int64_t row = row_first(p, c);
-      const bool last = (f + 1 == fe) || row_first(p, decode(p, f + 1)) != row;
-      if (row != cur_row) {
-        cur_row = row;
-        piece_start = f;
+    bool dead = false;
+    int64_t piece_start = 0;
+    // Every epilogue warp walks every tile and meets the piece-end barrier in
+    // the same order; a warp whose wait ran out keeps walking without waiting.
+    TileIter c;
+    for (c.init(p, fb, fe); c.valid(); c.next(p)) {
+      const bool last = c.last();
+      if (c.first(fb)) {
+        piece_start = c.f;
         m = -INFINITY;
         s = 0.f;
       }
       const int ts = jt & 1;
-      const uint32_t tph = (jt >> 1) & 1;
-      const bool ok = __all_sync(0xffffffffu, mbar_wait(&ctl->t_full[ts], tph, p.wait_ns));
-      if (!ok) { fail(ctl, p.err); break; }
-      tc_fence_after();
-      if (active) {
-        const int Lp = p.seq[c.s].Lp;
-        const int key0 = c.j * kTileKeys;
-        const uint32_t base = tmem + (static_cast<uint32_t>(quad * 32) << 16) + ts * 256 + mt * kTileKeys;
-#pragma unroll 1
-        for (int ch = 0; ch < 4; ++ch) {
-          float v[32];
-          tmem_ld32(base + ch * 32, v);
-          const int kc = key0 + ch * 32;
-          if (kc + 32 > Lp) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i)
-              if (kc + i >= Lp) v[i] = -INFINITY;
+      if (!dead) {
+        if (!__all_sync(kFull, mbar_wait(&ctl->t_full[ts], (jt >> 1) & 1, p.wait_ns))) {
+          fail(ctl, p.err);
+          dead = true;
+        } else {
+          tc_fence_after();
+          if (active) {
+            const int lim = p.seq[c.s].Lp - (c.j * kTileKeys + kofs);
+            stream16(base0 + ts * 256, nch, [&](const uint32_t(&v)[16], int ch) {
+              lse_update16(v, lim - ch * 16, sc, m, s);
+            });
           }
-          float cm = v[0];
-#pragma unroll
-          for (int i = 1; i < 32; ++i) cm = fmaxf(cm, v[i]);
-          const float mn = fmaxf(m, cm * sc);
-          if (mn != -INFINITY) {
-            s *= ex2_approx(m - mn);
-            float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-#pragma unroll
-            for (int i = 0; i < 32; i += 4) {
-              a0 += ex2_approx(fmaf(v[i + 0], sc, -mn));
-              a1 += ex2_approx(fmaf(v[i + 1], sc, -mn));
-              a2 += ex2_approx(fmaf(v[i + 2], sc, -mn));
-              a3 += ex2_approx(fmaf(v[i + 3], sc, -mn));
-            }
-            s += (a0 + a1) + (a2 + a3);
-            m = mn;
-          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&ctl->t_empty[ts]);
         }
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl->t_empty[ts]);
-      if (last && active && r < p.rows)
-        p.partials[piece_start * kMaxRows + r] = make_float2(m, s);
+      if (last) {
+        // merge the key parts of each row, write the piece's partial
+        pbuf[wg * 128 + q] = make_float2(m, s);
+        named_bar_sync(1, kEpiThreads);
+        const bool writer = two ? (wg & 1) == 0 : wg == 0;
+        if (writer && r < p.rows && !dead) {
+          const int n = two ? 2 : 4;
+          const int w0 = two ? wg : 0;
+          float mx = -INFINITY;
+          for (int i = 0; i < n; ++i) mx = fmaxf(mx, pbuf[(w0 + i) * 128 + q].x);
+          float sum = 0.f;
+          if (mx != -INFINITY)
+            for (int i = 0; i < n; ++i) {
+              const float2 v = pbuf[(w0 + i) * 128 + q];
+              if (v.x != -INFINITY) sum += v.y * ex2_approx(v.x - mx);
+            }
+          p.partials[piece_start * kMaxRows + r] = make_float2(mx, sum);
+        }
+        named_bar_sync(1, kEpiThreads);   // pbuf is reused by the next piece
+      }
       ++jt;
     }
   }
@@ -338,8 +465,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
   uint8_t* sQ = smem;                          // [2 halves][n2][128 B]  (<= 64 KB)
   uint8_t* sK = smem + 2 * kTileBytes;         // [kStages][2 halves][128][128 B]
   SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sK + kStages * kTileBytes);
-  float* lse2 = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ctl) + 256);  // [256]
-  float* red = lse2 + kMaxRows;                                                   // [2][128]
+  float* nlse = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ctl) + 256);  // [256] -lse2
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) ctl_init(ctl);
@@ -359,62 +485,45 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
     if (lane == 0) producer_loop<2>(p, ctl, sQ, sK, fb, fe);
   } else if (warp == 1) {
     if (lane == 0) mma_loop<2>(p, ctl, sQ, sK, tmem, fb, fe);
-  } else if (warp >= 4) {
-    const int et = threadIdx.x - 128;       // 0..255
-    const int wg = (warp - 4) >> 2;         // column half
+  } else if (warp >= kEpiWarp0) {
+    const int et = threadIdx.x - 32 * kEpiWarp0;   // 0..511
+    const int wg = et >> 7;                 // column quarter
     const int quad = warp & 3;
-    const int nch = p.n2 >> 4;              // 16-column chunks
-    const int nch0 = (nch + 1) >> 1;
-    const int ch_lo = wg == 0 ? 0 : nch0, ch_hi = wg == 0 ? nch0 : nch;
+    const int q = quad * 32 + lane;         // key within the tile
+    const int nc = p.n2 >> 4;               // 16-column chunks
+    const int ch0 = wg * (nc >> 2) + min(wg, nc & 3);
+    const int nch = (nc >> 2) + (wg < (nc & 3) ? 1 : 0);
+    const uint32_t base0 = tmem + (static_cast<uint32_t>(quad * 32) << 16) + ch0 * 16;
+    const float4* nl = reinterpret_cast<const float4*>(nlse + ch0 * 16);
     const float sc = p.scale2;
     int jt = 0;
-    int64_t cur_row = -1;
-    // Decisions to stop are taken together by all 256 epilogue threads at the
-    // per-tile named barrier, so no thread is left waiting at a barrier.
-    for (int64_t f = fb; f < fe; ++f) {
-      const TileCoord c = decode(p, f);
-      const int64_t row = row_first(p, c);
-      if (row != cur_row) {
-        cur_row = row;
-        named_bar_sync(1, 256);
-        lse2[et] = et < p.rows ? combine_lse2(p, row, p.seq[c.s].nt, et) : INFINITY;
-        named_bar_sync(1, 256);
+    bool dead = false;
+    TileIter c;
+    for (c.init(p, fb, fe); c.valid(); c.next(p)) {
+      if (c.first(fb)) {
+        named_bar_sync(1, kEpiThreads);   // the previous piece's readers are done
+        if (et < kMaxRows) nlse[et] = et < p.rows ? -combine_lse2(p, c.f - c.j, c.nt, et) : -INFINITY;
+        named_bar_sync(1, kEpiThreads);
       }
       const int ts = jt & 1;
-      const uint32_t tph = (jt >> 1) & 1;
-      const bool ok = __all_sync(0xffffffffu, mbar_wait(&ctl->t_full[ts], tph, p.wait_ns));
-      tc_fence_after();
-      const uint32_t base = tmem + (static_cast<uint32_t>(quad * 32) << 16) + ts * 256;
-      float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-#pragma unroll 1
-      for (int ch = ok ? ch_lo : ch_hi; ch < ch_hi; ++ch) {
-        float v[16];
-        tmem_ld16(base + ch * 16, v);
-        const float4* l4 = reinterpret_cast<const float4*>(lse2 + ch * 16);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const float4 l = l4[i];
-          a0 += ex2_approx(fmaf(v[4 * i + 0], sc, -l.x));
-          a1 += ex2_approx(fmaf(v[4 * i + 1], sc, -l.y));
-          a2 += ex2_approx(fmaf(v[4 * i + 2], sc, -l.z));
-          a3 += ex2_approx(fmaf(v[4 * i + 3], sc, -l.w));
+      if (!dead) {
+        if (!__all_sync(kFull, mbar_wait(&ctl->t_full[ts], (jt >> 1) & 1, p.wait_ns))) {
+          fail(ctl, p.err);
+          dead = true;
+        } else {
+          tc_fence_after();
+          float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
+          if (nch > 0)
+            stream16(base0 + ts * 256, nch, [&](const uint32_t(&v)[16], int ch) { accum16(v, nl + ch * 4, sc, a0, a1); });
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&ctl->t_empty[ts]);
+          const ScoreSeq& sq = p.seq[c.s];
+          const int key = c.j * kTileKeys + q;
+          const float2 a = fadd2(a0, a1);
+          if (key < sq.Lp)
+            sq.s_raw[(static_cast<int64_t>(c.l * p.G + c.g) * kRawCopies + wg) * sq.Lp + key] = a.x + a.y;
         }
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (ok && lane == 0) mbar_arrive(&ctl->t_empty[ts]);
-      const float acc = (a0 + a1) + (a2 + a3);
-      const int kl = quad * 32 + lane;
-      if (wg == 1) red[ts * 128 + kl] = acc;
-      if (named_bar_any(2, 256, !ok || ctl->abort != 0)) {
-        fail(ctl, p.err);
-        break;
-      }
-      if (wg == 0) {
-        const int key = c.j * kTileKeys + kl;
-        const ScoreSeq& sq = p.seq[c.s];
-        if (key < sq.Lp)
-          sq.s_raw[static_cast<int64_t>(c.l * p.G + c.g) * sq.Lp + key] = acc + red[ts * 128 + kl];
       }
       ++jt;
     }
@@ -427,26 +536,30 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
 }
 
 // S[g, t] = (G/H)(1/k) sum_{|j| <= k/2} S_raw[g, t + j]  (Eqs. 3-4; zero padding,
-// divisor k).  grid: (ceil(Lp_max / 256), nlayers * G, nseq)
+// divisor k), S_raw being the sum of its column-quarter copies.  grid: (ceil(Lp_max / 256), nlayers * G, nseq)
 __global__ void k_pool(const __grid_constant__ SeqBatch b, int G, int H, int pool) {
   const SeqView& s = b.s[blockIdx.z];
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= s.Lp) return;
   const int lg = blockIdx.y;                  // launch-local layer * G + g
   const int layer = b.layer0 + lg / G, g = lg % G;
-  const float* src = s.s_raw + static_cast<int64_t>(lg) * s.Lp;
+  const float* src = s.s_raw + static_cast<int64_t>(lg) * kRawCopies * s.Lp;
   const int half = pool >> 1;
   float acc = 0.f;
   for (int j = -half; j <= half; ++j) {
     const int u = t + j;
-    if (u >= 0 && u < s.Lp) acc += src[u];
+    if (u >= 0 && u < s.Lp) {
+      float r = 0.f;
+      for (int c = 0; c < kRawCopies; ++c) r += src[c * s.Lp + u];
+      acc += r;
+    }
   }
   const float scale = static_cast<float>(G) / static_cast<float>(H) / static_cast<float>(pool);
   s.S[(static_cast<int64_t>(layer) * G + g) * s.Lp + t] = acc * scale;
 }
 
 size_t score_smem_bytes() {
-  return 1024 + 2 * kTileBytes + kStages * kTileBytes + 256 + (kMaxRows + 256) * sizeof(float);
+  return 1024 + 2 * kTileBytes + kStages * kTileBytes + 256 + 4 * 128 * sizeof(float2);
 }
 
 cudaError_t score_configure() {

@@ -5,13 +5,13 @@
 
 namespace starkv {
 
-constexpr int kScoreThreads = 384;   // 12 warps: TMA, MMA, 2 idle, 8 epilogue
+constexpr int kScoreThreads = 640;   // 20 warps: TMA, MMA, 2 idle, 16 epilogue
 
 struct ScoreSeq {
   int Lp;              // scored (historical) keys
   int nt;              // ceil(Lp / 128) key tiles per (layer, group) row
   int64_t tile_base;   // flat index of this sequence's first tile in the launch
-  float* s_raw;        // [nlayers][G][Lp] unpooled group sums
+  float* s_raw;        // [nlayers][G][kRawCopies][Lp] unpooled group sums, one copy per column quarter
 };
 
 struct ScoreParams {

@@ -219,7 +219,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   // visual tokens, the first radix digit, the current frame on the grid
   const float pscale = static_cast<float>(G) / static_cast<float>(kp.H) / static_cast<float>(kp.pool);
   const int half = kp.pool >> 1;
-  const float* raw = FROM_RAW ? sv.s_raw + static_cast<int64_t>(ll * G + g) * Lp : nullptr;
+  const float* raw = FROM_RAW ? sv.s_raw + static_cast<int64_t>(ll * G + g) * kRawCopies * Lp : nullptr;
   int nv = 0;
   for (int base = s0; base < s1; base += 128) {
     float s[4];
@@ -235,7 +235,11 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
           float acc = 0.f;
           for (int j = -half; j <= half; ++j) {
             const int u = t + j;
-            if (u >= 0 && u < Lp) acc += raw[u];
+            if (u >= 0 && u < Lp) {
+              float r = 0.f;
+              for (int c = 0; c < kRawCopies; ++c) r += raw[c * Lp + u];
+              acc += r;
+            }
           }
           s[e] = acc * pscale;
         } else {

@@ -48,7 +48,7 @@ def test_noalloc_scoring_matches_workspace_call_on_two_calls_in_a_row():
 def test_noalloc_rejects_a_batch_beyond_its_static_scratch():
     wl = syn.WORKLOADS["uitars_layer"]
     si = syn.make_sequence(wl)
-    n = 16  # ~1.1 MB of scratch each at this shape: more than 16 MiB together
+    n = 16  # ~1.8 MB of scratch each at this shape: more than 16 MiB together
     st = sk.init_state(H.gpu_config(wl, H.hyper(), max_seqs=n))
     seqs = [H.device_seq(si, wl, slot=i, with_score=False, with_stats=False).seq for i in range(n)]
     with pytest.raises(sk.StarkvError) as e:
