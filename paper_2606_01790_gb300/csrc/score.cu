@@ -144,7 +144,7 @@ __device__ __forceinline__ void ctl_init(SmemCtl* ctl) {
 template <int PASS>
 __device__ void producer_loop(const ScoreParams& p, SmemCtl* ctl, uint8_t* sQ, uint8_t* sK,
                               int64_t fb, int64_t fe) {
-  const uint64_t pol_k = PASS == 1 ? policy_evict_last() : policy_evict_first();
+  const uint64_t pol_k = policy_evict_first();   // K streams through L2 once per pass
   int it = 0, pc = 0;
   int last_q_pc = -1;
   int last_it[kStages];
