@@ -31,6 +31,8 @@ constexpr int kMaxTargets = 15;      // K - 1 with K <= 16
 constexpr int kBins0 = 4096;         // first radix digit: key bits 31..20
 constexpr int kBins1 = 1024;         // second and third digits: bits 19..10 and 9..0
 constexpr uint16_t kNoCell = 0xFFFF; // not a (valid) visual token
+constexpr unsigned kFullMask = 0xffffffffu;
+constexpr int kBruteMax = 2048;      // largest boundary bucket ranked pairwise
 constexpr size_t kSmemMax = 227 * 1024;
 
 // Order-preserving map float -> uint32 (a < b  <=>  key(a) < key(b) for non-NaN).
@@ -85,38 +87,48 @@ __device__ int block_excl_scan(int v, int* tmp, int* total) {
   return tmp[warp] + incl - v;
 }
 
-// One warp: the bin of a 1024-bin histogram that holds rank `rank` (0-based)
+__device__ uint32_t block_min(uint32_t v, uint32_t* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  v = __reduce_min_sync(kFullMask, v);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  return __reduce_min_sync(kFullMask, red[lane]);
+}
+
+__device__ uint32_t block_max(uint32_t v, uint32_t* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  v = __reduce_max_sync(kFullMask, v);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  return __reduce_max_sync(kFullMask, red[lane]);
+}
+
+// One warp: the bin of a 256-bin histogram that holds rank `rank` (0-based)
 // and the count of keys in lower bins; written by the lane that finds it.
-__device__ void warp_find_1024(const int* hist, int rank, int* digit, int* below) {
+__device__ void warp_find_256(const int* hist, int rank, int* digit, int* below) {
   const int lane = threadIdx.x & 31;
-  const int4* h4 = reinterpret_cast<const int4*>(hist + lane * 32);
-  int v[32];
-  int sum = 0;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const int4 q = h4[i];
-    v[4 * i] = q.x;
-    v[4 * i + 1] = q.y;
-    v[4 * i + 2] = q.z;
-    v[4 * i + 3] = q.w;
-    sum += (q.x + q.y) + (q.z + q.w);
-  }
+  const int4 q0 = reinterpret_cast<const int4*>(hist + lane * 8)[0];
+  const int4 q1 = reinterpret_cast<const int4*>(hist + lane * 8)[1];
+  const int v[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
+  const int sum = ((v[0] + v[1]) + (v[2] + v[3])) + ((v[4] + v[5]) + (v[6] + v[7]));
   int incl = sum;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
-    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+    const int y = __shfl_up_sync(kFullMask, incl, o);
     if (lane >= o) incl += y;
   }
   const int excl = incl - sum;
   if (rank >= excl && rank < incl) {
     int c = excl, d = 0;
 #pragma unroll
-    for (int i = 0; i < 32; ++i)
+    for (int i = 0; i < 8; ++i)
       if (d == i && rank >= c + v[i]) {
         c += v[i];
         d = i + 1;
       }
-    *digit = lane * 32 + d;
+    *digit = lane * 8 + d;
     *below = c;
   }
 }
@@ -127,7 +139,13 @@ struct CalShared {
   int reach[kMaxTargets];         // boundary rank < N
   int dig[kMaxTargets], below[kMaxTargets];
   int eqcnt[kMaxTargets];         // keys equal to the boundary key
-  int slot_of[kMaxTargets];       // boundary -> index of its digit-1 bucket among the boundary buckets
+  int slot_of[kMaxTargets];       // boundary -> its slot (boundary bucket), in bucket order
+  int slot_off[kMaxTargets];      // slot -> first entry of its candidates in the pool
+  int slot_n[kMaxTargets];        // slot -> tokens in its bucket
+  int slot_j0[kMaxTargets];       // slot -> first boundary in it (= boundaries in lower buckets)
+  int slot_cnt[kMaxTargets];      // slot -> candidates placed so far
+  int nslot, ncand_all, brute;
+  uint32_t ured[32];
   int ncand[32];                  // boundary-bucket tokens of each warp's segment
   int eqw[32][kMaxTargets];       // keys equal to each boundary before each warp's segment
   int nb[16];                     // rank-bin marginals
@@ -152,9 +170,10 @@ constexpr size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 constexpr size_t kCalSharedBytes = align16(sizeof(CalShared));
 constexpr int kBucketTable = kBins0;   // bytes: rank bin of each digit-1 bucket, or 0x80 | slot
 
+// bucket histogram (4096) / top-B digits (4096 + 1024) / fallback digits (15 x 256)
 __host__ __device__ __forceinline__ int hist_ints(int K) {
-  const int a = 2 * kBins0, b = (K - 1) * kBins1;
-  return a > b ? a : b;
+  (void)K;
+  return kBins0 + kBins1;
 }
 
 size_t fixed_bytes(int K, int M, int R, int C) {
@@ -166,6 +185,90 @@ size_t fixed_bytes(int K, int M, int R, int C) {
 constexpr size_t kBytesPerToken = 10;
 
 }  // namespace
+
+// Exact boundaries inside the boundary buckets by a radix select over their
+// tokens (four 8-bit digits), equal keys ordered by position.  For rows whose
+// boundary buckets hold too many tokens to rank pairwise (many equal scores).
+// Adds the boundary-bucket tokens to the joint histogram.
+template <typename BucketF>
+__device__ void calibrate_refine_radix(CalShared& sh, int* hist, int* joint, const uint32_t* keys,
+                                       const uint16_t* cells, uint32_t* cand, const uint8_t* btab, int MM, int nt,
+                                       int s0, int s1, BucketF bucket_of) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const unsigned lanes_below = (1u << lane) - 1u;
+  // each warp's segment keeps its candidates in position order
+  int nc = 0;
+  for (int base = s0; base < s1; base += 32) {
+    const int t = base + lane;
+    const bool c = t < s1 && cells[t] != kNoCell && (btab[bucket_of(keys[t])] & 0x80);
+    const unsigned m = __ballot_sync(kFullMask, c);
+    if (c) cand[s0 + nc + __popc(m & lanes_below)] = static_cast<uint32_t>(t);
+    nc += __popc(m);
+  }
+  if (lane == 0) sh.ncand[warp] = nc;
+  if (tid < nt) sh.prefix[tid] = 0;
+  __syncthreads();
+  const int ncw = sh.ncand[warp];
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    const uint32_t hmask = pass == 0 ? 0u : (0xFFFFFFFFu << (shift + 8));
+    for (int i = tid; i < nt * 256; i += kCalThreads) hist[i] = 0;
+    __syncthreads();
+    for (int i = lane; i < ncw; i += 32) {
+      const uint32_t u = keys[cand[s0 + i]];
+      const int sl2 = btab[bucket_of(u)] & 0x7F;
+      for (int j = sh.slot_j0[sl2]; j < nt && sh.reach[j] && sh.slot_of[j] == sl2; ++j)
+        if (((u ^ sh.prefix[j]) & hmask) == 0) atomicAdd(&hist[j * 256 + ((u >> shift) & 255)], 1);
+    }
+    __syncthreads();
+    if (warp < nt && sh.reach[warp]) warp_find_256(hist + warp * 256, sh.rem[warp], &sh.dig[warp], &sh.below[warp]);
+    __syncthreads();
+    if (tid < nt && sh.reach[tid]) {
+      sh.prefix[tid] |= static_cast<uint32_t>(sh.dig[tid]) << shift;
+      sh.rem[tid] -= sh.below[tid];
+    }
+    __syncthreads();
+  }
+  // equal keys before each warp's segment, per boundary
+  for (int j = 0; j < nt; ++j) {
+    int cnt = 0;
+    for (int i = lane; i < ncw; i += 32) cnt += keys[cand[s0 + i]] == sh.prefix[j];
+    cnt = warp_sum(cnt);
+    if (lane == 0) sh.eqw[warp][j] = cnt;
+  }
+  __syncthreads();
+  if (tid < nt) {
+    int run = 0;
+    for (int w = 0; w < 32; ++w) {
+      const int c = sh.eqw[w][tid];
+      sh.eqw[w][tid] = run;
+      run += c;
+    }
+  }
+  __syncthreads();
+  int eqrun[kMaxTargets];
+#pragma unroll
+  for (int j = 0; j < kMaxTargets; ++j) eqrun[j] = j < nt ? sh.eqw[warp][j] : 0;
+  for (int base = 0; base < ncw; base += 32) {
+    const int i = base + lane;
+    const bool ok = i < ncw;
+    const int t = ok ? static_cast<int>(cand[s0 + i]) : 0;
+    const uint32_t u = ok ? keys[t] : 0;
+    int bin = 0;
+#pragma unroll
+    for (int j = 0; j < kMaxTargets; ++j) {
+      if (j >= nt) break;
+      const uint32_t P = sh.prefix[j];
+      const unsigned m = __ballot_sync(kFullMask, ok && u == P);
+      if (ok && sh.reach[j]) {
+        if (u > P) ++bin;
+        else if (u == P && eqrun[j] + __popc(m & lanes_below) >= sh.rem[j]) ++bin;
+      }
+      eqrun[j] += __popc(m);
+    }
+    if (ok) atomicAdd(&joint[bin * MM + cells[t]], 1);
+  }
+}
 
 template <bool FROM_RAW>
 __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_constant__ SeqBatch b,
@@ -189,7 +292,6 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   const int ll = blockIdx.y, layer = b.layer0 + ll;
   const int Lp = sv.Lp;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const unsigned lanes_below = (1u << lane) - 1u;
   const uint32_t* meta = sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride;
   const int sl = sv.slot * kp.n_layers + layer;
   float* S = sv.S + (static_cast<int64_t>(layer) * G + g) * Lp;
@@ -216,52 +318,76 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
 
   // ================= phase 1: group g =================
   // ---- one pass over the row: pooling (Eqs. 3-4), keys and cells of the
-  // visual tokens, the first radix digit, the current frame on the grid
+  // visual tokens, their key range, the current frame on the patch grid.
+  // Lane = token; the pooling window reaches the neighbouring rows of 32
+  // through shuffles (rows one and two ahead are loaded a row early).
   const float pscale = static_cast<float>(G) / static_cast<float>(kp.H) / static_cast<float>(kp.pool);
   const int half = kp.pool >> 1;
   const float* raw = FROM_RAW ? sv.s_raw + static_cast<int64_t>(ll * G + g) * kRawCopies * Lp : nullptr;
-  int nv = 0;
-  for (int base = s0; base < s1; base += 128) {
-    float s[4];
-    uint32_t mt[4];
+  auto raw_at = [&](int u) {   // sum of the column-quarter copies, zero outside the row
+    float r = 0.f;
+    if (u >= 0 && u < Lp) {
 #pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const int t = base + e * 32 + lane;
-      s[e] = 0.f;
-      mt[e] = 0;
-      if (t < s1) {
-        mt[e] = meta[t];
-        if (FROM_RAW) {
-          float acc = 0.f;
-          for (int j = -half; j <= half; ++j) {
-            const int u = t + j;
-            if (u >= 0 && u < Lp) {
-              float r = 0.f;
-              for (int c = 0; c < kRawCopies; ++c) r += raw[c * Lp + u];
-              acc += r;
-            }
-          }
-          s[e] = acc * pscale;
-        } else {
-          s[e] = S[t];
-        }
-      }
+      for (int c = 0; c < kRawCopies; ++c) r += raw[c * Lp + u];
     }
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const int t = base + e * 32 + lane;
-      if (t < s1) {
-        if (FROM_RAW) S[t] = s[e];
+    return r;
+  };
+  int nv = 0;
+  uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
+  {
+    float r_prev = 0.f, r_cur = 0.f, r_next = 0.f;
+    if (FROM_RAW) {
+      r_prev = raw_at(s0 - 32 + lane);
+      r_cur = raw_at(s0 + lane);
+      r_next = raw_at(s0 + 32 + lane);
+    }
+    uint32_t m_cur = s0 + lane < s1 ? meta[s0 + lane] : 0u;
+    for (int base = s0; base < s1; base += 32) {
+      const int t = base + lane;
+      const bool in = t < s1;
+      float r_nn = 0.f;
+      if (FROM_RAW) r_nn = raw_at(base + 64 + lane);
+      const uint32_t m_next = base + 32 + lane < s1 ? meta[base + 32 + lane] : 0u;
+      float s;
+      if (FROM_RAW) {
+        float acc = 0.f;
+        for (int j = -half; j <= half; ++j) {
+          float x;
+          if (j < 0) {
+            const int d = -j;
+            const float a = __shfl_up_sync(kFullMask, r_cur, d);
+            const float c = __shfl_sync(kFullMask, r_prev, (lane - d) & 31);
+            x = lane >= d ? a : c;
+          } else if (j > 0) {
+            const float a = __shfl_down_sync(kFullMask, r_cur, j);
+            const float c = __shfl_sync(kFullMask, r_next, (lane + j) & 31);
+            x = lane < 32 - j ? a : c;
+          } else {
+            x = r_cur;
+          }
+          acc += x;
+        }
+        s = acc * pscale;
+        r_prev = r_cur;
+        r_cur = r_next;
+        r_next = r_nn;
+      } else {
+        s = in ? S[t] : 0.f;
+      }
+      if (in) {
+        const uint32_t mt = m_cur;
+        if (FROM_RAW) S[t] = s;
         uint16_t cell = kNoCell;
         uint32_t key = 0;
-        if (meta_visual(mt[e])) {
-          const int r = meta_row(mt[e]), c = meta_col(mt[e]);
+        if (meta_visual(mt)) {
+          const int r = meta_row(mt), c = meta_col(mt);
           if (r < R && c < C) {
-            key = order_key(s[e]);
+            key = order_key(s);
             cell = static_cast<uint16_t>(rowc[r] * M + colc[c]);
             ++nv;
-            atomicAdd(&hist[key >> 20], 1);
-            if (meta_frame(mt[e]) == sv.cur_frame) atomicAdd(&cur[r * C + c], s[e]);
+            kmin = min(kmin, key);
+            kmax = max(kmax, key);
+            if (meta_frame(mt) == sv.cur_frame) atomicAdd(&cur[r * C + c], s);
           } else {
             atomicOr(st.err, kErrMeta);
           }
@@ -269,9 +395,18 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         keys[t] = key;
         cells[t] = cell;
       }
+      m_cur = m_next;
     }
   }
   const int N = block_sum<int>(nv, sh.ired);
+  kmin = block_min(kmin, sh.ured);
+  kmax = block_max(kmax, sh.ured);
+  // Sec. 3.4 RankBin, first digit: 4096 buckets spread linearly over the
+  // row's key range (monotone in the key, so bucket order is key order)
+  const float binv = 4096.f / (static_cast<float>(kmax - kmin) + 1.f);
+  auto bucket_of = [&](uint32_t u) {
+    return min(kBins0 - 1, static_cast<int>(static_cast<float>(u - kmin) * binv));
+  };
   if (tid < nt) {
     const int Rb = static_cast<int>((static_cast<int64_t>(tid + 1) * N + K - 1) / K);  // ceil(bN/K)
     sh.reach[tid] = Rb < N;
@@ -281,11 +416,16 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     sh.below[tid] = 0;
     sh.eqcnt[tid] = 0;
   }
+  if (tid < kMaxTargets) sh.slot_cnt[tid] = 0;
   __syncthreads();
 
   float mi = 0.f;
   if (N > 0) {
-    // ---- Sec. 3.4 RankBin, digit 1: one 4096-bin histogram serves every boundary
+    for (int base = s0; base < s1; base += 32) {
+      const int t = base + lane;
+      if (t < s1 && cells[t] != kNoCell) atomicAdd(&hist[bucket_of(keys[t])], 1);
+    }
+    __syncthreads();
     {
       const int4 h = reinterpret_cast<const int4*>(hist)[tid];
       const int sum = (h.x + h.y) + (h.z + h.w);
@@ -303,18 +443,27 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       }
       __syncthreads();
       if (tid == 0) {
-        // the boundaries are in rank order, so their buckets are non-decreasing
-        int slot = -1, prev = -1;
+        // boundaries are in rank order, so their buckets are non-decreasing;
+        // a slot is one boundary bucket with its candidate tokens
+        int slot = -1, prev = -1, off = 0, nmax = 0;
         for (int j = 0; j < nt; ++j) {
           if (!sh.reach[j]) continue;
           if (sh.dig[j] != prev) {
             ++slot;
             prev = sh.dig[j];
+            const int n = hist[prev];
+            sh.slot_off[slot] = off;
+            sh.slot_n[slot] = n;
+            sh.slot_j0[slot] = j;
+            off += n;
+            nmax = max(nmax, n);
           }
           sh.slot_of[j] = slot;
-          sh.prefix[j] = static_cast<uint32_t>(sh.dig[j]) << 20;
-          sh.rem[j] -= sh.below[j];
+          sh.rem[j] -= sh.below[j];   // rank inside the bucket
         }
+        sh.nslot = slot + 1;
+        sh.ncand_all = off;
+        sh.brute = off <= Lp / 2 && nmax <= kBruteMax;
       }
       __syncthreads();
     }
@@ -324,113 +473,52 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       int below = 0, slot = -1;
       for (int j = 0; j < nt; ++j) {
         if (!sh.reach[j]) break;
-        const int d = static_cast<int>(sh.prefix[j] >> 20);
-        below += d < bk;
-        if (d == bk) slot = sh.slot_of[j];
+        below += sh.dig[j] < bk;
+        if (sh.dig[j] == bk) slot = sh.slot_of[j];
       }
       btab[bk] = static_cast<uint8_t>(slot >= 0 ? (0x80 | slot) : below);
     }
-    for (int i = tid; i < nt * kBins1; i += kCalThreads) hist[i] = 0;   // digit 2, one histogram per slot
     __syncthreads();
-    // ---- joint histogram of the settled tokens; the boundary-bucket tokens
-    // go to the warp's ordered candidate list and to the digit-2 histograms
-    {
-      int nc = 0;
-      for (int base = s0; base < s1; base += 32) {
-        const int t = base + lane;
-        const int cell = t < s1 ? cells[t] : kNoCell;
-        const uint32_t u = cell != kNoCell ? keys[t] : 0;
-        const int v = cell != kNoCell ? btab[u >> 20] : 0;
-        const bool c = cell != kNoCell && (v & 0x80);
-        if (cell != kNoCell && !c) atomicAdd(&joint[v * MM + cell], 1);
-        const unsigned m = __ballot_sync(0xffffffffu, c);
-        if (c) {
-          cand[s0 + nc + __popc(m & lanes_below)] = t;
-          atomicAdd(&hist[(v & 0x7F) * kBins1 + ((u >> 10) & 1023)], 1);
-        }
-        nc += __popc(m);
+    const bool brute = sh.brute;
+    // ---- joint histogram of the settled tokens; boundary-bucket tokens go
+    // to their slot's (key, position) pool
+    uint32_t* pool = cand;   // [2 * candidates]
+    for (int base = s0; base < s1; base += 32) {
+      const int t = base + lane;
+      const int cell = t < s1 ? cells[t] : kNoCell;
+      if (cell == kNoCell) continue;
+      const uint32_t u = keys[t];
+      const int v = btab[bucket_of(u)];
+      if (!(v & 0x80)) {
+        atomicAdd(&joint[v * MM + cell], 1);
+      } else if (brute) {
+        const int sl2 = v & 0x7F;
+        const int i = sh.slot_off[sl2] + atomicAdd(&sh.slot_cnt[sl2], 1);
+        pool[2 * i] = u;
+        pool[2 * i + 1] = static_cast<uint32_t>(t);
       }
-      if (lane == 0) sh.ncand[warp] = nc;
     }
     __syncthreads();
-    // ---- digit 2 of each boundary (its slot's histogram)
-    if (warp < nt && sh.reach[warp])
-      warp_find_1024(hist + sh.slot_of[warp] * kBins1, sh.rem[warp], &sh.dig[warp], &sh.below[warp]);
-    __syncthreads();
-    if (tid < nt && sh.reach[tid]) {
-      sh.prefix[tid] |= static_cast<uint32_t>(sh.dig[tid]) << 10;
-      sh.rem[tid] -= sh.below[tid];
-    }
-    __syncthreads();
-    for (int i = tid; i < nt * kBins1; i += kCalThreads) hist[i] = 0;   // digit 3, one per boundary
-    __syncthreads();
-    const int ncw = sh.ncand[warp];
-    for (int i = lane; i < ncw; i += 32) {
-      const uint32_t u = keys[cand[s0 + i]];
-      for (int j = 0; j < nt; ++j)
-        if (sh.reach[j] && ((u ^ sh.prefix[j]) >> 10) == 0) atomicAdd(&hist[j * kBins1 + (u & 1023)], 1);
-    }
-    __syncthreads();
-    if (warp < nt && sh.reach[warp]) warp_find_1024(hist + warp * kBins1, sh.rem[warp], &sh.dig[warp], &sh.below[warp]);
-    __syncthreads();
-    if (tid < nt && sh.reach[tid]) {
-      sh.prefix[tid] |= static_cast<uint32_t>(sh.dig[tid]);
-      sh.rem[tid] -= sh.below[tid];
-      const int e = hist[tid * kBins1 + sh.dig[tid]];
-      sh.eqcnt[tid] = e;
-      if (e > 1) atomicOr(&sh.any_tie, 1);
-    }
-    __syncthreads();
-    // ---- rank bin of the candidates: the boundaries at or below them
-    if (!sh.any_tie) {
-      for (int i = lane; i < ncw; i += 32) {
-        const int t = cand[s0 + i];
-        const uint32_t u = keys[t];
-        int bin = 0;
-        for (int j = 0; j < nt; ++j) bin += (sh.reach[j] && u >= sh.prefix[j]);
-        atomicAdd(&joint[bin * MM + cells[t]], 1);
+    if (brute) {
+      // exact rank of each candidate inside its bucket by (key, position),
+      // then the boundaries of its bucket at or below that rank
+      const int nslot = sh.nslot;
+      for (int i = tid; i < sh.ncand_all; i += kCalThreads) {
+        int sl2 = 0;
+        while (sl2 + 1 < nslot && sh.slot_off[sl2 + 1] <= i) ++sl2;
+        const uint32_t ki = pool[2 * i], ti = pool[2 * i + 1];
+        const int o = sh.slot_off[sl2], n = sh.slot_n[sl2];
+        int rank = 0;
+        for (int j = o; j < o + n; ++j) {
+          const uint32_t kj = pool[2 * j], tj = pool[2 * j + 1];
+          rank += (kj < ki) || (kj == ki && tj < ti);
+        }
+        int bin = sh.slot_j0[sl2];
+        for (int j = sh.slot_j0[sl2]; j < nt && sh.reach[j] && sh.slot_of[j] == sl2; ++j) bin += sh.rem[j] <= rank;
+        atomicAdd(&joint[bin * MM + cells[ti]], 1);
       }
     } else {
-      // equal keys at a boundary are ordered by position: count them per
-      // warp segment, then walk each segment's candidates in order
-      for (int j = 0; j < nt; ++j) {
-        int cnt = 0;
-        for (int i = lane; i < ncw; i += 32) cnt += keys[cand[s0 + i]] == sh.prefix[j];
-        cnt = warp_sum(cnt);
-        if (lane == 0) sh.eqw[warp][j] = cnt;
-      }
-      __syncthreads();
-      if (tid < nt) {
-        int run = 0;
-        for (int w = 0; w < 32; ++w) {
-          const int c = sh.eqw[w][tid];
-          sh.eqw[w][tid] = run;
-          run += c;
-        }
-      }
-      __syncthreads();
-      int eqrun[kMaxTargets];
-#pragma unroll
-      for (int j = 0; j < kMaxTargets; ++j) eqrun[j] = j < nt ? sh.eqw[warp][j] : 0;
-      for (int base = 0; base < ncw; base += 32) {
-        const int i = base + lane;
-        const bool ok = i < ncw;
-        const int t = ok ? static_cast<int>(cand[s0 + i]) : 0;
-        const uint32_t u = ok ? keys[t] : 0;
-        int bin = 0;
-#pragma unroll
-        for (int j = 0; j < kMaxTargets; ++j) {
-          if (j >= nt) break;
-          const uint32_t P = sh.prefix[j];
-          const unsigned m = __ballot_sync(0xffffffffu, ok && u == P);
-          if (ok && sh.reach[j]) {
-            if (u > P) ++bin;
-            else if (u == P && eqrun[j] + __popc(m & lanes_below) >= sh.rem[j]) ++bin;
-          }
-          eqrun[j] += __popc(m);
-        }
-        if (ok) atomicAdd(&joint[bin * MM + cells[t]], 1);
-      }
+      calibrate_refine_radix(sh, hist, joint, keys, cells, cand, btab, MM, nt, s0, s1, bucket_of);
     }
     __syncthreads();
     // ---- Eq. (5): plug-in MI (nats) from the joint histogram

@@ -87,6 +87,10 @@ WORKLOADS: Dict[str, Workload] = {
     # 28 layers, 20 screenshots + 2048 text (L_p = 56,096), amplitude U[0.5, 4] per frame.
     "long": Workload("long", 4, n_layers=28, n_shots=20, n_text=2048,
                      amp_range=(0.5, 4.0)),
+    # one layer of the long shape (parity case for rows longer than the
+    # calibration kernel keeps on chip)
+    "long_layer": Workload("long_layer", 7, n_layers=1, n_shots=20, n_text=2048,
+                           amp_range=(0.5, 4.0)),
     # 16 ragged trajectories, 28 layers.
     "ragged": Workload("ragged", 5, n_layers=28, n_seqs=16, ragged=True),
     # the timed per-step workload: 28 layers of the 5-screenshot UI-TARS shape

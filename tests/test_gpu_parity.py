@@ -107,6 +107,60 @@ def test_select_stage_isolated_on_oracle_scores():
     assert ix["ok"], ix
 
 
+def _select_on_given_scores(wl, si, S32, h):
+    p = H.oracle_params(h)
+    st = sk.init_state(H.gpu_config(wl, h))
+    ds = H.device_seq(si, wl)
+    ds.seq.S.copy_(torch.from_numpy(S32)[None])
+    ws = sk.workspace(st, [ds.seq])
+    sk.select(st, 0, [ds.seq], ws)
+    torch.cuda.synchronize()
+    sk.check_device_error(st)
+    ref = H.oracle_layer(si, 0, wl, O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols), p,
+                         S_override=S32.astype(np.float64))
+    return ds, ref, p
+
+
+def test_select_with_heavy_score_ties():
+    """Scores quantised to 8 levels per group: thousands of equal keys at each
+    rank-bin boundary, ordered by position (the radix fallback of the rank
+    bins), and equal fused scores at the top-B threshold (lower index wins)."""
+    wl = syn.WORKLOADS["uitars_layer"]
+    si = syn.make_sequence(wl)
+    h = H.hyper(n_warmup=0, n_ramp=0)
+    p = H.oracle_params(h)
+    S = O.score_layer(si.q[0].double().numpy(), si.k[0].double().numpy(), wl.window, p)
+    top = S.max(axis=1, keepdims=True)
+    S32 = (np.floor(S / top * 8.0) / 8.0 * top).astype(np.float32)
+    ds, ref, p = _select_on_given_scores(wl, si, S32, h)
+    stats = ds.seq.stats[0].double().cpu().numpy()
+    G = wl.n_kv_heads
+    np.testing.assert_allclose(stats[8:8 + G], ref["mi"], rtol=1e-6)     # same bins -> same MI
+    sc = H.check_scores(ds.seq.score[0].double().cpu().numpy(), ref, ref["S"], si, 0, wl, p, rtol=1e-5)
+    assert sc["ok"], sc
+    ix = H.check_index_set(ds.seq.idx[0].cpu().numpy(), ref, si.budget, rtol=1e-5)
+    assert ix["ok"], ix
+
+
+def test_select_on_a_row_longer_than_shared_memory():
+    """20 screenshots (L_p = 56,096): the calibration kernel keeps the row's
+    keys in the workspace instead of shared memory."""
+    wl = syn.WORKLOADS["long_layer"]
+    si = syn.make_sequence(wl)
+    h = H.hyper(n_warmup=0, n_ramp=0)
+    p = H.oracle_params(h)
+    S32 = O.score_layer(si.q[0].double().numpy(), si.k[0].double().numpy(), wl.window, p).astype(np.float32)
+    ds, ref, p = _select_on_given_scores(wl, si, S32, h)
+    stats = ds.seq.stats[0].double().cpu().numpy()
+    G = wl.n_kv_heads
+    np.testing.assert_allclose(stats[8:8 + G], ref["mi"], rtol=1e-5)
+    np.testing.assert_allclose(stats[8 + 3 * G:8 + 4 * G], ref["phi"], atol=1e-6)
+    sc = H.check_scores(ds.seq.score[0].double().cpu().numpy(), ref, ref["S"], si, 0, wl, p, rtol=1e-5)
+    assert sc["ok"], sc
+    ix = H.check_index_set(ds.seq.idx[0].cpu().numpy(), ref, si.budget, rtol=1e-5)
+    assert ix["ok"], ix
+
+
 def test_carried_state_over_two_steps():
     """Second call sees a non-fresh state: MI EMA and the temporal EMA m_g act."""
     wl = syn.WORKLOADS["tiny"]
