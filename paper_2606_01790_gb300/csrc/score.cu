@@ -287,55 +287,93 @@ __device__ __forceinline__ void stream16(uint32_t base, int n, F&& consume) {
   }
 }
 
-// Adds exp2(v * sc - m) over 16 logits (packed pairs); keys at or beyond
-// `lim` (relative to the first) are masked.
-__device__ __forceinline__ float exp2_sum16(const float (&v)[16], float sc, float m) {
-  const float2 sc2 = make_float2(sc, sc), nm2 = make_float2(-m, -m);
-  float2 acc0 = make_float2(0.f, 0.f), acc1 = make_float2(0.f, 0.f);
+__device__ __forceinline__ float2 f2(uint32_t a, uint32_t b) { return make_float2(__uint_as_float(a), __uint_as_float(b)); }
+
+// a0, a1 += exp2(z * sc - m) over 16 logits given as raw TMEM words (packed pairs)
+__device__ __forceinline__ void exp2_acc16(const uint32_t (&r)[16], float2 sc2, float2 nm2, float2& a0, float2& a1) {
 #pragma unroll
   for (int i = 0; i < 16; i += 4) {
-    const float2 t0 = ffma2(make_float2(v[i], v[i + 1]), sc2, nm2);
-    const float2 t1 = ffma2(make_float2(v[i + 2], v[i + 3]), sc2, nm2);
-    acc0 = fadd2(acc0, make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
-    acc1 = fadd2(acc1, make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
+    const float2 t0 = ffma2(f2(r[i], r[i + 1]), sc2, nm2);
+    const float2 t1 = ffma2(f2(r[i + 2], r[i + 3]), sc2, nm2);
+    a0 = fadd2(a0, make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
+    a1 = fadd2(a1, make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
   }
-  const float2 a = fadd2(acc0, acc1);
-  return a.x + a.y;
 }
 
-__device__ __forceinline__ float max16(const float (&v)[16]) {
-  const float c0 = fmax3(v[0], v[1], v[2]), c1 = fmax3(v[3], v[4], v[5]);
-  const float c2 = fmax3(v[6], v[7], v[8]), c3 = fmax3(v[9], v[10], v[11]);
-  const float c4 = fmax3(v[12], v[13], v[14]);
-  return fmax3(fmax3(c0, c1, c2), fmax3(c3, c4, v[15]), -INFINITY);
+// the same over the first `lim` logits only (the ragged last tile of a row)
+__device__ __forceinline__ void exp2_acc16_masked(const uint32_t (&r)[16], int lim, float2 sc2, float2 nm2,
+                                                  float2& a0, float2& a1) {
+#pragma unroll
+  for (int i = 0; i < 16; i += 2) {
+    const float2 t = ffma2(f2(r[i], r[i + 1]), sc2, nm2);
+    a0 = fadd2(a0, make_float2(i < lim ? ex2_approx(t.x) : 0.f, i + 1 < lim ? ex2_approx(t.y) : 0.f));
+  }
 }
 
-// One row's (reference m, sum s of exp2(z sc - m)) over 16 more logits.  The
-// reference is the first chunk's maximum and only moves when a chunk sum
-// exceeds 2^64 (a logit more than 64 above it, or overflow); then the chunk is
-// redone against its own maximum.  Terms far below the reference underflow to
-// zero, which is below fp32 resolution of the sum anyway.
-__device__ __forceinline__ void lse_update16(const uint32_t (&r)[16], int lim, float sc, float& m, float& s) {
-  float v[16];
+// maximum over the first `lim` of 16 logits (-inf when none)
+__device__ __forceinline__ float max16_masked(const uint32_t (&r)[16], int lim) {
+  float mx = -INFINITY;
 #pragma unroll
-  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-  if (lim < 16) {
-#pragma unroll
-    for (int i = 0; i < 16; ++i)
-      if (i >= lim) v[i] = -INFINITY;
+  for (int i = 0; i < 16; ++i)
+    if (i < lim) mx = fmaxf(mx, __uint_as_float(r[i]));
+  return mx;
+}
+
+// Rare path of lse_tile: a logit more than 64 above the reference (or an
+// overflow) in some lane of the warp; every lane redoes the tile against
+// max(its reference, its tile maximum), which leaves a lane without overflow
+// with the same sum.
+__device__ __noinline__ void lse_tile_rescale(uint32_t base, int n, int lim, float sc, float& m, float& s) {
+  float mx = -INFINITY;
+  for (int ch = 0; ch < n; ++ch) {
+    uint32_t r[16];
+    tmem_ld16_async(base + ch * 16, r);
+    tmem_wait16(r);
+    mx = fmaxf(mx, max16_masked(r, lim - ch * 16));
   }
-  if (m == -INFINITY) {
-    m = max16(v) * sc;
-    if (m == -INFINITY) return;   // every key masked so far
+  const float mn = fmaxf(m, mx * sc);
+  s *= ex2_approx(m - mn);
+  m = mn;
+  const float2 sc2 = make_float2(sc, sc), nm2 = make_float2(-m, -m);
+  float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
+  for (int ch = 0; ch < n; ++ch) {
+    uint32_t r[16];
+    tmem_ld16_async(base + ch * 16, r);
+    tmem_wait16(r);
+    exp2_acc16_masked(r, lim - ch * 16, sc2, nm2, a0, a1);
   }
-  float cs = exp2_sum16(v, sc, m);
-  if (!(cs < 1.8446744e19f)) {    // 2^64, or inf
-    const float mn = fmaxf(m, max16(v) * sc);
-    s *= ex2_approx(m - mn);
-    m = mn;
-    cs = exp2_sum16(v, sc, m);
+  const float2 a = fadd2(a0, a1);
+  s += a.x + a.y;
+}
+
+// One row's running (reference m, sum s of exp2(z sc - m)) over this thread's
+// `nch` 16-key chunks of one tile, `lim` of which keys are valid.  The
+// reference is set from the first chunk a piece sees and moves only when a
+// tile's sum exceeds 2^64 (a logit more than 64 above it, or overflow); that
+// tile is then redone against its own maximum.  Terms far below the reference
+// underflow to zero, below the fp32 resolution of the sum.
+__device__ __forceinline__ void lse_tile(uint32_t base, int nch, int lim, float sc, float& m, float& s) {
+  if (lim <= 0) return;
+  const int n = min(nch, (lim + 15) >> 4);
+  const bool full = lim >= nch * 16;
+  const float2 sc2 = make_float2(sc, sc);
+  // TMEM loads are warp-collective: every branch around them is warp-uniform
+  if (__any_sync(kFull, m == -INFINITY)) {
+    uint32_t r[16];
+    tmem_ld16_async(base, r);
+    tmem_wait16(r);
+    if (m == -INFINITY) m = max16_masked(r, lim) * sc;
   }
-  s += cs;
+  const float2 nm2 = make_float2(-m, -m);
+  float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
+  if (full)
+    stream16(base, n, [&](const uint32_t(&r)[16], int) { exp2_acc16(r, sc2, nm2, a0, a1); });
+  else
+    stream16(base, n, [&](const uint32_t(&r)[16], int ch) { exp2_acc16_masked(r, lim - ch * 16, sc2, nm2, a0, a1); });
+  const float2 a = fadd2(a0, a1);
+  const float cs = a.x + a.y;
+  if (__all_sync(kFull, cs < 1.8446744e19f)) s += cs;   // below 2^64: the common case
+  else lse_tile_rescale(base, n, lim, sc, m, s);       // the whole warp, each lane from its own m
 }
 
 // sum over 16 columns of exp2(z * sc + nl[col]), nl = -lse2 of the columns
@@ -418,12 +456,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_lse(const __grid_con
           dead = true;
         } else {
           tc_fence_after();
-          if (active) {
-            const int lim = p.seq[c.s].Lp - (c.j * kTileKeys + kofs);
-            stream16(base0 + ts * 256, nch, [&](const uint32_t(&v)[16], int ch) {
-              lse_update16(v, lim - ch * 16, sc, m, s);
-            });
-          }
+          if (active) lse_tile(base0 + ts * 256, nch, p.seq[c.s].Lp - (c.j * kTileKeys + kofs), sc, m, s);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&ctl->t_empty[ts]);

@@ -55,6 +55,29 @@ def test_score_layer_matches_oracle(name):
     assert abs(S_gpu.sum(axis=1).mean() - S_ref.sum(axis=1).mean()) < 1e-4 * S_ref.sum(axis=1).mean()
 
 
+def test_score_layer_with_wide_logits():
+    """Queries scaled by 32 (exact in bf16): a row's logits span far more than
+    2^64 in exp2 units, so the running reference of pass 1 has to move after
+    its first chunk (the rescale path)."""
+    wl = syn.WORKLOADS["uitars_layer"]
+    si = syn.make_sequence(wl)
+    si.q = si.q * 32
+    h = H.hyper()
+    st = sk.init_state(H.gpu_config(wl, h))
+    ds = H.device_seq(si, wl)
+    ws = sk.workspace(st, [ds.seq])
+    sk.score_layer(st, 0, [ds.seq], ws)
+    torch.cuda.synchronize()
+    sk.check_device_error(st)
+    S_gpu = ds.seq.S[0].double().cpu().numpy()
+    S_ref = O.score_layer(si.q[0].double().numpy(), si.k[0].double().numpy(), wl.window, H.oracle_params(h))
+    # fp32 exp2 flushes terms below 2^-126 of a row's reference: an absolute
+    # floor far below any score that can matter
+    err = np.abs(S_gpu - S_ref)
+    assert np.all(err <= 1e-3 * np.abs(S_ref) + 1e-9 * S_ref.max()), float((err / np.abs(S_ref)).max())
+    assert abs(S_gpu.sum() - S_ref.sum()) < 1e-4 * S_ref.sum()
+
+
 @pytest.mark.parametrize("name", ["tiny", "uitars_layer"])
 @pytest.mark.parametrize("sched", ["paper", "prior_on"])
 def test_step_matches_oracle(name, sched):
