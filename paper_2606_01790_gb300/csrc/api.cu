@@ -283,6 +283,9 @@ starkv_status run_score(starkv_state* st, const starkv_seq* seqs, int i0, int i1
   p.rows = (H / G) * w;
   p.n2 = (p.rows + 15) & ~15;
   p.n_mtiles = (p.rows + kTileKeys - 1) / kTileKeys;
+  p.q_rows = p.n2;
+  p.kstages = score_kstages(p.q_rows);
+  if (p.kstages < 2) return set_error(STARKV_ERR_UNSUPPORTED, "window rows per group too large for shared memory");
   p.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(kHeadDim)));
   int64_t tiles = 0;
   for (int i = i0; i < i1; ++i) {
@@ -296,7 +299,12 @@ starkv_status run_score(starkv_state* st, const starkv_seq* seqs, int i0, int i1
     tiles += static_cast<int64_t>(nlayers) * G * ss.nt;
     if (ss.nt == 0) continue;
     if ((s = encode_3d(&p.tmk[i - i0], q.k, kHeadDim, q.L, static_cast<uint64_t>(c.n_layers) * G, kTileKeys)) != STARKV_OK) return s;
-    if ((s = encode_3d(&p.tmq1[i - i0], q.q, kHeadDim, static_cast<uint64_t>(H) * w, c.n_layers, kTileKeys)) != STARKV_OK) return s;
+    const uint64_t qrows = static_cast<uint64_t>(H) * w;
+    if ((s = encode_3d(&p.tmqa[i - i0], q.q, kHeadDim, qrows, c.n_layers, std::min(p.rows, kTileKeys))) != STARKV_OK)
+      return s;
+    if (p.rows > kTileKeys &&
+        (s = encode_3d(&p.tmqb[i - i0], q.q, kHeadDim, qrows, c.n_layers, p.rows - kTileKeys)) != STARKV_OK)
+      return s;
     if ((s = encode_3d(&p.tmq2[i - i0], q.q, kHeadDim, static_cast<uint64_t>(H) * w, c.n_layers, p.n2)) != STARKV_OK) return s;
   }
   if (tiles == 0) return STARKV_OK;

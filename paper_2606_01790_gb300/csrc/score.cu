@@ -33,10 +33,12 @@ namespace starkv {
 
 namespace {
 
-constexpr int kStages = 4;                    // K-tile pipeline depth
+constexpr int kMaxStages = 5;                 // K-tile pipeline depth (at most)
+constexpr size_t kSmemLimit = 227 * 1024;
 constexpr int kTileBytes = kTileKeys * 256;   // 128 keys x 128 bf16
 constexpr int kHalfBytes = kTileKeys * 128;   // one 64-column swizzled half
 constexpr int kTmemCols = 512;
+constexpr int kMmaThreads = 2;                // MMA issuers (warps 1 and 2): even / odd tiles
 constexpr int kEpiWarp0 = 4;                  // first epilogue warp (warpgroup aligned)
 constexpr int kEpiWarps = 16;
 constexpr int kEpiThreads = 32 * kEpiWarps;
@@ -102,8 +104,8 @@ struct TileIter {
 };
 
 struct SmemCtl {
-  uint64_t k_full[kStages];
-  uint64_t k_empty[kStages];
+  uint64_t k_full[kMaxStages];
+  uint64_t k_empty[kMaxStages];
   uint64_t t_full[2];
   uint64_t t_empty[2];
   uint64_t q_full;
@@ -122,8 +124,8 @@ __device__ __forceinline__ void fail(SmemCtl* ctl, uint32_t* err) {
   atomicOr(err, kErrTimeout);
 }
 
-__device__ __forceinline__ void ctl_init(SmemCtl* ctl) {
-  for (int i = 0; i < kStages; ++i) {
+__device__ __forceinline__ void ctl_init(SmemCtl* ctl, int kstages) {
+  for (int i = 0; i < kstages; ++i) {
     mbar_init(&ctl->k_full[i], 1);
     mbar_init(&ctl->k_empty[i], 1);
   }
@@ -132,110 +134,129 @@ __device__ __forceinline__ void ctl_init(SmemCtl* ctl) {
     mbar_init(&ctl->t_empty[i], kEpiWarps);   // one arrival per epilogue warp
   }
   mbar_init(&ctl->q_full, 1);
-  mbar_init(&ctl->q_empty, 1);
-  mbar_init(&ctl->drain, 1);
+  mbar_init(&ctl->q_empty, kMmaThreads);   // each MMA thread commits once per piece
+  mbar_init(&ctl->drain, kMmaThreads);
   ctl->abort = 0;
   fence_mbar_init();
 }
 
-// TMA producer shared by both passes.  Q tile: `q_boxes` boxes of (64, q_box_rows)
-// rows starting at row g*rows + b*q_box_rows, halves interleaved as the pass
-// expects; K tile: 128 keys as two 64-column halves.
+// TMA producer shared by both passes.  Q: [2 halves][q_rows][128 B]; pass 1
+// loads the group's rows as a 128-row box and a (rows - 128)-row box per half,
+// pass 2 one n2-row box per half.  K tile: 128 keys as two 64-column halves.
 template <int PASS>
 __device__ void producer_loop(const ScoreParams& p, SmemCtl* ctl, uint8_t* sQ, uint8_t* sK,
                               int64_t fb, int64_t fe) {
   const uint64_t pol_k = policy_evict_first();   // K streams through L2 once per pass
-  int it = 0, pc = 0;
+  const int qhalf = p.q_rows * 128;
+  int stage = 0, phase = 0, pc = 0;
   int last_q_pc = -1;
-  int last_it[kStages];
-  for (int i = 0; i < kStages; ++i) last_it[i] = -1;
+  int last_ph[kMaxStages];
+  for (int i = 0; i < kMaxStages; ++i) last_ph[i] = -1;
   TileIter c;
   for (c.init(p, fb, fe); c.valid(); c.next(p)) {
     if (ctl->abort) break;
     if (c.first(fb)) {
       if (!mbar_wait(&ctl->q_empty, (pc & 1) ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
-      const int zq = p.layer0 + c.l;
+      const int zq = p.layer0 + c.l, y = c.g * p.rows;
       if (PASS == 1) {
-        mbar_arrive_expect_tx(&ctl->q_full, p.n_mtiles * kTileBytes);
-        for (int mt = 0; mt < p.n_mtiles; ++mt)
-          for (int h = 0; h < 2; ++h)
-            tma_load_3d(sQ + mt * kTileBytes + h * kHalfBytes, &p.tmq1[c.s], &ctl->q_full, h * 64,
-                        c.g * p.rows + mt * kTileKeys, zq);
+        mbar_arrive_expect_tx(&ctl->q_full, p.rows * 256);
+        for (int h = 0; h < 2; ++h) {
+          tma_load_3d(sQ + h * qhalf, &p.tmqa[c.s], &ctl->q_full, h * 64, y, zq);
+          if (p.rows > kTileKeys)
+            tma_load_3d(sQ + h * qhalf + kTileKeys * 128, &p.tmqb[c.s], &ctl->q_full, h * 64, y + kTileKeys, zq);
+        }
       } else {
         mbar_arrive_expect_tx(&ctl->q_full, p.n2 * 256);
-        for (int h = 0; h < 2; ++h)
-          tma_load_3d(sQ + h * p.n2 * 128, &p.tmq2[c.s], &ctl->q_full, h * 64, c.g * p.rows, zq);
+        for (int h = 0; h < 2; ++h) tma_load_3d(sQ + h * qhalf, &p.tmq2[c.s], &ctl->q_full, h * 64, y, zq);
       }
       last_q_pc = pc;
       ++pc;
     }
-    const int stage = it % kStages;
-    const uint32_t ph = (it / kStages) & 1;
-    if (!mbar_wait(&ctl->k_empty[stage], ph ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
+    if (!mbar_wait(&ctl->k_empty[stage], phase ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
     mbar_arrive_expect_tx(&ctl->k_full[stage], kTileBytes);
     const int zk = (p.layer0 + c.l) * p.G + c.g;
     for (int h = 0; h < 2; ++h)
       tma_load_3d_hint(sK + stage * kTileBytes + h * kHalfBytes, &p.tmk[c.s], &ctl->k_full[stage],
                        h * 64, c.j * kTileKeys, zk, pol_k);
-    last_it[stage] = it;
-    ++it;
+    last_ph[stage] = phase;
+    if (++stage == p.kstages) {
+      stage = 0;
+      phase ^= 1;
+    }
   }
   if (ctl->abort) {
     // bring every issued copy to completion before the CTA can exit
-    for (int i = 0; i < kStages; ++i)
-      if (last_it[i] >= 0) mbar_wait(&ctl->k_full[i], (last_it[i] / kStages) & 1, p.wait_ns);
+    for (int i = 0; i < p.kstages; ++i)
+      if (last_ph[i] >= 0) mbar_wait(&ctl->k_full[i], last_ph[i], p.wait_ns);
     if (last_q_pc >= 0) mbar_wait(&ctl->q_full, last_q_pc & 1, p.wait_ns);
   }
 }
 
-// MMA issuer shared by both passes.
+// MMA issuer shared by both passes.  Two issuing threads (warps 1 and 2)
+// take the even and the odd tiles of the CTA's range, so the bookkeeping of
+// one (barrier waits, commits, tile iteration) overlaps the other's MMAs: a
+// single issuing thread leaves the tensor pipe idle for about that long every
+// tile.  Issuer `who` owns TMEM accumulator stage `who`; both walk every tile
+// to follow the piece boundaries and each commits the Q release of a piece
+// for its own MMAs.
 template <int PASS>
 __device__ void mma_loop(const ScoreParams& p, SmemCtl* ctl, const uint8_t* sQ, const uint8_t* sK,
-                         uint32_t tmem, int64_t fb, int64_t fe) {
+                         uint32_t tmem, int64_t fb, int64_t fe, int who) {
   const uint32_t idesc = PASS == 1 ? idesc_bf16(128, kTileKeys) : idesc_bf16(128, p.n2);
-  const uint32_t q_addr = smem_u32(sQ), k_addr = smem_u32(sK);
-  int it = 0, jt = 0, pc = 0;
+  // shared-memory descriptors are built once; an MMA only adds its operand's
+  // offset (in 16-byte units) to the start-address field, which cannot carry
+  // out of the field inside the 227 KB window
+  const uint64_t dq0 = sdesc_k_sw128(smem_u32(sQ)), dk0 = sdesc_k_sw128(smem_u32(sK));
+  const uint32_t qhalf16 = (p.q_rows * 128) >> 4;
+  // K stage and phase of tile jt = who, who + 2, ...
+  int stage = who % p.kstages, phase = 0, pc = 0, own = 0;
+  const uint32_t d0 = tmem + who * 256;
+  int64_t jt = 0;
   TileIter c;
-  for (c.init(p, fb, fe); c.valid(); c.next(p)) {
+  for (c.init(p, fb, fe); c.valid(); c.next(p), ++jt) {
     if (ctl->abort) break;
-    const bool last = c.last();
     if (c.first(fb)) {
       if (!mbar_wait(&ctl->q_full, pc & 1, p.wait_ns)) { fail(ctl, p.err); break; }
       ++pc;
     }
-    const int stage = it % kStages;
-    const uint32_t ph = (it / kStages) & 1;
-    const int ts = jt & 1;
-    const uint32_t tph = (jt >> 1) & 1;
-    if (!mbar_wait(&ctl->k_full[stage], ph, p.wait_ns)) { fail(ctl, p.err); break; }
-    if (!mbar_wait(&ctl->t_empty[ts], tph ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
-    tc_fence_after();
-    const uint32_t kbase = k_addr + stage * kTileBytes;
-    if (PASS == 1) {
-      for (int mt = 0; mt < p.n_mtiles; ++mt) {
-        const uint32_t d = tmem + ts * 256 + mt * kTileKeys;
+    if ((jt & 1) == who) {
+      if (!mbar_wait(&ctl->k_full[stage], phase, p.wait_ns)) { fail(ctl, p.err); break; }
+      if (!mbar_wait(&ctl->t_empty[who], (own & 1) ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
+      tc_fence_after();
+      const uint64_t dk = dk0 + static_cast<uint64_t>(stage * (kTileBytes >> 4));
+      if (PASS == 1) {
+#pragma unroll
+        for (int mt = 0; mt < 2; ++mt) {
+          if (mt >= p.n_mtiles) break;
+          const uint32_t d = d0 + mt * kTileKeys;
+          // M tile 1 reads rows 128..255 of each Q half; rows past q_rows are
+          // other shared memory and only feed accumulator rows that are dropped
+          const uint64_t dq = dq0 + static_cast<uint64_t>(mt * ((kTileKeys * 128) >> 4));
+#pragma unroll
+          for (int kk = 0; kk < 8; ++kk) {
+            const uint32_t koff16 = (kk >> 2) * (kHalfBytes >> 4) + (kk & 3) * 2;
+            const uint32_t qoff16 = (kk >> 2) * qhalf16 + (kk & 3) * 2;
+            mma_bf16(d, dq + qoff16, dk + koff16, idesc, kk > 0);
+          }
+        }
+      } else {
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk) {
-          const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-          mma_bf16(d, sdesc_k_sw128(q_addr + mt * kTileBytes + koff), sdesc_k_sw128(kbase + koff),
-                   idesc, kk > 0);
+          const uint32_t koff16 = (kk >> 2) * (kHalfBytes >> 4) + (kk & 3) * 2;
+          const uint32_t qoff16 = (kk >> 2) * qhalf16 + (kk & 3) * 2;
+          mma_bf16(d0, dk + koff16, dq0 + qoff16, idesc, kk > 0);
         }
       }
-    } else {
-      const uint32_t d = tmem + ts * 256;
-      const uint32_t qhalf = p.n2 * 128;
-#pragma unroll
-      for (int kk = 0; kk < 8; ++kk) {
-        const uint32_t koff = (kk >> 2) * kHalfBytes + (kk & 3) * 32;
-        const uint32_t qoff = (kk >> 2) * qhalf + (kk & 3) * 32;
-        mma_bf16(d, sdesc_k_sw128(kbase + koff), sdesc_k_sw128(q_addr + qoff), idesc, kk > 0);
+      mma_commit(&ctl->k_empty[stage]);
+      mma_commit(&ctl->t_full[who]);
+      ++own;
+      stage += 2;
+      if (stage >= p.kstages) {
+        stage -= p.kstages;
+        phase ^= 1;
       }
     }
-    mma_commit(&ctl->k_empty[stage]);
-    mma_commit(&ctl->t_full[ts]);
-    if (last) mma_commit(&ctl->q_empty);
-    ++it;
-    ++jt;
+    if (c.last()) mma_commit(&ctl->q_empty);
   }
   // every MMA issued above must be complete before TMEM is released
   mma_commit(&ctl->drain);
@@ -351,8 +372,10 @@ __device__ __noinline__ void lse_tile_rescale(uint32_t base, int n, int lim, flo
 // reference is set from the first chunk a piece sees and moves only when a
 // tile's sum exceeds 2^64 (a logit more than 64 above it, or overflow); that
 // tile is then redone against its own maximum.  Terms far below the reference
-// underflow to zero, below the fp32 resolution of the sum.
-__device__ __forceinline__ void lse_tile(uint32_t base, int nch, int lim, float sc, float& m, float& s) {
+// underflow to zero, below the fp32 resolution of the sum.  A lane that is
+// not `live` (a row past the group's window rows) takes part in the
+// warp-collective loads only.
+__device__ __forceinline__ void lse_tile(uint32_t base, int nch, int lim, float sc, bool live, float& m, float& s) {
   if (lim <= 0) return;
   const int n = min(nch, (lim + 15) >> 4);
   const bool full = lim >= nch * 16;
@@ -371,7 +394,7 @@ __device__ __forceinline__ void lse_tile(uint32_t base, int nch, int lim, float 
   else
     stream16(base, n, [&](const uint32_t(&r)[16], int ch) { exp2_acc16_masked(r, lim - ch * 16, sc2, nm2, a0, a1); });
   const float2 a = fadd2(a0, a1);
-  const float cs = a.x + a.y;
+  const float cs = live ? a.x + a.y : 0.f;   // a lane past the window rows holds garbage
   if (__all_sync(kFull, cs < 1.8446744e19f)) s += cs;   // below 2^64: the common case
   else lse_tile_rescale(base, n, lim, sc, m, s);       // the whole warp, each lane from its own m
 }
@@ -398,13 +421,13 @@ __device__ __forceinline__ void accum16(const uint32_t (&r)[16], const float4* n
 __global__ void __launch_bounds__(kScoreThreads, 1) k_score_lse(const __grid_constant__ ScoreParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* sQ = smem;                          // [2 M-tiles][2 halves][128][128 B]
-  uint8_t* sK = smem + 2 * kTileBytes;         // [kStages][2 halves][128][128 B]
-  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sK + kStages * kTileBytes);
+  uint8_t* sQ = smem;                          // [2 halves][q_rows][128 B]
+  uint8_t* sK = smem + 2 * p.q_rows * 128;     // [kstages][2 halves][128][128 B]
+  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sK + p.kstages * kTileBytes);
   float2* pbuf = reinterpret_cast<float2*>(reinterpret_cast<uint8_t*>(ctl) + 256);   // [4 wg][128]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  if (threadIdx.x == 0) ctl_init(ctl);
+  if (threadIdx.x == 0) ctl_init(ctl, p.kstages);
   if (warp == 1) {
     tmem_alloc(&ctl->tmem_base, kTmemCols);
     tmem_relinquish();
@@ -419,8 +442,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_lse(const __grid_con
 
   if (warp == 0) {
     if (lane == 0) producer_loop<1>(p, ctl, sQ, sK, fb, fe);
-  } else if (warp == 1) {
-    if (lane == 0) mma_loop<1>(p, ctl, sQ, sK, tmem, fb, fe);
+  } else if (warp == 1 || warp == 2) {
+    if (lane == 0) mma_loop<1>(p, ctl, sQ, sK, tmem, fb, fe, warp - 1);
   } else if (warp >= kEpiWarp0) {
     const int wg = (warp - kEpiWarp0) >> 2;  // epilogue warpgroup 0..3
     const int quad = warp & 3;              // TMEM lane quadrant
@@ -456,7 +479,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_lse(const __grid_con
           dead = true;
         } else {
           tc_fence_after();
-          if (active) lse_tile(base0 + ts * 256, nch, p.seq[c.s].Lp - (c.j * kTileKeys + kofs), sc, m, s);
+          if (active) lse_tile(base0 + ts * 256, nch, p.seq[c.s].Lp - (c.j * kTileKeys + kofs), sc, r < p.rows, m, s);
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&ctl->t_empty[ts]);
@@ -495,13 +518,13 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_lse(const __grid_con
 __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_constant__ ScoreParams p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
-  uint8_t* sQ = smem;                          // [2 halves][n2][128 B]  (<= 64 KB)
-  uint8_t* sK = smem + 2 * kTileBytes;         // [kStages][2 halves][128][128 B]
-  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sK + kStages * kTileBytes);
+  uint8_t* sQ = smem;                          // [2 halves][q_rows][128 B]
+  uint8_t* sK = smem + 2 * p.q_rows * 128;     // [kstages][2 halves][128][128 B]
+  SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sK + p.kstages * kTileBytes);
   float* nlse = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ctl) + 256);  // [256] -lse2
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
-  if (threadIdx.x == 0) ctl_init(ctl);
+  if (threadIdx.x == 0) ctl_init(ctl, p.kstages);
   if (warp == 1) {
     tmem_alloc(&ctl->tmem_base, kTmemCols);
     tmem_relinquish();
@@ -516,8 +539,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
 
   if (warp == 0) {
     if (lane == 0) producer_loop<2>(p, ctl, sQ, sK, fb, fe);
-  } else if (warp == 1) {
-    if (lane == 0) mma_loop<2>(p, ctl, sQ, sK, tmem, fb, fe);
+  } else if (warp == 1 || warp == 2) {
+    if (lane == 0) mma_loop<2>(p, ctl, sQ, sK, tmem, fb, fe, warp - 1);
   } else if (warp >= kEpiWarp0) {
     const int et = threadIdx.x - 32 * kEpiWarp0;   // 0..511
     const int wg = et >> 7;                 // column quarter
@@ -591,24 +614,32 @@ __global__ void k_pool(const __grid_constant__ SeqBatch b, int G, int H, int poo
   s.S[(static_cast<int64_t>(layer) * G + g) * s.Lp + t] = acc * scale;
 }
 
-size_t score_smem_bytes() {
-  return 1024 + 2 * kTileBytes + kStages * kTileBytes + 256 + 4 * 128 * sizeof(float2);
+// alignment slack + Q + K stages + control block + pass-1 merge buffer
+size_t score_smem_bytes(int q_rows, int kstages) {
+  return 1024 + static_cast<size_t>(2 * q_rows * 128) + static_cast<size_t>(kstages) * kTileBytes + 256 +
+         4 * 128 * sizeof(float2);
+}
+
+int score_kstages(int q_rows) {
+  int k = kMaxStages;
+  while (k > 0 && score_smem_bytes(q_rows, k) > kSmemLimit) --k;
+  return k;
 }
 
 cudaError_t score_configure() {
-  const int bytes = static_cast<int>(score_smem_bytes());
+  const int bytes = static_cast<int>(kSmemLimit);
   cudaError_t e = cudaFuncSetAttribute(k_score_lse, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
   if (e != cudaSuccess) return e;
   return cudaFuncSetAttribute(k_score_accum, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
 cudaError_t score_lse_launch(const ScoreParams& p, int grid, cudaStream_t stream) {
-  k_score_lse<<<grid, kScoreThreads, score_smem_bytes(), stream>>>(p);
+  k_score_lse<<<grid, kScoreThreads, score_smem_bytes(p.q_rows, p.kstages), stream>>>(p);
   return cudaGetLastError();
 }
 
 cudaError_t score_accum_launch(const ScoreParams& p, int grid, cudaStream_t stream) {
-  k_score_accum<<<grid, kScoreThreads, score_smem_bytes(), stream>>>(p);
+  k_score_accum<<<grid, kScoreThreads, score_smem_bytes(p.q_rows, p.kstages), stream>>>(p);
   return cudaGetLastError();
 }
 

@@ -16,13 +16,16 @@ struct ScoreSeq {
 
 struct ScoreParams {
   CUtensorMap tmk[kMaxBatch];    // K: dims (d, L, n_layers*G), box (64, 128, 1), 128B swizzle
-  CUtensorMap tmq1[kMaxBatch];   // Q: dims (d, H*w, n_layers), box (64, 128, 1)
-  CUtensorMap tmq2[kMaxBatch];   // Q: dims (d, H*w, n_layers), box (64, n2, 1)
+  CUtensorMap tmqa[kMaxBatch];   // Q: dims (d, H*w, n_layers), box (64, min(rows, 128), 1)
+  CUtensorMap tmqb[kMaxBatch];   // Q: same, box (64, rows - 128, 1) when rows > 128
+  CUtensorMap tmq2[kMaxBatch];   // Q: same, box (64, n2, 1)
   ScoreSeq seq[kMaxBatch];
   int nseq, layer0, nlayers, G;
   int rows;            // (H / G) * w window rows per group
   int n2;              // rows rounded up to 16 (pass-2 MMA N)
   int n_mtiles;        // ceil(rows / 128) (pass-1 M tiles)
+  int q_rows;          // shared-memory Q rows per 64-column half (= n2)
+  int kstages;         // K-tile pipeline depth (from the shared-memory budget)
   int grid1;           // pass-1 grid size (defines the partial-slot partition)
   int64_t total_tiles;
   float scale2;        // log2(e) / sqrt(d)
@@ -31,7 +34,8 @@ struct ScoreParams {
   uint64_t wait_ns;
 };
 
-size_t score_smem_bytes();
+size_t score_smem_bytes(int q_rows, int kstages);
+int score_kstages(int q_rows);
 cudaError_t score_configure();
 cudaError_t score_lse_launch(const ScoreParams& p, int grid, cudaStream_t stream);
 cudaError_t score_accum_launch(const ScoreParams& p, int grid, cudaStream_t stream);
