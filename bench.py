@@ -201,7 +201,7 @@ def run_oracle_subprocess(workload, budget_s=15.0, max_layers=28, repeat=0):
 def reference_arm(args):
     """--impl reference: the fp64 oracle as it stands, one layer of the
     workload per step, on the host cores (rank 0 only)."""
-    if int(os.environ.get("RANK", "0")) != 0:
+    if rank_env()[1] != 0:
         return
     from paper_2606_01790_gb300 import synthetic as syn
     wl = syn.WORKLOADS[args.workload]
@@ -223,6 +223,33 @@ def reference_arm(args):
     }))
 
 
+# ----------------------------------------------------------------------------- ranks
+
+def rank_env():
+    """(world size, rank, local rank) from the torchrun environment."""
+    return (int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("RANK", "0")),
+            int(os.environ.get("LOCAL_RANK", "0")))
+
+
+def rank_seeds(rank, n_seqs):
+    """Each rank compresses its own trajectories (weak scaling): distinct seeds."""
+    return [rank * 1000 + i for i in range(n_seqs)]
+
+
+def max_over_ranks(x, dist, device):
+    """The largest value of ``x`` over all ranks (the job's time is its slowest rank's)."""
+    import torch
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    if dist is not None:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_rank_step, world, steps, ms_max):
+    """Whole-job tokens/s: every rank's tokens over the slowest rank's time."""
+    return tokens_per_rank_step * world * steps / (ms_max / 1e3)
+
+
 # ----------------------------------------------------------------------------- GPU arm
 
 def gpu_arm(args):
@@ -232,9 +259,7 @@ def gpu_arm(args):
     from paper_2606_01790_gb300 import starkv as sk
     from paper_2606_01790_gb300 import synthetic as syn
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+    world, rank, local = rank_env()
     dist = None
     if world > 1:
         import torch.distributed as dist
@@ -244,7 +269,7 @@ def gpu_arm(args):
     __graft_entry__.build()
 
     wl = syn.WORKLOADS[args.workload]
-    seeds = [rank * 1000 + i for i in range(wl.n_seqs)]
+    seeds = rank_seeds(rank, wl.n_seqs)
     sis = [syn.make_sequence(wl, seq=i, seed=s) for i, s in enumerate(seeds)]
     cfg = sk.Config(n_layers=wl.n_layers, n_heads=wl.n_heads, n_kv_heads=wl.n_kv_heads,
                     head_dim=wl.head_dim, window=wl.window, grid_rows=wl.grid_rows,
@@ -305,12 +330,9 @@ def gpu_arm(args):
     kt = sk.kernel_times(st)
     sk.check_device_error(st)
     clocks.stop()
-    ms_t = torch.tensor([ms], dtype=torch.float64, device=dev)
-    if dist is not None:
-        dist.all_reduce(ms_t, op=dist.ReduceOp.MAX)
-    ms_max = float(ms_t.item())
+    ms_max = max_over_ranks(ms, dist, dev)
     ms_step = ms_max / args.steps
-    value = work["tokens"] * world * args.steps / (ms_max / 1e3)
+    value = job_throughput(work["tokens"], world, args.steps, ms_max)
     launches = sum(v[0] for v in kt.values())
 
     # roofline of the dominant kernel
@@ -352,12 +374,10 @@ def gpu_arm(args):
             sk.step_host(st, hseqs, hws)
         b.record(stream)
         barrier()
-        e_ms = torch.tensor([a.elapsed_time(b)], dtype=torch.float64, device=dev)
-        if dist is not None:
-            dist.all_reduce(e_ms, op=dist.ReduceOp.MAX)
-        e2e = {"value": work["tokens"] * world * n_e2e / (float(e_ms.item()) / 1e3), "unit": UNIT,
+        e_ms = max_over_ranks(a.elapsed_time(b), dist, dev)
+        e2e = {"value": job_throughput(work["tokens"], world, n_e2e, e_ms), "unit": UNIT,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n_e2e,
-               "ms_per_step": float(e_ms.item()) / n_e2e}
+               "ms_per_step": e_ms / n_e2e}
         sk.check_device_error(st)
 
     cpu = None

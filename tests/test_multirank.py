@@ -1,0 +1,62 @@
+"""Host logic of the multi-GPU benchmark path, on CPU with gloo and two ranks:
+each rank draws its own trajectories, the job time is the slowest rank's, the
+whole-job throughput counts every rank's tokens, and only rank 0 reports.
+(The data path shards into independent (sequence, layer) units: there is no
+collective besides the timing reduction.)"""
+import json
+import os
+import subprocess
+import sys
+
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+import bench  # noqa: E402
+
+
+def _worker(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    w, r, _ = bench.rank_env()
+    ms = 10.0 + 5.0 * r                      # rank 1 is the slow one
+    ms_max = bench.max_over_ranks(ms, dist, "cpu")
+    seeds = bench.rank_seeds(r, 3)
+    gathered = [None] * world
+    dist.all_gather_object(gathered, seeds)
+    out[r] = (w, ms_max, bench.job_throughput(1000, w, 4, ms_max), gathered)
+    dist.destroy_process_group()
+
+
+def _free_port():
+    import socket
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def test_two_gloo_ranks_reduce_the_job_time_and_draw_distinct_inputs():
+    world = 2
+    with mp.Manager() as m:
+        out = m.dict()
+        mp.spawn(_worker, args=(world, _free_port(), out), nprocs=world, join=True)
+        res = dict(out)
+    for r in range(world):
+        w, ms_max, thr, seeds = res[r]
+        assert w == world
+        assert ms_max == 15.0                          # max over ranks, seen by every rank
+        assert abs(thr - 1000 * 2 * 4 / 0.015) < 1e-6  # all ranks' tokens over the slowest time
+        flat = [s for per in seeds for s in per]
+        assert len(set(flat)) == len(flat)             # weak scaling: independent trajectories
+
+
+def test_reference_arm_prints_on_rank_zero_only():
+    env = dict(os.environ, RANK="1", WORLD_SIZE="2", LOCAL_RANK="1")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                        "--steps", "1", "--warmup", "0"], env=env, capture_output=True, text=True,
+                       timeout=120)
+    assert r.returncode == 0, r.stderr
+    assert r.stdout.strip() == ""
