@@ -340,11 +340,12 @@ __device__ __forceinline__ float max16_masked(const uint32_t (&r)[16], int lim) 
   return mx;
 }
 
-// Rare path of lse_tile: a logit more than 64 above the reference (or an
-// overflow) in some lane of the warp; every lane redoes the tile against
-// max(its reference, its tile maximum), which leaves a lane without overflow
-// with the same sum.
-__device__ __noinline__ void lse_tile_rescale(uint32_t base, int n, int lim, float sc, float& m, float& s) {
+// Slow path of lse_tile, taken by the whole warp (TMEM loads are
+// warp-collective): the first tile of a piece (no reference yet), the ragged
+// last tile of a row, or a tile with a logit more than 64 above the
+// reference in some lane.  Each lane moves its reference to max(reference,
+// its tile maximum), rescales its sum and adds the tile's valid keys.
+__device__ __forceinline__ void lse_tile_slow(uint32_t base, int n, int lim, float sc, bool live, float& m, float& s) {
   float mx = -INFINITY;
   for (int ch = 0; ch < n; ++ch) {
     uint32_t r[16];
@@ -353,7 +354,7 @@ __device__ __noinline__ void lse_tile_rescale(uint32_t base, int n, int lim, flo
     mx = fmaxf(mx, max16_masked(r, lim - ch * 16));
   }
   const float mn = fmaxf(m, mx * sc);
-  s *= ex2_approx(m - mn);
+  if (m != -INFINITY) s *= ex2_approx(m - mn);
   m = mn;
   const float2 sc2 = make_float2(sc, sc), nm2 = make_float2(-m, -m);
   float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
@@ -364,39 +365,33 @@ __device__ __noinline__ void lse_tile_rescale(uint32_t base, int n, int lim, flo
     exp2_acc16_masked(r, lim - ch * 16, sc2, nm2, a0, a1);
   }
   const float2 a = fadd2(a0, a1);
-  s += a.x + a.y;
+  if (live) s += a.x + a.y;   // a lane past the window rows holds garbage
 }
 
 // One row's running (reference m, sum s of exp2(z sc - m)) over this thread's
 // `nch` 16-key chunks of one tile, `lim` of which keys are valid.  The
-// reference is set from the first chunk a piece sees and moves only when a
-// tile's sum exceeds 2^64 (a logit more than 64 above it, or overflow); that
-// tile is then redone against its own maximum.  Terms far below the reference
-// underflow to zero, below the fp32 resolution of the sum.  A lane that is
-// not `live` (a row past the group's window rows) takes part in the
-// warp-collective loads only.
+// reference is set on a piece's first tile and moves only when a tile's sum
+// exceeds 2^64 (a logit more than 64 above it, or overflow); that tile is then
+// redone.  Terms far below the reference underflow to zero, below the fp32
+// resolution of the sum.  A lane that is not `live` (a row past the group's
+// window rows) takes part in the warp-collective loads only.  The full-tile
+// path is straight-line; everything else goes through the slow path.
 __device__ __forceinline__ void lse_tile(uint32_t base, int nch, int lim, float sc, bool live, float& m, float& s) {
-  if (lim <= 0) return;
-  const int n = min(nch, (lim + 15) >> 4);
-  const bool full = lim >= nch * 16;
-  const float2 sc2 = make_float2(sc, sc);
-  // TMEM loads are warp-collective: every branch around them is warp-uniform
-  if (__any_sync(kFull, m == -INFINITY)) {
-    uint32_t r[16];
-    tmem_ld16_async(base, r);
-    tmem_wait16(r);
-    if (m == -INFINITY) m = max16_masked(r, lim) * sc;
+  if (lim <= 0) return;   // lim is the same in every lane
+  if (lim < nch * 16 || __any_sync(kFull, m == -INFINITY)) {
+    lse_tile_slow(base, min(nch, (lim + 15) >> 4), lim, sc, live, m, s);
+    return;
   }
-  const float2 nm2 = make_float2(-m, -m);
+  const float2 sc2 = make_float2(sc, sc), nm2 = make_float2(-m, -m);
   float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
-  if (full)
-    stream16(base, n, [&](const uint32_t(&r)[16], int) { exp2_acc16(r, sc2, nm2, a0, a1); });
-  else
-    stream16(base, n, [&](const uint32_t(&r)[16], int ch) { exp2_acc16_masked(r, lim - ch * 16, sc2, nm2, a0, a1); });
+  stream16(base, nch, [&](const uint32_t(&r)[16], int) { exp2_acc16(r, sc2, nm2, a0, a1); });
   const float2 a = fadd2(a0, a1);
-  const float cs = live ? a.x + a.y : 0.f;   // a lane past the window rows holds garbage
-  if (__all_sync(kFull, cs < 1.8446744e19f)) s += cs;   // below 2^64: the common case
-  else lse_tile_rescale(base, n, lim, sc, m, s);       // the whole warp, each lane from its own m
+  const float cs = a.x + a.y;
+  if (__all_sync(kFull, !live || cs < 1.8446744e19f)) {   // below 2^64: the common case
+    if (live) s += cs;
+  } else {
+    lse_tile_slow(base, nch, lim, sc, live, m, s);
+  }
 }
 
 // sum over 16 columns of exp2(z * sc + nl[col]), nl = -lse2 of the columns
@@ -554,11 +549,16 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
     const float sc = p.scale2;
     int jt = 0;
     bool dead = false;
+    float* dst = nullptr;   // this thread's copy of the piece's unpooled row
+    int lp = 0;
     TileIter c;
     for (c.init(p, fb, fe); c.valid(); c.next(p)) {
       if (c.first(fb)) {
         named_bar_sync(1, kEpiThreads);   // the previous piece's readers are done
         if (et < kMaxRows) nlse[et] = et < p.rows ? -combine_lse2(p, c.f - c.j, c.nt, et) : -INFINITY;
+        const ScoreSeq& sq = p.seq[c.s];
+        lp = sq.Lp;
+        dst = sq.s_raw + (static_cast<int64_t>(c.l * p.G + c.g) * kRawCopies + wg) * lp + q;
         named_bar_sync(1, kEpiThreads);
       }
       const int ts = jt & 1;
@@ -574,11 +574,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&ctl->t_empty[ts]);
-          const ScoreSeq& sq = p.seq[c.s];
-          const int key = c.j * kTileKeys + q;
+          const int key0 = c.j * kTileKeys;
           const float2 a = fadd2(a0, a1);
-          if (key < sq.Lp)
-            sq.s_raw[(static_cast<int64_t>(c.l * p.G + c.g) * kRawCopies + wg) * sq.Lp + key] = a.x + a.y;
+          if (key0 + q < lp) dst[key0] = a.x + a.y;
         }
       }
       ++jt;
