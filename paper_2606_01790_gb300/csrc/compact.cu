@@ -1,7 +1,10 @@
 // Compressed cache of Sec. 3.7, Eq. (11) (Algorithm 1 last step):
 //   K' = [K_past[I]; K_rec],  V' = [V_past[I]; V_rec],  meta' likewise.
-// A bit copy bound by HBM bandwidth: every 256-byte row (d = 128 bf16) moves
-// as one 16-lane x 16-byte vector access, four rows per half-warp in flight.
+// A bit copy bound by HBM bandwidth.  A warp task is 32 consecutive output
+// rows of one (tensor, group): lane i resolves the source row of output row
+// i, the source rows are broadcast by shuffle, and every instruction moves
+// two 256-byte rows (d = 128 bf16) as one 16-byte access per lane, with eight
+// such accesses per lane in flight.
 #include "common.cuh"
 #include "compact.cuh"
 
@@ -10,7 +13,9 @@ namespace starkv {
 namespace {
 
 constexpr int kCompactThreads = 256;
-constexpr int kRowsInFlight = 4;
+constexpr int kWarps = kCompactThreads / 32;
+constexpr int kTaskRows = 32;   // output rows per warp task
+constexpr int kInFlight = 8;    // 16-byte accesses per lane in flight (16 rows per warp)
 
 __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
   uint4 v;
@@ -28,71 +33,64 @@ __device__ __forceinline__ void st_stream(uint4* p, const uint4& v) {
 
 }  // namespace
 
-// grid: (blocks, nlayers, nseq).  Rows of one (seq, layer): 2 tensors x G x (B + w).
+// grid: (blocks, nlayers, nseq).  Tasks of one (seq, layer): 2 tensors x G x
+// ceil((B + w) / 32) row blocks, one per warp, strided over the grid.
 __global__ void __launch_bounds__(kCompactThreads) k_compact(const __grid_constant__ SeqBatch b, int G, int w,
                                                               uint32_t* err) {
   const SeqView& sv = b.s[blockIdx.z];
   const int layer = b.layer0 + blockIdx.y;
   const int B = sv.budget, Lp = sv.Lp, L = sv.L;
   const int rows_out = B + w;
+  const int lane = threadIdx.x & 31, half = lane >> 4, hl = lane & 15;
   const int32_t* idx = sv.idx + static_cast<int64_t>(layer) * B;
-  const int64_t in_layer = static_cast<int64_t>(layer) * G * L;          // rows
-  const int64_t out_layer = static_cast<int64_t>(layer) * G * rows_out;  // rows
-
-  // metadata: one thread per output row
   const uint32_t* meta = sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride;
   uint32_t* meta_out = sv.meta_out + static_cast<int64_t>(layer) * rows_out;
-  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < rows_out; r += gridDim.x * blockDim.x) {
-    int src = r < B ? idx[r] : Lp + (r - B);
-    if (src < 0 || src >= L) {   // an index outside the cache: report, copy row 0
-      atomicOr(err, kErrIndex);
-      src = 0;
+  const int nblk = ceil_div(rows_out, kTaskRows);
+  const int ntask = 2 * G * nblk;
+  for (int task = blockIdx.x * kWarps + (threadIdx.x >> 5); task < ntask; task += gridDim.x * kWarps) {
+    const int tensor = task / (G * nblk);
+    const int rem = task - tensor * G * nblk;
+    const int g = rem / nblk, r0 = (rem - g * nblk) * kTaskRows;
+    // source row of output row r0 + lane
+    const int r = r0 + lane;
+    int src = 0;
+    if (r < rows_out) {
+      src = r < B ? idx[r] : Lp + (r - B);
+      if (src < 0 || src >= L) {   // an index outside the cache: report, copy row 0
+        atomicOr(err, kErrIndex);
+        src = 0;
+      }
+      if (tensor == 0 && g == 0) meta_out[r] = meta[src];
     }
-    meta_out[r] = meta[src];
-  }
-
-  // K and V rows: a half-warp per row, 16 lanes x 16 bytes
-  const int hl = threadIdx.x & 15;
-  const int64_t n_items = 2LL * G * rows_out;
-  const int64_t hw0 = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) >> 4;
-  const int64_t hstride = (static_cast<int64_t>(gridDim.x) * blockDim.x) >> 4;
-  for (int64_t base = hw0; base < n_items; base += hstride * kRowsInFlight) {
-    uint4 v[kRowsInFlight];
-    uint4* dst[kRowsInFlight];
+    const __nv_bfloat16* in = (tensor == 0 ? sv.k : sv.v) + (static_cast<int64_t>(layer) * G + g) * L * kHeadDim;
+    __nv_bfloat16* out = (tensor == 0 ? sv.k_out : sv.v_out) + (static_cast<int64_t>(layer) * G + g) * rows_out * kHeadDim;
+    const uint4* in4 = reinterpret_cast<const uint4*>(in) + hl;
+    uint4* out4 = reinterpret_cast<uint4*>(out) + static_cast<int64_t>(r0) * (kHeadDim / 8) + hl;
+    const int nrows = min(kTaskRows, rows_out - r0);
 #pragma unroll
-    for (int i = 0; i < kRowsInFlight; ++i) {
-      const int64_t item = base + i * hstride;
-      dst[i] = nullptr;
-      if (item < n_items) {
-        const int tensor = static_cast<int>(item / (static_cast<int64_t>(G) * rows_out));
-        const int rem = static_cast<int>(item - static_cast<int64_t>(tensor) * G * rows_out);
-        const int g = rem / rows_out, r = rem - g * rows_out;
-        int src = r < B ? idx[r] : Lp + (r - B);
-        if (src < 0 || src >= L) src = 0;   // reported by the metadata loop above
-        const __nv_bfloat16* in = tensor == 0 ? sv.k : sv.v;
-        __nv_bfloat16* out = tensor == 0 ? sv.k_out : sv.v_out;
-        const uint4* s = reinterpret_cast<const uint4*>(in + (in_layer + static_cast<int64_t>(g) * L + src) * kHeadDim);
-        dst[i] = reinterpret_cast<uint4*>(out + (out_layer + static_cast<int64_t>(g) * rows_out + r) * kHeadDim) + hl;
-        v[i] = ld_stream(s + hl);
+    for (int j0 = 0; j0 < kTaskRows; j0 += 2 * kInFlight) {
+      uint4 v[kInFlight];
+#pragma unroll
+      for (int k = 0; k < kInFlight; ++k) {
+        const int row = j0 + 2 * k + half;
+        const int s_row = __shfl_sync(0xffffffffu, src, row);
+        if (row < nrows) v[k] = ld_stream(in4 + static_cast<int64_t>(s_row) * (kHeadDim / 8));
+      }
+#pragma unroll
+      for (int k = 0; k < kInFlight; ++k) {
+        const int row = j0 + 2 * k + half;
+        if (row < nrows) st_stream(out4 + row * (kHeadDim / 8), v[k]);
       }
     }
-#pragma unroll
-    for (int i = 0; i < kRowsInFlight; ++i)
-      if (dst[i]) st_stream(dst[i], v[i]);
   }
 }
 
 cudaError_t compact_launch(const SeqBatch& b, int G, int w, int rows_out_max, int num_sms, uint32_t* err,
                            cudaStream_t stream) {
+  (void)num_sms;
   if (rows_out_max <= 0) return cudaSuccess;
-  // enough half-warps for every row of a (seq, layer) with kRowsInFlight rows each,
-  // capped so the whole launch stays a few waves of the GPU
-  const int64_t rows = 2LL * G * rows_out_max;
-  int64_t blocks = (rows * 16 / kRowsInFlight + kCompactThreads - 1) / kCompactThreads;
-  const int64_t cap = (8LL * num_sms + b.nlayers * b.nseq - 1) / (b.nlayers * b.nseq);
-  if (blocks > cap) blocks = cap;
-  if (blocks < 1) blocks = 1;
-  dim3 grid(static_cast<unsigned>(blocks), b.nlayers, b.nseq);
+  const int ntask = 2 * G * ceil_div(rows_out_max, kTaskRows);
+  dim3 grid(static_cast<unsigned>(ceil_div(ntask, kWarps)), b.nlayers, b.nseq);
   k_compact<<<grid, kCompactThreads, 0, stream>>>(b, G, w, err);
   return cudaGetLastError();
 }
