@@ -317,86 +317,78 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   __syncthreads();
 
   // ================= phase 1: group g =================
-  // ---- one pass over the row: pooling (Eqs. 3-4), keys and cells of the
-  // visual tokens, their key range, the current frame on the patch grid.
-  // Lane = token; the pooling window reaches the neighbouring rows of 32
-  // through shuffles (rows one and two ahead are loaded a row early).
+  // ---- the row, staged in shared memory by one pass of independent loads:
+  // the unpooled sums (the four column-quarter copies added in order) or the
+  // given S, into the candidate region; the metadata words into the key region
   const float pscale = static_cast<float>(G) / static_cast<float>(kp.H) / static_cast<float>(kp.pool);
   const int half = kp.pool >> 1;
   const float* raw = FROM_RAW ? sv.s_raw + static_cast<int64_t>(ll * G + g) * kRawCopies * Lp : nullptr;
-  auto raw_at = [&](int u) {   // sum of the column-quarter copies, zero outside the row
-    float r = 0.f;
-    if (u >= 0 && u < Lp) {
+  float* stage = reinterpret_cast<float*>(cand);
+  for (int t0 = 0; t0 < Lp; t0 += 4 * kCalThreads) {
+    float v[4];
+    uint32_t mw[4];
 #pragma unroll
-      for (int c = 0; c < kRawCopies; ++c) r += raw[c * Lp + u];
+    for (int k = 0; k < 4; ++k) {
+      const int t = t0 + k * kCalThreads + tid;
+      v[k] = 0.f;
+      mw[k] = 0u;
+      if (t < Lp) {
+        mw[k] = meta[t];
+        if (FROM_RAW) {
+          float r = 0.f;
+#pragma unroll
+          for (int c = 0; c < kRawCopies; ++c) r += raw[c * Lp + t];
+          v[k] = r;
+        } else {
+          v[k] = S[t];
+        }
+      }
     }
-    return r;
-  };
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const int t = t0 + k * kCalThreads + tid;
+      if (t < Lp) {
+        stage[t] = v[k];
+        keys[t] = mw[k];
+      }
+    }
+  }
+  __syncthreads();
+  // ---- pooling (Eqs. 3-4), keys and cells of the visual tokens, their key
+  // range, the current frame on the patch grid
   int nv = 0;
   uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
-  {
-    float r_prev = 0.f, r_cur = 0.f, r_next = 0.f;
+  for (int t = tid; t < Lp; t += kCalThreads) {
+    float s;
     if (FROM_RAW) {
-      r_prev = raw_at(s0 - 32 + lane);
-      r_cur = raw_at(s0 + lane);
-      r_next = raw_at(s0 + 32 + lane);
+      float acc = 0.f;
+      for (int j = -half; j <= half; ++j) {
+        const int u = t + j;
+        acc += (u >= 0 && u < Lp) ? stage[u] : 0.f;
+      }
+      s = acc * pscale;
+      S[t] = s;
+    } else {
+      s = stage[t];
     }
-    uint32_t m_cur = s0 + lane < s1 ? meta[s0 + lane] : 0u;
-    for (int base = s0; base < s1; base += 32) {
-      const int t = base + lane;
-      const bool in = t < s1;
-      float r_nn = 0.f;
-      if (FROM_RAW) r_nn = raw_at(base + 64 + lane);
-      const uint32_t m_next = base + 32 + lane < s1 ? meta[base + 32 + lane] : 0u;
-      float s;
-      if (FROM_RAW) {
-        float acc = 0.f;
-        for (int j = -half; j <= half; ++j) {
-          float x;
-          if (j < 0) {
-            const int d = -j;
-            const float a = __shfl_up_sync(kFullMask, r_cur, d);
-            const float c = __shfl_sync(kFullMask, r_prev, (lane - d) & 31);
-            x = lane >= d ? a : c;
-          } else if (j > 0) {
-            const float a = __shfl_down_sync(kFullMask, r_cur, j);
-            const float c = __shfl_sync(kFullMask, r_next, (lane + j) & 31);
-            x = lane < 32 - j ? a : c;
-          } else {
-            x = r_cur;
-          }
-          acc += x;
-        }
-        s = acc * pscale;
-        r_prev = r_cur;
-        r_cur = r_next;
-        r_next = r_nn;
+    const uint32_t mt = keys[t];
+    uint16_t cell = kNoCell;
+    uint32_t key = 0;
+    if (meta_visual(mt)) {
+      const int r = meta_row(mt), c = meta_col(mt);
+      if (r < R && c < C) {
+        key = order_key(s);
+        cell = static_cast<uint16_t>(rowc[r] * M + colc[c]);
+        ++nv;
+        kmin = min(kmin, key);
+        kmax = max(kmax, key);
+        if (meta_frame(mt) == sv.cur_frame) atomicAdd(&cur[r * C + c], s);
       } else {
-        s = in ? S[t] : 0.f;
+        atomicOr(st.err, kErrMeta);
       }
-      if (in) {
-        const uint32_t mt = m_cur;
-        if (FROM_RAW) S[t] = s;
-        uint16_t cell = kNoCell;
-        uint32_t key = 0;
-        if (meta_visual(mt)) {
-          const int r = meta_row(mt), c = meta_col(mt);
-          if (r < R && c < C) {
-            key = order_key(s);
-            cell = static_cast<uint16_t>(rowc[r] * M + colc[c]);
-            ++nv;
-            kmin = min(kmin, key);
-            kmax = max(kmax, key);
-            if (meta_frame(mt) == sv.cur_frame) atomicAdd(&cur[r * C + c], s);
-          } else {
-            atomicOr(st.err, kErrMeta);
-          }
-        }
-        keys[t] = key;
-        cells[t] = cell;
-      }
-      m_cur = m_next;
     }
+    keys[t] = key;
+    cells[t] = cell;
   }
   const int N = block_sum<int>(nv, sh.ired);
   kmin = block_min(kmin, sh.ured);
@@ -635,31 +627,54 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   const int nr = tb - ta;
   const float* S0 = sv.S + static_cast<int64_t>(layer) * G * Lp;
   const float invG = 1.f / static_cast<float>(G);
-  // s_bar (Eq. 4) of token t and its governing group g* (lowest on ties)
-  auto sbar_of = [&](int t, int& gs) {
-    float best = S0[t], acc = best;
-    gs = 0;
-    for (int gg = 1; gg < G; ++gg) {
-      const float v = S0[static_cast<int64_t>(gg) * Lp + t];
-      acc += v;
-      if (v > best) {
-        best = v;
-        gs = gg;
-      }
-    }
-    return acc * invG;
-  };
   // ---- Sec. 3.6 in one pass: Z = sum s_bar and sum s_bar log s_bar over the
   // cluster, then H = -sum p log p / log L_p with p = s_bar / (Z + eps)
-  // (the eps inside the log changes H by less than L_p eps)
+  // (the eps inside the log changes H by less than L_p eps).  The pass stages
+  // s_bar, g* and the metadata word of its tokens for the fused score.
+  float* sbar_s = reinterpret_cast<float*>(cand);   // [nr]
   float z = 0.f, zl = 0.f;
   int nvr = 0;
-  for (int t = ta + tid; t < tb; t += kCalThreads) {
-    int gs;
-    const float sb = sbar_of(t, gs);
-    z += sb;
-    if (sb > 0.f) zl += sb * logf(sb);
-    nvr += meta_visual(meta[t]);
+  for (int i0 = 0; i0 < nr; i0 += 2 * kCalThreads) {
+    float v[2][kMaxGroups];
+    uint32_t mw[2];
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int i = i0 + k * kCalThreads + tid;
+      mw[k] = 0u;
+#pragma unroll
+      for (int gg = 0; gg < kMaxGroups; ++gg) v[k][gg] = 0.f;
+      if (i < nr) {
+        const int t = ta + i;
+        mw[k] = meta[t];
+#pragma unroll
+        for (int gg = 0; gg < kMaxGroups; ++gg)
+          if (gg < G) v[k][gg] = S0[static_cast<int64_t>(gg) * Lp + t];
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < 2; ++k) {
+      const int i = i0 + k * kCalThreads + tid;
+      if (i >= nr) continue;
+      // s_bar (Eq. 4) and its governing group g* (lowest on ties)
+      float best = v[k][0], acc = best;
+      int gs = 0;
+#pragma unroll
+      for (int gg = 1; gg < kMaxGroups; ++gg) {
+        if (gg >= G) break;
+        acc += v[k][gg];
+        if (v[k][gg] > best) {
+          best = v[k][gg];
+          gs = gg;
+        }
+      }
+      const float sb = acc * invG;
+      z += sb;
+      if (sb > 0.f) zl += sb * logf(sb);
+      nvr += meta_visual(mw[k]);
+      sbar_s[i] = sb;
+      keys[i] = mw[k];
+      cells[i] = static_cast<uint16_t>(gs);
+    }
   }
   z = block_sum<float>(z, sh.fred);
   zl = block_sum<float>(zl, sh.fred);
@@ -692,20 +707,20 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   // the first digit of the top-B select
   const float lam = sh.lam;
   float* score = sv.score + static_cast<int64_t>(layer) * Lp;
-  for (int t = ta + tid; t < tb; t += kCalThreads) {
-    int gs;
-    const float sb = sbar_of(t, gs);
+  for (int i = tid; i < nr; i += kCalThreads) {
+    const float sb = sbar_s[i];
+    const int gs = cells[i];
+    const uint32_t mt = keys[i];
     const float beta = (1.f - lam) + lam * static_cast<float>(G) * sh.w[gs];
     float d = 1.f;
-    const uint32_t mt = meta[t];
     if (meta_visual(mt)) {
       const float df = static_cast<float>(sv.cur_frame - meta_frame(mt));
       d = kp.d_min + (1.f - kp.d_min) * expf(-kp.delta * df * sh.ph[gs]);
     }
     const float s = powf(fmaxf(sb * beta * d, 0.f), invT);
-    score[t] = s;
+    score[ta + i] = s;
     const uint32_t key = ~order_key(s);   // descending score = ascending key
-    keys[t - ta] = key;
+    keys[i] = key;
     atomicAdd(&hist[key >> 20], 1);
   }
 
