@@ -6,6 +6,7 @@
 // two 256-byte rows (d = 128 bf16) as one 16-byte access per lane, with eight
 // such accesses per lane in flight.
 #include "common.cuh"
+#include "ptx.cuh"
 #include "compact.cuh"
 
 namespace starkv {
@@ -37,6 +38,8 @@ __device__ __forceinline__ void st_stream(uint4* p, const uint4& v) {
 // ceil((B + w) / 32) row blocks, one per warp, strided over the grid.
 __global__ void __launch_bounds__(kCompactThreads) k_compact(const __grid_constant__ SeqBatch b, int G, int w,
                                                               uint32_t* err) {
+  griddep_launch_dependents();
+  griddep_wait();   // idx comes from the previous kernel
   const SeqView& sv = b.s[blockIdx.z];
   const int layer = b.layer0 + blockIdx.y;
   const int B = sv.budget, Lp = sv.Lp, L = sv.L;
@@ -90,9 +93,16 @@ cudaError_t compact_launch(const SeqBatch& b, int G, int w, int rows_out_max, in
   (void)num_sms;
   if (rows_out_max <= 0) return cudaSuccess;
   const int ntask = 2 * G * ceil_div(rows_out_max, kTaskRows);
-  dim3 grid(static_cast<unsigned>(ceil_div(ntask, kWarps)), b.nlayers, b.nseq);
-  k_compact<<<grid, kCompactThreads, 0, stream>>>(b, G, w, err);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(ceil_div(ntask, kWarps)), b.nlayers, b.nseq);
+  cfg.blockDim = dim3(kCompactThreads);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // starts under the previous kernel's tail
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, k_compact, b, G, w, err);
 }
 
 }  // namespace starkv

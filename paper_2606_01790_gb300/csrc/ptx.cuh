@@ -287,6 +287,19 @@ __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t* p) {
   return v;
 }
 
+// ------------------------------------------------------------------ programmatic dependent launch
+
+// Lets the next kernel of the stream be scheduled before this one ends (it
+// still waits in griddep_wait for this kernel's completion and memory).
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Waits until the preceding kernel of the stream has completed and its memory
+// operations are visible; a no-op for a kernel launched without the
+// programmatic-serialization attribute.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // ------------------------------------------------------------------ thread-block clusters
 
 __device__ __forceinline__ uint32_t cluster_rank() {

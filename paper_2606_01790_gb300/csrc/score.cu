@@ -25,6 +25,8 @@
 // warps.  Two 256-column TMEM accumulator stages let the MMA of tile i+1 run
 // under the epilogue of tile i; TMEM is read in 16-column loads with the next
 // load in flight under the arithmetic, which runs on packed fp32 pairs.
+#include <utility>
+
 #include "common.cuh"
 #include "ptx.cuh"
 #include "score.cuh"
@@ -430,6 +432,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_lse(const __grid_con
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // the set-up above overlaps the previous kernel's tail; its outputs are read below
+  griddep_launch_dependents();
+  griddep_wait();
   const uint32_t tmem = ctl->tmem_base;
   const int64_t T = p.total_tiles;
   const int64_t fb = range_begin(T, blockIdx.x, gridDim.x);
@@ -527,6 +532,9 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // the set-up above overlaps the previous kernel's tail; its outputs are read below
+  griddep_launch_dependents();
+  griddep_wait();
   const uint32_t tmem = ctl->tmem_base;
   const int64_t T = p.total_tiles;
   const int64_t fb = range_begin(T, blockIdx.x, gridDim.x);
@@ -592,6 +600,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
 // S[g, t] = (G/H)(1/k) sum_{|j| <= k/2} S_raw[g, t + j]  (Eqs. 3-4; zero padding,
 // divisor k), S_raw being the sum of its column-quarter copies.  grid: (ceil(Lp_max / 256), nlayers * G, nseq)
 __global__ void k_pool(const __grid_constant__ SeqBatch b, int G, int H, int pool) {
+  griddep_launch_dependents();
+  griddep_wait();
   const SeqView& s = b.s[blockIdx.z];
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
   if (t >= s.Lp) return;
@@ -631,21 +641,41 @@ cudaError_t score_configure() {
   return cudaFuncSetAttribute(k_score_accum, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
+namespace {
+
+// Launch with programmatic stream serialization: the kernel may start its
+// set-up while the previous kernel of the stream drains (it waits in
+// griddep_wait before reading that kernel's outputs).
+template <typename... Args, typename... Act>
+cudaError_t launch_pdl(void (*kernel)(Args...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                       Act&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Act>(args)...);
+}
+
+}  // namespace
+
 cudaError_t score_lse_launch(const ScoreParams& p, int grid, cudaStream_t stream) {
-  k_score_lse<<<grid, kScoreThreads, score_smem_bytes(p.q_rows, p.kstages), stream>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(k_score_lse, dim3(grid), dim3(kScoreThreads), score_smem_bytes(p.q_rows, p.kstages), stream, p);
 }
 
 cudaError_t score_accum_launch(const ScoreParams& p, int grid, cudaStream_t stream) {
-  k_score_accum<<<grid, kScoreThreads, score_smem_bytes(p.q_rows, p.kstages), stream>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(k_score_accum, dim3(grid), dim3(kScoreThreads), score_smem_bytes(p.q_rows, p.kstages), stream, p);
 }
 
 cudaError_t pool_launch(const SeqBatch& b, int G, int H, int pool, int lp_max, cudaStream_t stream) {
   if (lp_max <= 0) return cudaSuccess;
   dim3 grid(ceil_div(lp_max, 256), b.nlayers * G, b.nseq);
-  k_pool<<<grid, 256, 0, stream>>>(b, G, H, pool);
-  return cudaGetLastError();
+  return launch_pdl(k_pool, grid, dim3(256), 0, stream, b, G, H, pool);
 }
 
 }  // namespace starkv

@@ -304,17 +304,18 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   const int seg = ceil_div(Lp, 32 * 32) * 32;
   const int s0 = min(Lp, warp * seg), s1 = min(Lp, s0 + seg);
 
-  if (tid < G) sh.mib_old[tid] = st.mi_bar[sl * G + tid];
-  if (tid == 0) {
-    sh.n_old = st.n[sl];
-    sh.any_tie = 0;
-  }
+  if (tid == 0) sh.any_tie = 0;
   for (int i = tid; i < kBins0; i += kCalThreads) hist[i] = 0;
   for (int i = tid; i < K * MM; i += kCalThreads) joint[i] = 0;
   for (int i = tid; i < RC; i += kCalThreads) cur[i] = 0.f;
   for (int r = tid; r < R; r += kCalThreads) rowc[r] = static_cast<uint8_t>(r * M / R);
   for (int c = tid; c < C; c += kCalThreads) colc[c] = static_cast<uint8_t>(c * M / C);
   __syncthreads();
+  // the set-up above overlaps the previous kernel's tail; its outputs are read below
+  griddep_launch_dependents();
+  griddep_wait();
+  if (tid < G) sh.mib_old[tid] = st.mi_bar[sl * G + tid];
+  if (tid == 0) sh.n_old = st.n[sl];
 
   // ================= phase 1: group g =================
   // ---- the row, staged in shared memory by one pass of independent loads:
@@ -839,13 +840,15 @@ cudaError_t calibrate_launch(const SeqBatch& b, const KParams& kp, const DevStat
   cfg.blockDim = dim3(kCalThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = kp.G;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // set-up under the previous kernel's tail
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   if (from_raw) return cudaLaunchKernelEx(&cfg, k_calibrate<true>, b, kp, st, capl);
   return cudaLaunchKernelEx(&cfg, k_calibrate<false>, b, kp, st, capl);
 }
