@@ -359,15 +359,23 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   // range, the current frame on the patch grid
   int nv = 0;
   uint32_t kmin = 0xFFFFFFFFu, kmax = 0u;
-  for (int t = tid; t < Lp; t += kCalThreads) {
-    float s;
-    if (FROM_RAW) {
-      float acc = 0.f;
+  auto pooled = [&](int t) {   // window sum in tap order, zero outside the row
+    float acc = 0.f;
+    if (half == 2 && t >= 2 && t + 2 < Lp) {   // the default window, away from the ends
+      const float x0 = stage[t - 2], x1 = stage[t - 1], x2 = stage[t], x3 = stage[t + 1], x4 = stage[t + 2];
+      acc = (((x0 + x1) + x2) + x3) + x4;
+    } else {
       for (int j = -half; j <= half; ++j) {
         const int u = t + j;
         acc += (u >= 0 && u < Lp) ? stage[u] : 0.f;
       }
-      s = acc * pscale;
+    }
+    return acc * pscale;
+  };
+  for (int t = tid; t < Lp; t += kCalThreads) {
+    float s;
+    if (FROM_RAW) {
+      s = pooled(t);
       S[t] = s;
     } else {
       s = stage[t];
