@@ -367,7 +367,9 @@ def gpu_arm(args):
     if not args.no_e2e:
         hseqs = [make_seq(si, i, None, pin=True) for i, si in enumerate(sis)]
         hws = sk.workspace(st, hseqs, host=True, device=dev)
-        h2d = sum(s.k.numel() * 2 + s.v.numel() * 2 + s.q.numel() * 2 + s.meta.numel() * 4 for s in hseqs)
+        # K, Q and metadata are uploaded; V is page-locked, so the gather reads
+        # only its kept rows in place (the same bytes as V')
+        h2d = sum(s.k.numel() * 2 + s.v_out.numel() * 2 + s.q.numel() * 2 + s.meta.numel() * 4 for s in hseqs)
         d2h = sum(s.k_out.numel() * 2 + s.v_out.numel() * 2 + s.meta_out.numel() * 4 + s.idx.numel() * 4
                   for s in hseqs)
         for _ in range(2):

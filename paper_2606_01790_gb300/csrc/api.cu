@@ -37,6 +37,9 @@ struct starkv_state {
   };
   std::vector<Rec> recs;
   std::vector<cudaEvent_t> pool;
+  // starkv_step_host: copy-in / copy-out streams and their ordering events
+  cudaStream_t pipe_in = nullptr, pipe_out = nullptr;
+  std::vector<cudaEvent_t> pipe_ev;
 };
 
 namespace {
@@ -506,6 +509,9 @@ starkv_status starkv_destroy_state(starkv_state* st) {
     cudaEventDestroy(r.b);
   }
   for (auto ev : st->pool) cudaEventDestroy(ev);
+  for (auto ev : st->pipe_ev) cudaEventDestroy(ev);
+  if (st->pipe_in) cudaStreamDestroy(st->pipe_in);
+  if (st->pipe_out) cudaStreamDestroy(st->pipe_out);
   if (e == cudaSuccess) e = cudaFree(st->mem);
   delete st;
   if (e != cudaSuccess) return set_error(STARKV_ERR_CUDA, "destroy failed: %s", cudaGetErrorString(e));
@@ -597,56 +603,114 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
   if ((s = starkv_workspace_bytes(st, seqs, nseq, 1, &need)) != STARKV_OK) return s;
   if ((s = check_ws(st, workspace, workspace_bytes, need)) != STARKV_OK) return s;
   const starkv_config& c = st->cfg;
-  cudaStream_t strm = static_cast<cudaStream_t>(stream);
+  const int G = c.n_kv_heads, NL = c.n_layers;
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  if (!st->pipe_in) {
+    CUDA_TRY(cudaStreamCreateWithFlags(&st->pipe_in, cudaStreamNonBlocking));
+    CUDA_TRY(cudaStreamCreateWithFlags(&st->pipe_out, cudaStreamNonBlocking));
+  }
+  // layers are independent: the step runs in chunks of layers so that the
+  // upload of chunk i+1 and the download of chunk i-1 overlap the compute of
+  // chunk i (the host link carries both directions at once)
+  const int chunk = std::min(NL, 4);
+  const int nchunk = (NL + chunk - 1) / chunk;
+  const size_t n_ev = 2 + 2 * static_cast<size_t>(nchunk);
+  while (st->pipe_ev.size() < n_ev) {
+    cudaEvent_t e = nullptr;
+    CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+    st->pipe_ev.push_back(e);
+  }
+  cudaEvent_t* ev = st->pipe_ev.data();
   char* cur = static_cast<char*>(workspace);
   auto take = [&](size_t bytes) {
     char* p = cur;
     cur += align256(bytes);
     return p;
   };
+  struct Rows { size_t kv_layer, q_layer, meta_layer, out_layer, lp; bool v_in_place; };
   std::vector<starkv_seq> dev(seqs, seqs + nseq);
+  std::vector<Rows> rows(nseq);
   for (int i = 0; i < nseq; ++i) {
     const starkv_seq& h = seqs[i];
     starkv_seq& d = dev[i];
-    const size_t kv = static_cast<size_t>(c.n_layers) * c.n_kv_heads * h.L * kHeadDim * 2;
-    const size_t qb = static_cast<size_t>(c.n_layers) * c.n_heads * c.window * kHeadDim * 2;
-    const size_t mb = (h.meta_layer_stride ? static_cast<size_t>(c.n_layers) * h.meta_layer_stride : h.L) * 4;
-    d.k = take(kv);
-    d.v = take(kv);
-    d.q = take(qb);
+    Rows& r = rows[i];
+    r.kv_layer = static_cast<size_t>(G) * h.L * kHeadDim * 2;
+    r.q_layer = static_cast<size_t>(c.n_heads) * c.window * kHeadDim * 2;
+    r.meta_layer = static_cast<size_t>(h.meta_layer_stride) * 4;
+    r.lp = static_cast<size_t>(h.L - c.window);
+    r.out_layer = static_cast<size_t>(h.budget + c.window);
+    const size_t mb = (h.meta_layer_stride ? static_cast<size_t>(NL) * h.meta_layer_stride : h.L) * 4;
+    d.k = take(NL * r.kv_layer);
+    // V is read only at the kept rows: from page-locked host memory the gather
+    // reads them in place instead of uploading all of V
+    cudaPointerAttributes pa;
+    r.v_in_place = cudaPointerGetAttributes(&pa, h.v) == cudaSuccess && pa.type == cudaMemoryTypeHost &&
+                   pa.devicePointer != nullptr;
+    if (!r.v_in_place) cudaGetLastError();
+    d.v = r.v_in_place ? static_cast<const void*>(pa.devicePointer) : take(NL * r.kv_layer);
+    d.q = take(NL * r.q_layer);
     d.meta = reinterpret_cast<const uint32_t*>(take(mb));
-    CUDA_TRY(cudaMemcpyAsync(const_cast<void*>(d.k), h.k, kv, cudaMemcpyHostToDevice, strm));
-    CUDA_TRY(cudaMemcpyAsync(const_cast<void*>(d.v), h.v, kv, cudaMemcpyHostToDevice, strm));
-    CUDA_TRY(cudaMemcpyAsync(const_cast<void*>(d.q), h.q, qb, cudaMemcpyHostToDevice, strm));
-    CUDA_TRY(cudaMemcpyAsync(const_cast<uint32_t*>(d.meta), h.meta, mb, cudaMemcpyHostToDevice, strm));
-    const size_t ro = h.budget + c.window, lp = h.L - c.window;
-    d.k_out = take(static_cast<size_t>(c.n_layers) * c.n_kv_heads * ro * kHeadDim * 2);
-    d.v_out = take(static_cast<size_t>(c.n_layers) * c.n_kv_heads * ro * kHeadDim * 2);
-    d.meta_out = reinterpret_cast<uint32_t*>(take(static_cast<size_t>(c.n_layers) * ro * 4));
-    d.idx = reinterpret_cast<int32_t*>(take(static_cast<size_t>(c.n_layers) * h.budget * 4));
-    d.S = h.S ? reinterpret_cast<float*>(take(static_cast<size_t>(c.n_layers) * c.n_kv_heads * lp * 4)) : nullptr;
-    d.score = h.score ? reinterpret_cast<float*>(take(static_cast<size_t>(c.n_layers) * lp * 4)) : nullptr;
-    d.stats = h.stats ? reinterpret_cast<float*>(take(static_cast<size_t>(c.n_layers) * (8 + 4 * c.n_kv_heads) * 4)) : nullptr;
+    d.k_out = take(NL * static_cast<size_t>(G) * r.out_layer * kHeadDim * 2);
+    d.v_out = take(NL * static_cast<size_t>(G) * r.out_layer * kHeadDim * 2);
+    d.meta_out = reinterpret_cast<uint32_t*>(take(NL * r.out_layer * 4));
+    d.idx = reinterpret_cast<int32_t*>(take(NL * static_cast<size_t>(h.budget) * 4));
+    d.S = h.S ? reinterpret_cast<float*>(take(NL * static_cast<size_t>(G) * r.lp * 4)) : nullptr;
+    d.score = h.score ? reinterpret_cast<float*>(take(NL * r.lp * 4)) : nullptr;
+    d.stats = h.stats ? reinterpret_cast<float*>(take(static_cast<size_t>(NL) * (8 + 4 * G) * 4)) : nullptr;
   }
   const size_t used = static_cast<size_t>(cur - static_cast<char*>(workspace));
-  s = starkv_step(st, dev.data(), nseq, cur, workspace_bytes - used, stream);
-  if (s != STARKV_OK) return s;
-  for (int i = 0; i < nseq; ++i) {
-    const starkv_seq& h = seqs[i];
-    const starkv_seq& d = dev[i];
-    const size_t ro = h.budget + c.window, lp = h.L - c.window;
-    CUDA_TRY(cudaMemcpyAsync(h.k_out, d.k_out, static_cast<size_t>(c.n_layers) * c.n_kv_heads * ro * kHeadDim * 2, cudaMemcpyDeviceToHost, strm));
-    CUDA_TRY(cudaMemcpyAsync(h.v_out, d.v_out, static_cast<size_t>(c.n_layers) * c.n_kv_heads * ro * kHeadDim * 2, cudaMemcpyDeviceToHost, strm));
-    CUDA_TRY(cudaMemcpyAsync(h.meta_out, d.meta_out, static_cast<size_t>(c.n_layers) * ro * 4, cudaMemcpyDeviceToHost, strm));
-    if (h.budget > 0)
-      CUDA_TRY(cudaMemcpyAsync(h.idx, d.idx, static_cast<size_t>(c.n_layers) * h.budget * 4, cudaMemcpyDeviceToHost, strm));
-    if (h.S && lp > 0)
-      CUDA_TRY(cudaMemcpyAsync(h.S, d.S, static_cast<size_t>(c.n_layers) * c.n_kv_heads * lp * 4, cudaMemcpyDeviceToHost, strm));
-    if (h.score && lp > 0)
-      CUDA_TRY(cudaMemcpyAsync(h.score, d.score, static_cast<size_t>(c.n_layers) * lp * 4, cudaMemcpyDeviceToHost, strm));
-    if (h.stats)
-      CUDA_TRY(cudaMemcpyAsync(h.stats, d.stats, static_cast<size_t>(c.n_layers) * (8 + 4 * c.n_kv_heads) * 4, cudaMemcpyDeviceToHost, strm));
+  // the uploads may start once earlier work on the caller's stream (which may
+  // still read these staging buffers) is done
+  CUDA_TRY(cudaEventRecord(ev[0], cs));
+  CUDA_TRY(cudaStreamWaitEvent(st->pipe_in, ev[0], 0));
+  auto h2d = [&](const void* dst, const void* src, size_t off, size_t bytes) {
+    return cudaMemcpyAsync(static_cast<char*>(const_cast<void*>(dst)) + off, static_cast<const char*>(src) + off,
+                           bytes, cudaMemcpyHostToDevice, st->pipe_in);
+  };
+  auto d2h = [&](void* dst, const void* src, size_t off, size_t bytes) {
+    return cudaMemcpyAsync(static_cast<char*>(dst) + off, static_cast<const char*>(src) + off, bytes,
+                           cudaMemcpyDeviceToHost, st->pipe_out);
+  };
+  for (int k = 0; k < nchunk; ++k) {
+    const int l0 = k * chunk, nl = std::min(chunk, NL - l0);
+    for (int i = 0; i < nseq; ++i) {
+      const starkv_seq& h = seqs[i];
+      const starkv_seq& d = dev[i];
+      const Rows& r = rows[i];
+      CUDA_TRY(h2d(d.k, h.k, l0 * r.kv_layer, nl * r.kv_layer));
+      if (!r.v_in_place) CUDA_TRY(h2d(d.v, h.v, l0 * r.kv_layer, nl * r.kv_layer));
+      CUDA_TRY(h2d(d.q, h.q, l0 * r.q_layer, nl * r.q_layer));
+      if (h.meta_layer_stride) CUDA_TRY(h2d(d.meta, h.meta, l0 * r.meta_layer, nl * r.meta_layer));
+      else if (k == 0) CUDA_TRY(h2d(d.meta, h.meta, 0, static_cast<size_t>(h.L) * 4));
+    }
+    CUDA_TRY(cudaEventRecord(ev[2 + 2 * k], st->pipe_in));
+    CUDA_TRY(cudaStreamWaitEvent(cs, ev[2 + 2 * k], 0));
+    s = run_stages(st, dev.data(), nseq, l0, nl, kScore | kStatsRaw | kSelect | kCompact, cur,
+                   workspace_bytes - used, cs);
+    if (s != STARKV_OK) return s;
+    CUDA_TRY(cudaEventRecord(ev[3 + 2 * k], cs));
+    CUDA_TRY(cudaStreamWaitEvent(st->pipe_out, ev[3 + 2 * k], 0));
+    for (int i = 0; i < nseq; ++i) {
+      const starkv_seq& h = seqs[i];
+      const starkv_seq& d = dev[i];
+      const Rows& r = rows[i];
+      const size_t kvo = static_cast<size_t>(G) * r.out_layer * kHeadDim * 2;
+      CUDA_TRY(d2h(h.k_out, d.k_out, l0 * kvo, nl * kvo));
+      CUDA_TRY(d2h(h.v_out, d.v_out, l0 * kvo, nl * kvo));
+      CUDA_TRY(d2h(h.meta_out, d.meta_out, l0 * r.out_layer * 4, nl * r.out_layer * 4));
+      if (h.budget > 0)
+        CUDA_TRY(d2h(h.idx, d.idx, l0 * static_cast<size_t>(h.budget) * 4, nl * static_cast<size_t>(h.budget) * 4));
+      if (h.S && r.lp > 0) CUDA_TRY(d2h(h.S, d.S, l0 * G * r.lp * 4, nl * G * r.lp * 4));
+      if (h.score && r.lp > 0) CUDA_TRY(d2h(h.score, d.score, l0 * r.lp * 4, nl * r.lp * 4));
+      if (h.stats) {
+        const size_t sb = static_cast<size_t>(8 + 4 * G) * 4;
+        CUDA_TRY(d2h(h.stats, d.stats, l0 * sb, nl * sb));
+      }
+    }
   }
+  // the call's results are in host memory when the caller's stream reaches here
+  CUDA_TRY(cudaEventRecord(ev[1], st->pipe_out));
+  CUDA_TRY(cudaStreamWaitEvent(cs, ev[1], 0));
   return STARKV_OK;
 }
 
