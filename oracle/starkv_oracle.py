@@ -31,6 +31,15 @@ parameter with the stated default):
   with no visual tokens: phi_g = 0 and m_g unchanged.
 * Top-B (Sec. 3.7, Algorithm 1 "Sort(TopK)"): one global token-level set per
   layer, ties to the lower index, returned ascending.
+* Per-KV-head selection (an optional mode; the paper's method is the global
+  set above; App. A.3 names head-wise top-K as the SnapKV-style alternative):
+  each group g ranks its own row s_{g,t} = max(S[g,t] beta_g D_{g,t}, 0)^(1/T_g)
+  with beta_g = (1 - lambda) + lambda G w_g, D_{g,t} from Eq. (9) with phi_g,
+  and T_g from the entropy of S[g, .] (Sec. 3.6 on that row); it keeps its own
+  B tokens (ties to the lower index), and the compressed cache of group g is
+  [X_g[I_g]; X_g,rec] with the metadata gathered per group.  beta_g is one
+  factor per row, so in this mode the MI prior scales the scores without
+  changing any set; only D changes the ranking.
 
 Parity of the absolute values of MI, w and phi on realistic inputs is
 unpinned beyond the closed forms and library cross-checks in the tests: the
@@ -304,6 +313,34 @@ def score_layer(q: np.ndarray, k: np.ndarray, window: int, p: Params) -> np.ndar
     return group_scores(a, k.shape[0])
 
 
+def calibrate_layer(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarray, row: np.ndarray,
+                    col: np.ndarray, cur_frame: int, R: int, C: int, st: LayerState,
+                    p: Params) -> Dict:
+    """Algorithm 1's per-group calibration, shared by both selection modes:
+    MI_g (Eq. 5) -> MI EMA (Eq. 6) -> prior w (Eq. 7) and lambda_n (Sec. 3.4);
+    phi_g and the m_g update (Eq. 8).  Does not modify ``st``; returns the new
+    EMAs as ``mi_bar`` and ``m_new``."""
+    G, lp = s.shape
+    vis = is_visual[:lp] != 0
+    n_cells = p.mi_grid * p.mi_grid
+    cells = spatial_cells(row[:lp][vis], col[:lp][vis], R, C, p.mi_grid)
+    mi = np.array([mutual_information(rank_bins(s[g][vis], p.mi_bins), cells, p.mi_bins, n_cells)
+                   for g in range(G)])
+    mi_bar = mi_ema(st.mi_bar, mi, p.rho_mi, st.n == 0)
+    w = subspace_prior(mi_bar, p.eps, p.tau)
+    lam_n = lambda_at(st.n, p.lam, p.n_warmup, p.n_ramp)
+    phi = np.zeros(G)
+    m_new = st.m.copy()
+    for g in range(G):
+        cur = current_row(s[g], is_visual[:lp], frame[:lp], row[:lp], col[:lp], cur_frame, R, C)
+        phi[g], m_new[g] = temporal_stability(cur, st.m[g], p.rho_t)
+    return dict(mi=mi, mi_bar=mi_bar, w=w, lam=lam_n, phi=phi, m_new=m_new)
+
+
+def _advance(st: LayerState, cal: Dict) -> None:
+    st.mi_bar, st.m, st.n = cal["mi_bar"], cal["m_new"], st.n + 1
+
+
 def select_layer(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarray, row: np.ndarray,
                  col: np.ndarray, cur_frame: int, budget: int, R: int, C: int,
                  st: LayerState, p: Params, gstar_override: Optional[np.ndarray] = None) -> Dict:
@@ -314,44 +351,70 @@ def select_layer(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarray, row: n
     ``gstar_override`` replaces argmax_g S (for tests of near-tie tokens).
     """
     G, lp = s.shape
-    vis = is_visual[:lp] != 0
     sbar = base_score(s)
     gstar = governing_group(s) if gstar_override is None else gstar_override
+    cal = calibrate_layer(s, is_visual, frame, row, col, cur_frame, R, C, st, p)
     # online MI prior (Sec. 3.4)
-    n_cells = p.mi_grid * p.mi_grid
-    cells = spatial_cells(row[:lp][vis], col[:lp][vis], R, C, p.mi_grid)
-    mi = np.array([mutual_information(rank_bins(s[g][vis], p.mi_bins), cells, p.mi_bins, n_cells)
-                   for g in range(G)])
-    mi_bar = mi_ema(st.mi_bar, mi, p.rho_mi, st.n == 0)
-    w = subspace_prior(mi_bar, p.eps, p.tau)
-    lam_n = lambda_at(st.n, p.lam, p.n_warmup, p.n_ramp)
-    beta = mi_weight(gstar, w, lam_n)
+    beta = mi_weight(gstar, cal["w"], cal["lam"])
     # temporal discount (Sec. 3.5)
-    phi = np.zeros(G)
-    m_new = st.m.copy()
-    for g in range(G):
-        cur = current_row(s[g], is_visual[:lp], frame[:lp], row[:lp], col[:lp], cur_frame, R, C)
-        phi[g], m_new[g] = temporal_stability(cur, st.m[g], p.rho_t)
-    d = temporal_decay(is_visual[:lp], frame[:lp], cur_frame, phi[gstar], p.delta, p.d_min)
+    d = temporal_decay(is_visual[:lp], frame[:lp], cur_frame, cal["phi"][gstar], p.delta, p.d_min)
     # entropy temperature (Sec. 3.6) and fused score
     h, temp = entropy_temperature(sbar, p.t_min, p.t_max, p.eps_h)
     score = final_score(sbar, beta, d, temp)
     idx = top_b(score, budget)
-    st.mi_bar, st.m, st.n = mi_bar, m_new, st.n + 1
-    return dict(sbar=sbar, gstar=gstar, mi=mi, mi_bar=mi_bar, w=w, lam=lam_n, beta=beta,
-                phi=phi, D=d, H=h, T=temp, score=score, idx=idx)
+    _advance(st, cal)
+    return dict(sbar=sbar, gstar=gstar, mi=cal["mi"], mi_bar=cal["mi_bar"], w=cal["w"],
+                lam=cal["lam"], beta=beta, phi=cal["phi"], D=d, H=h, T=temp, score=score, idx=idx)
+
+
+def select_layer_per_head(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarray,
+                          row: np.ndarray, col: np.ndarray, cur_frame: int, budget: int, R: int,
+                          C: int, st: LayerState, p: Params) -> Dict:
+    """Per-KV-head selection mode (the SnapKV-style head-wise top-K of App. A.3,
+    with the STaR-KV factors of group g): score [G][L_past], idx [G][B], one
+    temperature per group.  ``st`` is updated in place as in select_layer."""
+    G, lp = s.shape
+    cal = calibrate_layer(s, is_visual, frame, row, col, cur_frame, R, C, st, p)
+    own = np.arange(G)
+    beta = mi_weight(own, cal["w"], cal["lam"])                       # [G]
+    d = np.stack([temporal_decay(is_visual[:lp], frame[:lp], cur_frame, np.full(lp, cal["phi"][g]),
+                                 p.delta, p.d_min) for g in range(G)])  # [G][L_past]
+    ht = [entropy_temperature(s[g], p.t_min, p.t_max, p.eps_h) for g in range(G)]
+    h = np.array([x[0] for x in ht])
+    temp = np.array([x[1] for x in ht])
+    score = np.stack([final_score(s[g], beta[g], d[g], temp[g]) for g in range(G)])
+    idx = np.stack([top_b(score[g], budget) for g in range(G)]) if G else np.zeros((0, budget), np.int64)
+    _advance(st, cal)
+    return dict(mi=cal["mi"], mi_bar=cal["mi_bar"], w=cal["w"], lam=cal["lam"], beta=beta,
+                phi=cal["phi"], D=d, H=h, T=temp, score=score, idx=idx)
+
+
+def compact_per_head(x: np.ndarray, idx: np.ndarray, window: int) -> np.ndarray:
+    """Eq. (11) per group: X'[g] = [X[g, I_g]; X[g, L_past:]] for [G][L][d]
+    caches, and [G][B + w] metadata gathered per group for [L] arrays."""
+    if x.ndim == 1:
+        return np.stack([compact(x, idx[g], window) for g in range(idx.shape[0])])
+    return np.stack([compact(x[g], idx[g], window) for g in range(x.shape[0])])
 
 
 def step_layer(q: np.ndarray, k: np.ndarray, v: np.ndarray, is_visual: np.ndarray,
                frame: np.ndarray, row: np.ndarray, col: np.ndarray, cur_frame: int,
-               budget: int, window: int, R: int, C: int, st: LayerState, p: Params) -> Dict:
+               budget: int, window: int, R: int, C: int, st: LayerState, p: Params,
+               per_head: bool = False) -> Dict:
     """Algorithm 1 for one layer: scores, calibration, selection and the
-    compressed cache (K', V', metadata')."""
+    compressed cache (K', V', metadata'); ``per_head`` picks the per-KV-head
+    selection mode (idx [G][B], metadata' [G][B + w])."""
     s = score_layer(q, k, window, p)
-    out = select_layer(s, is_visual, frame, row, col, cur_frame, budget, R, C, st, p)
+    meta = (is_visual, frame, row, col)
+    if per_head:
+        out = select_layer_per_head(s, *meta, cur_frame, budget, R, C, st, p)
+        gather = compact_per_head
+    else:
+        out = select_layer(s, *meta, cur_frame, budget, R, C, st, p)
+        gather = compact
     idx = out["idx"]
     out["S"] = s
-    out["k_out"] = compact(k, idx, window)
-    out["v_out"] = compact(v, idx, window)
-    out["meta_out"] = tuple(compact(a, idx, window) for a in (is_visual, frame, row, col))
+    out["k_out"] = gather(k, idx, window)
+    out["v_out"] = gather(v, idx, window)
+    out["meta_out"] = tuple(gather(a, idx, window) for a in meta)
     return out

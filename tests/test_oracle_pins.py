@@ -350,3 +350,137 @@ def test_single_group_prior_is_neutral():
     o = O.select_layer(O.score_layer(q, k, q.shape[1], p), *meta, F_, 9, 4, 5, st, p)
     np.testing.assert_allclose(o["beta"], 1.0)
     assert st.n == 1 and o["w"].tolist() == [1.0]
+
+
+# ------------------------------------------------------------------ per-KV-head selection mode
+
+def _headwise_topk(s_row, b):
+    """Head-wise top-K by a plain sort (values descending, then lower index first)."""
+    order = sorted(range(len(s_row)), key=lambda i: (-float(s_row[i]), i))
+    return sorted(order[:b])
+
+
+def test_per_head_base_configuration_equals_headwise_topk_of_pooled_attention():
+    """lambda = 0, no temporal term, T = 1: each group keeps the top-B of its own
+    pooled, group-averaged window attention (SnapKV-style head-wise top-K,
+    App. A.3), computed here with torch."""
+    q, k, meta, F_ = _small_case(40, G=4)
+    w = q.shape[1]
+    p = O.Params(lam=0.0, delta=0.0, t_min=1.0, t_max=1.0, pool_kernel=3)
+    st = O.LayerState.fresh(4, 4, 5)
+    out = O.select_layer_per_head(O.score_layer(q, k, w, p), *meta, F_, 13, 4, 5, st, p)
+    a = torch.from_numpy(_torch_window_attention(q, k, w))
+    a = F.avg_pool1d(a[None], 3, stride=1, padding=1, count_include_pad=True)[0]
+    s = a.reshape(4, -1, a.shape[-1]).mean(dim=1).numpy()
+    assert out["idx"].shape == (4, 13)
+    for g in range(4):
+        assert out["idx"][g].tolist() == _headwise_topk(s[g], 13)
+    assert len({tuple(r) for r in out["idx"].tolist()}) > 1   # the groups really differ
+
+
+def test_per_head_single_group_equals_global_mode():
+    q, k, meta, F_ = _small_case(41, H=4, G=1)
+    p = O.Params(n_warmup=0, n_ramp=0)
+    s = O.score_layer(q, k, q.shape[1], p)
+    st0 = O.LayerState.fresh(1, 4, 5)
+    st0.n, st0.mi_bar, st0.m = 2, np.array([0.3]), _rng(6).random((1, 20))
+    st1 = st0.copy()
+    g = O.select_layer(s, *meta, F_, 11, 4, 5, st0, p)
+    h = O.select_layer_per_head(s, *meta, F_, 11, 4, 5, st1, p)
+    np.testing.assert_allclose(h["score"][0], g["score"], rtol=1e-14)
+    assert h["idx"][0].tolist() == g["idx"].tolist()
+    assert h["T"][0] == g["T"] and st0.n == st1.n == 3
+    np.testing.assert_allclose(st1.m, st0.m, rtol=0)
+
+
+def test_per_head_temperature_is_each_rows_own():
+    """Sec. 3.6 per row: a uniform row has H = 1 (T = T_max), a one-hot row H = 0
+    (T = T_min); a third row lies in between."""
+    lp = 64
+    s = np.stack([np.full(lp, 0.5), np.eye(lp)[7] * 3.0, _rng(7).random(lp)])
+    z = np.zeros(lp, np.int64)
+    p = O.Params(t_min=0.9, t_max=1.1)
+    o = O.select_layer_per_head(s, z, z, z, z, 0, 5, 4, 5, O.LayerState.fresh(3, 4, 5), p)
+    np.testing.assert_allclose(o["H"][:2], [1.0, 0.0], atol=1e-9)
+    np.testing.assert_allclose(o["T"][:2], [1.1, 0.9], atol=1e-9)
+    assert 0.0 < o["H"][2] < 1.0
+    assert 7 in o["idx"][1].tolist()
+
+
+def test_per_head_sets_invariant_to_prior_and_temperature():
+    """beta_g is one factor per row and x -> x^(1/T) is increasing, so neither
+    lambda, tau nor the temperature range changes any group's set."""
+    q, k, meta, F_ = _small_case(42, G=4)
+    s = O.score_layer(q, k, q.shape[1], O.Params())
+    st0 = O.LayerState.fresh(4, 4, 5)
+    st0.n, st0.mi_bar, st0.m = 6, np.array([0.1, 0.7, 0.3, 0.2]), _rng(8).random((4, 20))
+    sets = []
+    for lam, tau, tmin, tmax in [(0.0, 1.0, 1.0, 1.0), (0.5, 1.0, 0.95, 1.05), (1.0, 0.1, 0.5, 3.0)]:
+        p = O.Params(lam=lam, tau=tau, t_min=tmin, t_max=tmax, n_warmup=0, n_ramp=0, delta=0.7)
+        sets.append(O.select_layer_per_head(s, *meta, F_, 15, 4, 5, st0.copy(), p)["idx"].tolist())
+    assert all(x == sets[0] for x in sets)
+
+
+def test_per_head_temporal_discount_uses_each_groups_own_phi():
+    """Group 0's m equals its current-frame row (phi_0 = 1), group 1's m is
+    orthogonal to its row (phi_1 = 0), and group 1 governs every token
+    (S[1] > S[0]).  With D_min = 0 and a steep delta, group 0 keeps only text
+    and current-frame tokens (its B largest among them), group 1 is
+    undiscounted (plain top-B of its row)."""
+    q, k, meta, F_ = _small_case(43, G=2, shots=3, n_text=40)
+    is_vis, frame, row, col = meta
+    lp = k.shape[1] - q.shape[1]
+    r = _rng(11)
+    s0 = 0.01 + r.random(lp)
+    s = np.stack([s0, 1.5 * s0 + 0.5 * r.random(lp)])
+    R, C = 4, 5
+    cur = np.zeros((2, R * C))
+    for t in range(lp):
+        if is_vis[t] and frame[t] == F_:
+            cur[:, row[t] * C + col[t]] = s[:, t]
+    m1 = r.standard_normal(R * C)
+    m1 -= (m1 @ cur[1]) / (cur[1] @ cur[1]) * cur[1]
+    st = O.LayerState.fresh(2, R, C)
+    st.n, st.mi_bar, st.m = 3, np.array([0.2, 0.4]), np.stack([cur[0], m1])
+    p = O.Params(delta=200.0, d_min=0.0, n_warmup=0, n_ramp=0)
+    B = 10
+    o = O.select_layer_per_head(s, *meta, F_, B, R, C, st, p)
+    np.testing.assert_allclose(o["phi"], [1.0, 0.0], atol=1e-12)
+    fresh = np.array([(not is_vis[t]) or frame[t] == F_ for t in range(lp)])
+    assert fresh.sum() >= B
+    keep0 = sorted(sorted(np.nonzero(fresh)[0], key=lambda t: (-s[0, t], t))[:B])
+    assert o["idx"][0].tolist() == keep0
+    assert o["idx"][0].tolist() != _headwise_topk(s[0], B)   # the discount took part
+    assert o["idx"][1].tolist() == _headwise_topk(s[1], B)
+
+
+def test_per_head_selection_invariant_to_token_permutation():
+    q, k, meta, F_ = _small_case(44, G=4)
+    w = q.shape[1]
+    L = k.shape[1]
+    lp = L - w
+    p = O.Params(pool_kernel=1, n_warmup=0, n_ramp=0)
+    st0 = O.LayerState.fresh(4, 4, 5)
+    st0.n, st0.mi_bar, st0.m = 3, np.array([0.2, 0.5, 0.1, 0.9]), _rng(10).random((4, 20))
+    perm = np.r_[_rng(45).permutation(lp), np.arange(lp, L)]
+    outs = []
+    for pm in (np.arange(L), perm):
+        o = O.select_layer_per_head(O.score_layer(q, k[:, pm], w, p), *(a[pm] for a in meta), F_, 9,
+                                    4, 5, st0.copy(), p)
+        outs.append([set(pm[r].tolist()) for r in o["idx"]])
+    assert outs[0] == outs[1]
+
+
+def test_compact_per_head_vs_index_select():
+    r = _rng(46)
+    G, L, d, w, B = 3, 30, 8, 4, 6
+    x = r.standard_normal((G, L, d))
+    meta = r.integers(0, 1 << 20, L)
+    idx = np.stack([np.sort(r.choice(L - w, B, replace=False)) for _ in range(G)])
+    got = O.compact_per_head(x, idx, w)
+    got_m = O.compact_per_head(meta, idx, w)
+    for g in range(G):
+        rows = torch.cat([torch.from_numpy(idx[g]), torch.arange(L - w, L)])
+        ref = torch.from_numpy(x[g]).index_select(0, rows)
+        assert torch.equal(torch.from_numpy(got[g]), ref)
+        assert torch.equal(torch.from_numpy(got_m[g]), torch.from_numpy(meta).index_select(0, rows))
