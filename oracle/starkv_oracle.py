@@ -313,27 +313,35 @@ def score_layer(q: np.ndarray, k: np.ndarray, window: int, p: Params) -> np.ndar
     return group_scores(a, k.shape[0])
 
 
+def _group_meta(a: np.ndarray, g: int) -> np.ndarray:
+    """Metadata array of group g: a shared [L] array, or row g of a per-group
+    [G][L] array (per-KV-head mode after a per-group compaction)."""
+    return a[g] if a.ndim == 2 else a
+
+
 def calibrate_layer(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarray, row: np.ndarray,
                     col: np.ndarray, cur_frame: int, R: int, C: int, st: LayerState,
                     p: Params) -> Dict:
     """Algorithm 1's per-group calibration, shared by both selection modes:
     MI_g (Eq. 5) -> MI EMA (Eq. 6) -> prior w (Eq. 7) and lambda_n (Sec. 3.4);
-    phi_g and the m_g update (Eq. 8).  Does not modify ``st``; returns the new
-    EMAs as ``mi_bar`` and ``m_new``."""
+    phi_g and the m_g update (Eq. 8).  The metadata arrays are [L] (shared) or
+    [G][L] (one row per group).  Does not modify ``st``; returns the new EMAs
+    as ``mi_bar`` and ``m_new``."""
     G, lp = s.shape
-    vis = is_visual[:lp] != 0
     n_cells = p.mi_grid * p.mi_grid
-    cells = spatial_cells(row[:lp][vis], col[:lp][vis], R, C, p.mi_grid)
-    mi = np.array([mutual_information(rank_bins(s[g][vis], p.mi_bins), cells, p.mi_bins, n_cells)
-                   for g in range(G)])
-    mi_bar = mi_ema(st.mi_bar, mi, p.rho_mi, st.n == 0)
-    w = subspace_prior(mi_bar, p.eps, p.tau)
-    lam_n = lambda_at(st.n, p.lam, p.n_warmup, p.n_ramp)
+    mi = np.zeros(G)
     phi = np.zeros(G)
     m_new = st.m.copy()
     for g in range(G):
-        cur = current_row(s[g], is_visual[:lp], frame[:lp], row[:lp], col[:lp], cur_frame, R, C)
+        vis_g, fr_g, row_g, col_g = (_group_meta(a, g)[:lp] for a in (is_visual, frame, row, col))
+        vis = vis_g != 0
+        cells = spatial_cells(row_g[vis], col_g[vis], R, C, p.mi_grid)
+        mi[g] = mutual_information(rank_bins(s[g][vis], p.mi_bins), cells, p.mi_bins, n_cells)
+        cur = current_row(s[g], vis_g, fr_g, row_g, col_g, cur_frame, R, C)
         phi[g], m_new[g] = temporal_stability(cur, st.m[g], p.rho_t)
+    mi_bar = mi_ema(st.mi_bar, mi, p.rho_mi, st.n == 0)
+    w = subspace_prior(mi_bar, p.eps, p.tau)
+    lam_n = lambda_at(st.n, p.lam, p.n_warmup, p.n_ramp)
     return dict(mi=mi, mi_bar=mi_bar, w=w, lam=lam_n, phi=phi, m_new=m_new)
 
 
@@ -351,6 +359,7 @@ def select_layer(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarray, row: n
     ``gstar_override`` replaces argmax_g S (for tests of near-tie tokens).
     """
     G, lp = s.shape
+    assert is_visual.ndim == 1, "the global mode ranks tokens shared by every group"
     sbar = base_score(s)
     gstar = governing_group(s) if gstar_override is None else gstar_override
     cal = calibrate_layer(s, is_visual, frame, row, col, cur_frame, R, C, st, p)
@@ -372,13 +381,15 @@ def select_layer_per_head(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarra
                           C: int, st: LayerState, p: Params) -> Dict:
     """Per-KV-head selection mode (the SnapKV-style head-wise top-K of App. A.3,
     with the STaR-KV factors of group g): score [G][L_past], idx [G][B], one
-    temperature per group.  ``st`` is updated in place as in select_layer."""
+    temperature per group.  The metadata arrays are [L] or [G][L] (each group's
+    own tokens).  ``st`` is updated in place as in select_layer."""
     G, lp = s.shape
     cal = calibrate_layer(s, is_visual, frame, row, col, cur_frame, R, C, st, p)
     own = np.arange(G)
     beta = mi_weight(own, cal["w"], cal["lam"])                       # [G]
-    d = np.stack([temporal_decay(is_visual[:lp], frame[:lp], cur_frame, np.full(lp, cal["phi"][g]),
-                                 p.delta, p.d_min) for g in range(G)])  # [G][L_past]
+    d = np.stack([temporal_decay(_group_meta(is_visual, g)[:lp], _group_meta(frame, g)[:lp], cur_frame,
+                                 np.full(lp, cal["phi"][g]), p.delta, p.d_min)
+                  for g in range(G)])                                  # [G][L_past]
     ht = [entropy_temperature(s[g], p.t_min, p.t_max, p.eps_h) for g in range(G)]
     h = np.array([x[0] for x in ht])
     temp = np.array([x[1] for x in ht])
@@ -391,9 +402,11 @@ def select_layer_per_head(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarra
 
 def compact_per_head(x: np.ndarray, idx: np.ndarray, window: int) -> np.ndarray:
     """Eq. (11) per group: X'[g] = [X[g, I_g]; X[g, L_past:]] for [G][L][d]
-    caches, and [G][B + w] metadata gathered per group for [L] arrays."""
+    caches, and [G][B + w] metadata gathered per group for [L] or [G][L] arrays."""
     if x.ndim == 1:
         return np.stack([compact(x, idx[g], window) for g in range(idx.shape[0])])
+    if x.ndim == 2:   # [G][L] metadata, one row per group
+        return np.stack([compact(x[g], idx[g], window) for g in range(idx.shape[0])])
     return np.stack([compact(x[g], idx[g], window) for g in range(x.shape[0])])
 
 

@@ -484,3 +484,28 @@ def test_compact_per_head_vs_index_select():
         ref = torch.from_numpy(x[g]).index_select(0, rows)
         assert torch.equal(torch.from_numpy(got[g]), ref)
         assert torch.equal(torch.from_numpy(got_m[g]), torch.from_numpy(meta).index_select(0, rows))
+
+
+def test_per_head_per_group_metadata_follows_each_groups_tokens():
+    """Per-group metadata rows: shuffling group g's tokens (its S row and its
+    metadata row together, each group with its own permutation) maps every
+    group's kept set and every group statistic through that permutation; a row
+    of metadata equal for all groups gives the shared-metadata result."""
+    q, k, meta, F_ = _small_case(47, G=3, shots=3, n_text=30)
+    lp = k.shape[1] - q.shape[1]
+    s = O.score_layer(q, k, q.shape[1], O.Params(pool_kernel=1))
+    p = O.Params(n_warmup=0, n_ramp=0, delta=0.5)
+    st0 = O.LayerState.fresh(3, 4, 5)
+    st0.n, st0.mi_bar, st0.m = 4, np.array([0.3, 0.1, 0.6]), _rng(12).random((3, 20))
+    shared = O.select_layer_per_head(s, *meta, F_, 12, 4, 5, st0.copy(), p)
+    tiled = O.select_layer_per_head(s, *(np.tile(a[:lp], (3, 1)) for a in meta), F_, 12, 4, 5,
+                                    st0.copy(), p)
+    assert shared["idx"].tolist() == tiled["idx"].tolist()
+    perms = [_rng(48 + g).permutation(lp) for g in range(3)]
+    s_p = np.stack([s[g][perms[g]] for g in range(3)])
+    meta_p = tuple(np.stack([a[:lp][perms[g]] for g in range(3)]) for a in meta)
+    o = O.select_layer_per_head(s_p, *meta_p, F_, 12, 4, 5, st0.copy(), p)
+    for g in range(3):
+        assert sorted(perms[g][o["idx"][g]].tolist()) == shared["idx"][g].tolist()
+    np.testing.assert_allclose(o["mi"], shared["mi"], rtol=1e-12)
+    np.testing.assert_allclose(o["phi"], shared["phi"], rtol=1e-12)
