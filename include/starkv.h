@@ -12,6 +12,13 @@
  *   4. reshape by an entropy-derived temperature (Sec. 3.6);
  *   5. keep the global top-B historical tokens plus the recent window and
  *      gather them into a new contiguous cache (Sec. 3.7).
+ * An optional per-KV-head selection mode (select_mode = STARKV_SELECT_PER_HEAD,
+ * the head-wise top-K of App. A.3 with the STaR-KV factors) lets each group g
+ * keep its own B tokens: it ranks s_{g,t} = max(S[g,t] beta_g D_{g,t}, 0)^(1/T_g)
+ * with beta_g = (1 - lambda) + lambda G w_g, D_{g,t} of Eq. (9) with phi_g and
+ * T_g from the entropy of S[g, .] (Sec. 3.6 on that row).  beta_g is one factor
+ * per row, so in this mode the MI prior scales the scores without changing
+ * any group's set.
  *
  * Conventions shared by every call
  * --------------------------------
@@ -27,12 +34,16 @@
  * - Layouts (all row-major, contiguous):
  *     k, v        bf16  [n_layers][G][L][d]
  *     q           bf16  [n_layers][H][w][d]   post-RoPE queries of the last w tokens
- *     meta        u32   [n_layers][L]  or [L] shared (meta_layer_stride = 0)
+ *     meta        u32   [n_layers][L]  or [L] shared (meta_layer_stride = 0);
+ *                       per-KV-head mode: optionally one row per group,
+ *                       [n_layers][G][L] (meta_group_stride = L, see below)
  *     S           f32   [n_layers][G][L_p]     group score map, L_p = L - w
- *     score       f32   [n_layers][L_p]        fused score s_t
- *     idx         i32   [n_layers][B]          kept historical positions, ascending
+ *     score       f32   [n_layers][P][L_p]     fused score s_t (s_{g,t})
+ *     idx         i32   [n_layers][P][B]       kept historical positions, ascending
  *     k_out,v_out bf16  [n_layers][G][B + w][d]
- *     meta_out    u32   [n_layers][B + w]
+ *     meta_out    u32   [n_layers][P][B + w]
+ *   where P = 1 in the global selection mode and P = G in the per-KV-head mode
+ *   (row g of idx / meta_out belongs to group g of k_out / v_out).
  *     stats       f32   [n_layers][STARKV_STATS_STRIDE(G)]
  *   Token metadata word: bit 31 = visual, bits 20..30 = frame id f(t),
  *   bits 10..19 = patch row r_t, bits 0..9 = patch column c_t (Sec. 3.1).
@@ -96,7 +107,12 @@ typedef struct {
   float t_min, t_max;   /* AEB temperature range (Sec. 3.6)                        */
   float eps;            /* epsilon of the min-max prior (Eq. 7)                    */
   float eps_h;          /* epsilon of the AEB entropy (Algorithm 1)                */
+  int32_t select_mode;  /* STARKV_SELECT_GLOBAL (the paper's, default) or
+                           STARKV_SELECT_PER_HEAD (one top-B set per KV group)     */
 } starkv_config;
+
+/* Values of starkv_config.select_mode. */
+enum { STARKV_SELECT_GLOBAL = 0, STARKV_SELECT_PER_HEAD = 1 };
 
 /* One sequence (trajectory) of a batch: inputs and caller-owned outputs.  For
  * per-layer calls (score_layer / select / compact) the `layer` argument picks
@@ -113,12 +129,19 @@ typedef struct {
   int32_t slot;                 /* state slot in [0, max_seqs)                      */
   void* k_out;                  /* bf16 [n_layers][G][B + w][d]       (compact)    */
   void* v_out;                  /* bf16 [n_layers][G][B + w][d]       (compact)    */
-  uint32_t* meta_out;           /* u32  [n_layers][B + w]             (compact)    */
-  int32_t* idx;                 /* i32  [n_layers][B]      select writes, compact reads */
+  uint32_t* meta_out;           /* u32  [n_layers][P][B + w]          (compact)    */
+  int32_t* idx;                 /* i32  [n_layers][P][B]   select writes, compact reads */
   float* S;                     /* f32  [n_layers][G][L_p] score_layer writes, select
                                    reads; may be NULL for starkv_step (workspace)   */
-  float* score;                 /* f32  [n_layers][L_p] fused s_t, optional (NULL)  */
+  float* score;                 /* f32  [n_layers][P][L_p] fused s_t, optional (NULL) */
   float* stats;                 /* f32  [n_layers][STARKV_STATS_STRIDE(G)], optional */
+  int64_t meta_group_stride;    /* elements between the metadata rows of groups g
+                                   and g + 1 of one layer: 0 = every group shares
+                                   one row (required in the global mode), else >= L
+                                   (per-KV-head mode, where each group's cache holds
+                                   its own tokens after a compaction); with a
+                                   nonzero meta_layer_stride it must be
+                                   >= (G - 1) * meta_group_stride + L                */
 } starkv_seq;
 
 /* Per-layer diagnostics written to starkv_seq.stats (floats):
@@ -127,8 +150,13 @@ typedef struct {
  *   [8 + g]       MI_g of this step            (Eq. 5)
  *   [8 + G + g]   MI_bar_g after the EMA       (Eq. 6)
  *   [8 + 2G + g]  w_g                          (Eq. 7)
- *   [8 + 3G + g]  phi_g                        (Eq. 8)                         */
-#define STARKV_STATS_STRIDE(G) (8 + 4 * (G))
+ *   [8 + 3G + g]  phi_g                        (Eq. 8)
+ *   [8 + 4G + g]  H_hat of the row group g ranks: s_bar (global mode, the same
+ *                 for every g) or S[g, .] (per-KV-head mode)
+ *   [8 + 5G + g]  its temperature T
+ * In the per-KV-head mode [0] and [1] are the means of [8 + 4G ..] and
+ * [8 + 5G ..] over g.                                                         */
+#define STARKV_STATS_STRIDE(G) (8 + 6 * (G))
 
 typedef struct starkv_state starkv_state;
 
@@ -191,13 +219,16 @@ starkv_status starkv_score_layer_noalloc(starkv_state* st, int32_t layer, const 
  * S of layer `layer`: s_bar, g*, online MI per group (Eq. 5) -> EMA (Eq. 6) ->
  * prior w (Eq. 7) -> beta; phi_g and the m_g update (Eq. 8) -> D_t (Eq. 9);
  * H_hat and T (Sec. 3.6); s_t = max(s_bar beta D, 0)^(1/T); global top-B with
- * ties to the lower index -> idx ascending.  Writes idx, and score / stats when
- * non-NULL.  Advances this layer's state by one step (n += 1 and both EMAs). */
+ * ties to the lower index -> idx ascending (per-KV-head mode: each group's own
+ * scores and top-B, see the top of this file).  Writes idx, and score / stats
+ * when non-NULL.  Advances this layer's state by one step (n += 1 and both
+ * EMAs). */
 starkv_status starkv_select(starkv_state* st, int32_t layer, const starkv_seq* seqs,
                             int32_t nseq, void* workspace, size_t workspace_bytes, void* stream);
 
 /* Sec. 3.7, Eq. (11): K' = [K_past[I]; K_rec], V' = [V_past[I]; V_rec] and the
- * same gather of meta, for layer `layer`, from idx.  Bit copies. */
+ * same gather of meta, for layer `layer`, from idx.  Bit copies.  In the
+ * per-KV-head mode group g gathers its own rows idx[g] (and meta_out[g]). */
 starkv_status starkv_compact(starkv_state* st, int32_t layer, const starkv_seq* seqs,
                              int32_t nseq, void* workspace, size_t workspace_bytes, void* stream);
 

@@ -144,6 +144,8 @@ starkv_status validate_config(const starkv_config& c) {
   if (c.n_warmup < 0 || c.n_ramp < 0) return set_error(STARKV_ERR_INVALID_ARG, "config: negative schedule");
   if (!(c.t_min > 0.f) || !(c.t_max > 0.f) || !(c.tau > 0.f))
     return set_error(STARKV_ERR_INVALID_ARG, "config: t_min, t_max and tau must be > 0");
+  if (c.select_mode != STARKV_SELECT_GLOBAL && c.select_mode != STARKV_SELECT_PER_HEAD)
+    return set_error(STARKV_ERR_INVALID_ARG, "config: select_mode must be 0 (global) or 1 (per KV head)");
   if (!(c.rho_mi >= 0.f && c.rho_mi <= 1.f) || !(c.rho_t >= 0.f && c.rho_t <= 1.f) ||
       !(c.d_min >= 0.f && c.d_min <= 1.f) || !(c.eps >= 0.f) || !(c.eps_h >= 0.f) || !(c.delta >= 0.f))
     return set_error(STARKV_ERR_INVALID_ARG, "config: a rate or epsilon is out of range");
@@ -176,8 +178,15 @@ starkv_status validate_seqs(const starkv_state* st, const starkv_seq* seqs, int 
     if ((need & kNeedV) && (!s.v || !aligned16(s.v))) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: v NULL or not 16-byte aligned", i);
     if (need & kNeedMeta) {
       if (!s.meta) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: meta is NULL", i);
-      if (s.meta_layer_stride != 0 && s.meta_layer_stride < s.L)
-        return set_error(STARKV_ERR_INVALID_ARG, "seq %d: meta_layer_stride must be 0 or >= L", i);
+      if (s.meta_group_stride != 0) {
+        if (c.select_mode != STARKV_SELECT_PER_HEAD)
+          return set_error(STARKV_ERR_INVALID_ARG, "seq %d: meta_group_stride must be 0 in the global selection mode", i);
+        if (s.meta_group_stride < s.L)
+          return set_error(STARKV_ERR_INVALID_ARG, "seq %d: meta_group_stride must be 0 or >= L", i);
+      }
+      const int64_t span = static_cast<int64_t>(c.n_kv_heads - 1) * s.meta_group_stride + s.L;
+      if (s.meta_layer_stride != 0 && s.meta_layer_stride < span)
+        return set_error(STARKV_ERR_INVALID_ARG, "seq %d: meta_layer_stride must be 0 or >= (G-1)*meta_group_stride + L", i);
     }
     if ((need & kNeedS) && !s.S && lp > 0) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: S is NULL", i);
     if ((need & kNeedIdx) && !s.idx && s.budget > 0) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: idx is NULL", i);
@@ -197,6 +206,7 @@ KParams make_kparams(const starkv_state* st) {
   k.n_warmup = c.n_warmup; k.n_ramp = c.n_ramp;
   k.lambda = c.lambda; k.tau = c.tau; k.rho_mi = c.rho_mi; k.rho_t = c.rho_t; k.delta = c.delta;
   k.d_min = c.d_min; k.t_min = c.t_min; k.t_max = c.t_max; k.eps = c.eps; k.eps_h = c.eps_h;
+  k.per_head = c.select_mode == STARKV_SELECT_PER_HEAD;
   k.wait_ns = st->wait_ns;
   return k;
 }
@@ -208,6 +218,13 @@ struct WsPlan {
 };
 
 int tiles_of(int lp) { return (lp + kTileKeys - 1) / kTileKeys; }
+
+// Rows of idx, score and meta_out per layer: 1 (global selection) or G (per KV head).
+size_t sel_rows(const starkv_config& c) {
+  return c.select_mode == STARKV_SELECT_PER_HEAD ? static_cast<size_t>(c.n_kv_heads) : 1;
+}
+
+size_t stats_bytes(const starkv_config& c) { return static_cast<size_t>(STARKV_STATS_STRIDE(c.n_kv_heads)) * 4; }
 
 // ws_score: the calibration kernel runs (fused score region; key/cell region
 // of the rows longer than its shared-memory capacity).
@@ -239,7 +256,7 @@ void plan_ws(const starkv_state* st, const starkv_seq* seqs, int nseq, int nlaye
     }
     if (ws_score && !seqs[i].score) {
       p->score_off[i] = off;
-      off += align256(static_cast<size_t>(c.n_layers) * lp * sizeof(float));
+      off += align256(static_cast<size_t>(c.n_layers) * sel_rows(c) * lp * sizeof(float));
     }
   }
   p->total = std::max<size_t>(off, 256);
@@ -252,6 +269,7 @@ SeqView make_view(const starkv_state* st, const starkv_seq& s, char* ws, const W
   v.v = static_cast<const __nv_bfloat16*>(s.v);
   v.meta = s.meta;
   v.meta_layer_stride = s.meta_layer_stride;
+  v.meta_group_stride = s.meta_group_stride;
   v.L = s.L;
   v.Lp = s.L - c.window;
   v.cur_frame = s.cur_frame;
@@ -386,27 +404,34 @@ starkv_status run_stages(starkv_state* st, const starkv_seq* seqs, int nseq, int
       }));
     if ((stages & kCompact) && rows_out_max > 0)
       CUDA_TRY(launch(st, STARKV_KERNEL_COMPACT, stream, [&] {
-        return compact_launch(b, c.n_kv_heads, c.window, rows_out_max, st->num_sms, st->dev.err, stream);
+        return compact_launch(b, c.n_kv_heads, c.window, kp.per_head, rows_out_max, st->dev.err, stream);
       }));
   }
   return STARKV_OK;
 }
 
+// Elements of a metadata buffer over `nl` layers (one layer if it is shared).
+size_t meta_elems(const starkv_config& c, const starkv_seq& s, int nl) {
+  if (s.meta_layer_stride) return static_cast<size_t>(nl) * s.meta_layer_stride;
+  return static_cast<size_t>(c.n_kv_heads - 1) * s.meta_group_stride + s.L;
+}
+
 size_t seq_bytes_in(const starkv_config& c, const starkv_seq& s) {
   const size_t kv = static_cast<size_t>(c.n_layers) * c.n_kv_heads * s.L * kHeadDim * 2;
   const size_t q = static_cast<size_t>(c.n_layers) * c.n_heads * c.window * kHeadDim * 2;
-  const size_t meta = (s.meta_layer_stride ? static_cast<size_t>(c.n_layers) * s.meta_layer_stride : s.L) * 4;
+  const size_t meta = meta_elems(c, s, c.n_layers) * 4;
   return align256(kv) * 2 + align256(q) + align256(meta);
 }
 
 size_t seq_bytes_out(const starkv_config& c, const starkv_seq& s) {
   const size_t ro = s.budget + c.window, lp = s.L - c.window;
   size_t b = align256(static_cast<size_t>(c.n_layers) * c.n_kv_heads * ro * kHeadDim * 2) * 2;
-  b += align256(static_cast<size_t>(c.n_layers) * ro * 4);
-  b += align256(static_cast<size_t>(c.n_layers) * s.budget * 4);
+  const size_t P = sel_rows(c);
+  b += align256(static_cast<size_t>(c.n_layers) * P * ro * 4);
+  b += align256(static_cast<size_t>(c.n_layers) * P * s.budget * 4);
   if (s.S) b += align256(static_cast<size_t>(c.n_layers) * c.n_kv_heads * lp * 4);
-  if (s.score) b += align256(static_cast<size_t>(c.n_layers) * lp * 4);
-  if (s.stats) b += align256(static_cast<size_t>(c.n_layers) * (8 + 4 * c.n_kv_heads) * 4);
+  if (s.score) b += align256(static_cast<size_t>(c.n_layers) * P * lp * 4);
+  if (s.stats) b += align256(static_cast<size_t>(c.n_layers) * stats_bytes(c));
   return b;
 }
 
@@ -440,6 +465,7 @@ void starkv_default_config(starkv_config* c) {
   c->t_max = 1.05f;
   c->eps = 1e-6f;
   c->eps_h = 1e-12f;
+  c->select_mode = STARKV_SELECT_GLOBAL;
 }
 
 starkv_status starkv_init_state(const starkv_config* cfg, starkv_state** out, void* stream) {
@@ -627,7 +653,8 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
     cur += align256(bytes);
     return p;
   };
-  struct Rows { size_t kv_layer, q_layer, meta_layer, out_layer, lp; bool v_in_place; };
+  struct Rows { size_t kv_layer, q_layer, meta_layer, out_layer, sel_layer, meta_out_layer, lp; bool v_in_place; };
+  const size_t P = sel_rows(c);
   std::vector<starkv_seq> dev(seqs, seqs + nseq);
   std::vector<Rows> rows(nseq);
   for (int i = 0; i < nseq; ++i) {
@@ -639,7 +666,9 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
     r.meta_layer = static_cast<size_t>(h.meta_layer_stride) * 4;
     r.lp = static_cast<size_t>(h.L - c.window);
     r.out_layer = static_cast<size_t>(h.budget + c.window);
-    const size_t mb = (h.meta_layer_stride ? static_cast<size_t>(NL) * h.meta_layer_stride : h.L) * 4;
+    r.sel_layer = P * h.budget;
+    r.meta_out_layer = P * r.out_layer;
+    const size_t mb = meta_elems(c, h, NL) * 4;
     d.k = take(NL * r.kv_layer);
     // V is read only at the kept rows: from page-locked host memory the gather
     // reads them in place instead of uploading all of V
@@ -652,11 +681,11 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
     d.meta = reinterpret_cast<const uint32_t*>(take(mb));
     d.k_out = take(NL * static_cast<size_t>(G) * r.out_layer * kHeadDim * 2);
     d.v_out = take(NL * static_cast<size_t>(G) * r.out_layer * kHeadDim * 2);
-    d.meta_out = reinterpret_cast<uint32_t*>(take(NL * r.out_layer * 4));
-    d.idx = reinterpret_cast<int32_t*>(take(NL * static_cast<size_t>(h.budget) * 4));
+    d.meta_out = reinterpret_cast<uint32_t*>(take(NL * r.meta_out_layer * 4));
+    d.idx = reinterpret_cast<int32_t*>(take(NL * r.sel_layer * 4));
     d.S = h.S ? reinterpret_cast<float*>(take(NL * static_cast<size_t>(G) * r.lp * 4)) : nullptr;
-    d.score = h.score ? reinterpret_cast<float*>(take(NL * r.lp * 4)) : nullptr;
-    d.stats = h.stats ? reinterpret_cast<float*>(take(static_cast<size_t>(NL) * (8 + 4 * G) * 4)) : nullptr;
+    d.score = h.score ? reinterpret_cast<float*>(take(NL * P * r.lp * 4)) : nullptr;
+    d.stats = h.stats ? reinterpret_cast<float*>(take(static_cast<size_t>(NL) * stats_bytes(c))) : nullptr;
   }
   const size_t used = static_cast<size_t>(cur - static_cast<char*>(workspace));
   // the uploads may start once earlier work on the caller's stream (which may
@@ -681,7 +710,7 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
       if (!r.v_in_place) CUDA_TRY(h2d(d.v, h.v, l0 * r.kv_layer, nl * r.kv_layer));
       CUDA_TRY(h2d(d.q, h.q, l0 * r.q_layer, nl * r.q_layer));
       if (h.meta_layer_stride) CUDA_TRY(h2d(d.meta, h.meta, l0 * r.meta_layer, nl * r.meta_layer));
-      else if (k == 0) CUDA_TRY(h2d(d.meta, h.meta, 0, static_cast<size_t>(h.L) * 4));
+      else if (k == 0) CUDA_TRY(h2d(d.meta, h.meta, 0, meta_elems(c, h, NL) * 4));
     }
     CUDA_TRY(cudaEventRecord(ev[2 + 2 * k], st->pipe_in));
     CUDA_TRY(cudaStreamWaitEvent(cs, ev[2 + 2 * k], 0));
@@ -697,13 +726,12 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
       const size_t kvo = static_cast<size_t>(G) * r.out_layer * kHeadDim * 2;
       CUDA_TRY(d2h(h.k_out, d.k_out, l0 * kvo, nl * kvo));
       CUDA_TRY(d2h(h.v_out, d.v_out, l0 * kvo, nl * kvo));
-      CUDA_TRY(d2h(h.meta_out, d.meta_out, l0 * r.out_layer * 4, nl * r.out_layer * 4));
-      if (h.budget > 0)
-        CUDA_TRY(d2h(h.idx, d.idx, l0 * static_cast<size_t>(h.budget) * 4, nl * static_cast<size_t>(h.budget) * 4));
+      CUDA_TRY(d2h(h.meta_out, d.meta_out, l0 * r.meta_out_layer * 4, nl * r.meta_out_layer * 4));
+      if (h.budget > 0) CUDA_TRY(d2h(h.idx, d.idx, l0 * r.sel_layer * 4, nl * r.sel_layer * 4));
       if (h.S && r.lp > 0) CUDA_TRY(d2h(h.S, d.S, l0 * G * r.lp * 4, nl * G * r.lp * 4));
-      if (h.score && r.lp > 0) CUDA_TRY(d2h(h.score, d.score, l0 * r.lp * 4, nl * r.lp * 4));
+      if (h.score && r.lp > 0) CUDA_TRY(d2h(h.score, d.score, l0 * P * r.lp * 4, nl * P * r.lp * 4));
       if (h.stats) {
-        const size_t sb = static_cast<size_t>(8 + 4 * G) * 4;
+        const size_t sb = stats_bytes(c);
         CUDA_TRY(d2h(h.stats, d.stats, l0 * sb, nl * sb));
       }
     }

@@ -45,6 +45,7 @@ struct DevState {
 struct KParams {
   int n_layers, H, G, w, R, C, pool, K, M, n_warmup, n_ramp;
   float lambda, tau, rho_mi, rho_t, delta, d_min, t_min, t_max, eps, eps_h;
+  int per_head;        // selection mode: 0 = one global top-B per layer, 1 = one per KV group
   uint64_t wait_ns;    // bounded-wait limit
 };
 
@@ -54,14 +55,15 @@ struct SeqView {
   const __nv_bfloat16* v;
   const uint32_t* meta;
   int64_t meta_layer_stride;
+  int64_t meta_group_stride;   // 0: one row shared by the groups
   int L, Lp, cur_frame, budget, slot, pad_;
   __nv_bfloat16* k_out;
   __nv_bfloat16* v_out;
   uint32_t* meta_out;
-  int32_t* idx;
+  int32_t* idx;    // [n_layers][P][B]
   float* S;        // [n_layers][G][Lp] (a workspace region when the caller passed NULL)
   float* s_raw;    // [n_layers_in_launch][G][kRawCopies][Lp] unpooled sums (workspace) or NULL
-  float* score;    // [n_layers][Lp] fused score (a workspace region when NULL)
+  float* score;    // [n_layers][P][Lp] fused score, P = 1 or G (a workspace region when NULL)
   float* stats;    // optional
   uint32_t* vis;   // [n_layers_in_launch][G][3 Lp] keys, candidate list and cells of
                    // rows too long for shared memory (workspace), else NULL

@@ -4,7 +4,8 @@
 // rows of one (tensor, group): lane i resolves the source row of output row
 // i, the source rows are broadcast by shuffle, and every instruction moves
 // two 256-byte rows (d = 128 bf16) as one 16-byte access per lane, with eight
-// such accesses per lane in flight.
+// such accesses per lane in flight.  In the per-KV-head selection mode group g
+// gathers its own index row I_g and writes its own metadata row.
 #include "common.cuh"
 #include "ptx.cuh"
 #include "compact.cuh"
@@ -37,7 +38,7 @@ __device__ __forceinline__ void st_stream(uint4* p, const uint4& v) {
 // grid: (blocks, nlayers, nseq).  Tasks of one (seq, layer): 2 tensors x G x
 // ceil((B + w) / 32) row blocks, one per warp, strided over the grid.
 __global__ void __launch_bounds__(kCompactThreads) k_compact(const __grid_constant__ SeqBatch b, int G, int w,
-                                                              uint32_t* err) {
+                                                              int per_head, uint32_t* err) {
   griddep_launch_dependents();
   griddep_wait();   // idx comes from the previous kernel
   const SeqView& sv = b.s[blockIdx.z];
@@ -45,25 +46,27 @@ __global__ void __launch_bounds__(kCompactThreads) k_compact(const __grid_consta
   const int B = sv.budget, Lp = sv.Lp, L = sv.L;
   const int rows_out = B + w;
   const int lane = threadIdx.x & 31, half = lane >> 4, hl = lane & 15;
-  const int32_t* idx = sv.idx + static_cast<int64_t>(layer) * B;
-  const uint32_t* meta = sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride;
-  uint32_t* meta_out = sv.meta_out + static_cast<int64_t>(layer) * rows_out;
+  const int P = per_head ? G : 1;   // index / metadata rows per layer
+  const int32_t* idx_l = sv.idx + static_cast<int64_t>(layer) * P * B;
+  const uint32_t* meta_l = sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride;
+  uint32_t* meta_out_l = sv.meta_out + static_cast<int64_t>(layer) * P * rows_out;
   const int nblk = ceil_div(rows_out, kTaskRows);
   const int ntask = 2 * G * nblk;
   for (int task = blockIdx.x * kWarps + (threadIdx.x >> 5); task < ntask; task += gridDim.x * kWarps) {
     const int tensor = task / (G * nblk);
     const int rem = task - tensor * G * nblk;
     const int g = rem / nblk, r0 = (rem - g * nblk) * kTaskRows;
+    const int p = per_head ? g : 0;
     // source row of output row r0 + lane
     const int r = r0 + lane;
     int src = 0;
     if (r < rows_out) {
-      src = r < B ? idx[r] : Lp + (r - B);
+      src = r < B ? idx_l[static_cast<int64_t>(p) * B + r] : Lp + (r - B);
       if (src < 0 || src >= L) {   // an index outside the cache: report, copy row 0
         atomicOr(err, kErrIndex);
         src = 0;
       }
-      if (tensor == 0 && g == 0) meta_out[r] = meta[src];
+      if (tensor == 0 && g == p) meta_out_l[static_cast<int64_t>(p) * rows_out + r] = meta_l[p * sv.meta_group_stride + src];
     }
     const __nv_bfloat16* in = (tensor == 0 ? sv.k : sv.v) + (static_cast<int64_t>(layer) * G + g) * L * kHeadDim;
     __nv_bfloat16* out = (tensor == 0 ? sv.k_out : sv.v_out) + (static_cast<int64_t>(layer) * G + g) * rows_out * kHeadDim;
@@ -88,9 +91,8 @@ __global__ void __launch_bounds__(kCompactThreads) k_compact(const __grid_consta
   }
 }
 
-cudaError_t compact_launch(const SeqBatch& b, int G, int w, int rows_out_max, int num_sms, uint32_t* err,
+cudaError_t compact_launch(const SeqBatch& b, int G, int w, int per_head, int rows_out_max, uint32_t* err,
                            cudaStream_t stream) {
-  (void)num_sms;
   if (rows_out_max <= 0) return cudaSuccess;
   const int ntask = 2 * G * ceil_div(rows_out_max, kTaskRows);
   cudaLaunchConfig_t cfg = {};
@@ -102,7 +104,7 @@ cudaError_t compact_launch(const SeqBatch& b, int G, int w, int rows_out_max, in
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, k_compact, b, G, w, err);
+  return cudaLaunchKernelEx(&cfg, k_compact, b, G, w, per_head, err);
 }
 
 }  // namespace starkv

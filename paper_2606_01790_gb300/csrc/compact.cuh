@@ -5,7 +5,8 @@
 
 namespace starkv {
 
-cudaError_t compact_launch(const SeqBatch& b, int G, int w, int rows_out_max, int num_sms, uint32_t* err,
+// per_head: idx and meta_out hold one row per KV group ([G][B], [G][B + w]).
+cudaError_t compact_launch(const SeqBatch& b, int G, int w, int per_head, int rows_out_max, uint32_t* err,
                            cudaStream_t stream);
 
 }  // namespace starkv

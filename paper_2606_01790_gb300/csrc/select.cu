@@ -16,6 +16,9 @@
 //   global top-B with ties to the lower index (Sec. 3.7): one radix select
 //     whose digit histograms are summed over the cluster, then an ordered
 //     compaction whose offsets come from the lower-ranked CTAs.
+// Per-KV-head selection mode: in phase 2 CTA g works on its own row instead,
+//   s_{g,t} = max(S[g,t] beta_g D_{g,t}, 0)^(1/T_g) with phi_g and the entropy of
+//   S[g, .], and the same radix select over that row alone.
 #include <algorithm>
 
 #include "common.cuh"
@@ -292,7 +295,8 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   const int ll = blockIdx.y, layer = b.layer0 + ll;
   const int Lp = sv.Lp;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const uint32_t* meta = sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride;
+  // this group's metadata row (the one shared row when meta_group_stride is 0)
+  const uint32_t* meta = sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride + g * sv.meta_group_stride;
   const int sl = sv.slot * kp.n_layers + layer;
   float* S = sv.S + (static_cast<int64_t>(layer) * G + g) * Lp;
   const bool in_smem = Lp <= capl;
@@ -581,7 +585,8 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   cluster_sync();   // every group's S row, MI_g and phi_g are complete
 
   // ================= phase 2: tokens [ta, tb) =================
-  float* stats = sv.stats ? sv.stats + static_cast<int64_t>(layer) * (8 + 4 * G) : nullptr;
+  float* stats = sv.stats ? sv.stats + static_cast<int64_t>(layer) * (8 + 6 * G) : nullptr;
+  const bool per_head = kp.per_head != 0;
   // ---- Eqs. (6)-(7): MI EMA (double state), min-max, softmax prior; lambda
   // schedule.  The same arithmetic in every CTA; CTA 0 stores the new state.
   if (tid == 0) {
@@ -631,8 +636,9 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       }
     }
   }
-  const int ta = static_cast<int>(static_cast<int64_t>(g) * Lp / G);
-  const int tb = static_cast<int>(static_cast<int64_t>(g + 1) * Lp / G);
+  // global mode: tokens [ta, tb) of the layer; per-KV-head mode: the whole row g
+  const int ta = per_head ? 0 : static_cast<int>(static_cast<int64_t>(g) * Lp / G);
+  const int tb = per_head ? Lp : static_cast<int>(static_cast<int64_t>(g + 1) * Lp / G);
   const int nr = tb - ta;
   const float* S0 = sv.S + static_cast<int64_t>(layer) * G * Lp;
   const float invG = 1.f / static_cast<float>(G);
@@ -643,7 +649,36 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   float* sbar_s = reinterpret_cast<float*>(cand);   // [nr]
   float z = 0.f, zl = 0.f;
   int nvr = 0;
-  for (int i0 = 0; i0 < nr; i0 += 2 * kCalThreads) {
+  if (per_head) {
+    // the ranked row is S[g, .] itself; its "governing group" is g
+    const float* Sg = S0 + static_cast<int64_t>(g) * Lp;
+    for (int i0 = 0; i0 < nr; i0 += 4 * kCalThreads) {
+      float v[4];
+      uint32_t mw[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int i = i0 + k * kCalThreads + tid;
+        v[k] = 0.f;
+        mw[k] = 0u;
+        if (i < nr) {
+          v[k] = Sg[i];
+          mw[k] = meta[i];
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int i = i0 + k * kCalThreads + tid;
+        if (i >= nr) continue;
+        z += v[k];
+        if (v[k] > 0.f) zl += v[k] * logf(v[k]);
+        nvr += meta_visual(mw[k]);
+        sbar_s[i] = v[k];
+        keys[i] = mw[k];
+        cells[i] = static_cast<uint16_t>(g);
+      }
+    }
+  }
+  for (int i0 = 0; i0 < (per_head ? 0 : nr); i0 += 2 * kCalThreads) {
     float v[2][kMaxGroups];
     uint32_t mw[2];
 #pragma unroll
@@ -694,28 +729,59 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     sh.vpart = nvr;
   }
   cluster_sync();
-  float Z = 0.f, ZL = 0.f;
-  int nvis = 0;
-  for (int r = 0; r < G; ++r) {
-    Z += dsmem_ld_f32(dsmem_map(&sh.zpart, r));
-    ZL += dsmem_ld_f32(dsmem_map(&sh.hpart, r));
-    nvis += dsmem_ld_s32(dsmem_map(&sh.vpart, r));
+  auto entropy = [&](float Zr, float ZLr) {
+    const float Ze = Zr + kp.eps_h;
+    const float plogp = Zr > 0.f ? ZLr / Ze - (Zr / Ze) * logf(Ze) : 0.f;
+    return Lp > 1 ? -plogp / logf(static_cast<float>(Lp)) : 0.f;
+  };
+  float Hn, T;
+  if (per_head) {
+    Hn = entropy(z, zl);   // this CTA's own row
+    T = kp.t_min + (kp.t_max - kp.t_min) * Hn;
+    if (tid == 0 && g == 0 && stats) {
+      float hs = 0.f, ts = 0.f, zs = 0.f;
+      for (int r = 0; r < G; ++r) {
+        const float Zr = dsmem_ld_f32(dsmem_map(&sh.zpart, r));
+        const float Hr = entropy(Zr, dsmem_ld_f32(dsmem_map(&sh.hpart, r)));
+        const float Tr = kp.t_min + (kp.t_max - kp.t_min) * Hr;
+        stats[8 + 4 * G + r] = Hr;
+        stats[8 + 5 * G + r] = Tr;
+        hs += Hr;
+        ts += Tr;
+        zs += Zr;
+      }
+      stats[0] = hs * invG;
+      stats[1] = ts * invG;
+      stats[4] = zs * invG;   // sum_t s_bar_t = mean over g of the row sums
+      stats[5] = static_cast<float>(nvr);
+    }
+  } else {
+    float Z = 0.f, ZL = 0.f;
+    int nvis = 0;
+    for (int r = 0; r < G; ++r) {
+      Z += dsmem_ld_f32(dsmem_map(&sh.zpart, r));
+      ZL += dsmem_ld_f32(dsmem_map(&sh.hpart, r));
+      nvis += dsmem_ld_s32(dsmem_map(&sh.vpart, r));
+    }
+    Hn = entropy(Z, ZL);
+    T = kp.t_min + (kp.t_max - kp.t_min) * Hn;
+    if (tid == 0 && g == 0 && stats) {
+      stats[0] = Hn;
+      stats[1] = T;
+      stats[4] = Z;
+      stats[5] = static_cast<float>(nvis);
+      for (int r = 0; r < G; ++r) {
+        stats[8 + 4 * G + r] = Hn;
+        stats[8 + 5 * G + r] = T;
+      }
+    }
   }
-  const float Ze = Z + kp.eps_h;
-  const float plogp = Z > 0.f ? ZL / Ze - (Z / Ze) * logf(Ze) : 0.f;
-  const float Hn = Lp > 1 ? -plogp / logf(static_cast<float>(Lp)) : 0.f;
-  const float T = kp.t_min + (kp.t_max - kp.t_min) * Hn;
   const float invT = 1.f / T;
-  if (tid == 0 && g == 0 && stats) {
-    stats[0] = Hn;
-    stats[1] = T;
-    stats[4] = Z;
-    stats[5] = static_cast<float>(nvis);
-  }
   // ---- Eq. (final_score) with Eq. (9): fused score, its descending key and
   // the first digit of the top-B select
   const float lam = sh.lam;
-  float* score = sv.score + static_cast<int64_t>(layer) * Lp;
+  float* score = per_head ? sv.score + (static_cast<int64_t>(layer) * G + g) * Lp
+                          : sv.score + static_cast<int64_t>(layer) * Lp + ta;
   for (int i = tid; i < nr; i += kCalThreads) {
     const float sb = sbar_s[i];
     const int gs = cells[i];
@@ -727,20 +793,22 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       d = kp.d_min + (1.f - kp.d_min) * expf(-kp.delta * df * sh.ph[gs]);
     }
     const float s = powf(fmaxf(sb * beta * d, 0.f), invT);
-    score[ta + i] = s;
+    score[i] = s;
     const uint32_t key = ~order_key(s);   // descending score = ascending key
     keys[i] = key;
     atomicAdd(&hist[key >> 20], 1);
   }
 
-  // ---- Sec. 3.7: global top-B, ties to the lower index
+  // ---- Sec. 3.7: global top-B, ties to the lower index (per-KV-head mode:
+  // the histograms and offsets of this CTA's row alone)
   const int B = sv.budget;   // the same in every CTA of the cluster
+  const int r_lo = per_head ? g : 0, r_hi = per_head ? g + 1 : G;
   if (B > 0) {
     cluster_sync();
     // digit 1 over the cluster: 4 bins per thread
     {
       int4 h = make_int4(0, 0, 0, 0);
-      for (int r = 0; r < G; ++r) {
+      for (int r = r_lo; r < r_hi; ++r) {
         const int4 q = dsmem_ld_v4(dsmem_map(hist + 4 * tid, r));
         h.x += q.x;
         h.y += q.y;
@@ -775,7 +843,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       }
       cluster_sync();
       int v = 0;
-      for (int r = 0; r < G; ++r) v += dsmem_ld_s32(dsmem_map(hp + tid, r));
+      for (int r = r_lo; r < r_hi; ++r) v += dsmem_ld_s32(dsmem_map(hp + tid, r));
       const int excl = block_excl_scan(v, sh.scan, nullptr);
       if (rk >= excl && rk < excl + v) {
         sh.tprefix = P | (static_cast<uint32_t>(tid) << shift);
@@ -803,11 +871,11 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       sh.neq = tot_eq;
     }
     cluster_sync();
-    for (int r = 0; r < g; ++r) {
+    for (int r = r_lo; r < g; ++r) {
       lt_b += dsmem_ld_s32(dsmem_map(&sh.nlt, r));
       eq_b += dsmem_ld_s32(dsmem_map(&sh.neq, r));
     }
-    int32_t* idx = sv.idx + static_cast<int64_t>(layer) * B;
+    int32_t* idx = sv.idx + (static_cast<int64_t>(layer) * (per_head ? G : 1) + (per_head ? g : 0)) * B;
     for (int i = i0; i < i1; ++i) {
       const uint32_t u = keys[i];
       int pos = -1;

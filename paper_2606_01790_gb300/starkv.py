@@ -31,6 +31,9 @@ ABI_FUNCTIONS = [
 KERNELS = ["score_lse", "score_accum", "pool", "calibrate", "compact"]
 
 
+SELECT_GLOBAL, SELECT_PER_HEAD = 0, 1   # starkv_config.select_mode
+
+
 class StarkvError(RuntimeError):
     def __init__(self, status: int, msg: str):
         super().__init__(f"starkv status {status}: {msg}")
@@ -42,7 +45,8 @@ class CConfig(C.Structure):
         "n_layers", "n_heads", "n_kv_heads", "head_dim", "window", "grid_rows", "grid_cols",
         "pool_kernel", "mi_bins", "mi_grid", "n_warmup", "n_ramp", "max_seqs")] + \
         [(n, C.c_float) for n in (
-            "lambda_", "tau", "rho_mi", "rho_t", "delta", "d_min", "t_min", "t_max", "eps", "eps_h")]
+            "lambda_", "tau", "rho_mi", "rho_t", "delta", "d_min", "t_min", "t_max", "eps", "eps_h")] + \
+        [("select_mode", C.c_int32)]
 
 
 class CSeq(C.Structure):
@@ -50,7 +54,8 @@ class CSeq(C.Structure):
                 ("meta_layer_stride", C.c_int64), ("L", C.c_int32), ("cur_frame", C.c_int32),
                 ("budget", C.c_int32), ("slot", C.c_int32), ("k_out", C.c_void_p),
                 ("v_out", C.c_void_p), ("meta_out", C.c_void_p), ("idx", C.c_void_p),
-                ("S", C.c_void_p), ("score", C.c_void_p), ("stats", C.c_void_p)]
+                ("S", C.c_void_p), ("score", C.c_void_p), ("stats", C.c_void_p),
+                ("meta_group_stride", C.c_int64)]
 
 
 _lib: Optional[C.CDLL] = None
@@ -124,6 +129,7 @@ class Config:
     t_max: float = 1.05
     eps: float = 1e-6
     eps_h: float = 1e-12
+    select_mode: int = 0    # SELECT_GLOBAL (the paper's) or SELECT_PER_HEAD
 
     def to_c(self) -> CConfig:
         c = CConfig()
@@ -140,7 +146,12 @@ class Config:
 
 def stats_stride(n_kv_heads: int) -> int:
     """Floats per layer in a stats buffer (``STARKV_STATS_STRIDE``)."""
-    return 8 + 4 * n_kv_heads
+    return 8 + 6 * n_kv_heads
+
+
+def sel_rows(cfg: "Config") -> int:
+    """Rows of idx / score / meta_out per layer: 1 (global selection) or G (per KV head)."""
+    return cfg.n_kv_heads if cfg.select_mode == SELECT_PER_HEAD else 1
 
 
 def pack_meta(is_visual, frame, row, col) -> np.ndarray:
@@ -194,12 +205,14 @@ class Seq:
     S: Optional[torch.Tensor] = None
     score: Optional[torch.Tensor] = None
     stats: Optional[torch.Tensor] = None
+    meta_group_stride: int = 0              # per-KV-head mode: one metadata row per group
 
     def to_c(self) -> CSeq:
         s = CSeq()
         for name in ("k", "v", "q", "meta", "k_out", "v_out", "meta_out", "idx", "S", "score", "stats"):
             setattr(s, name, _ptr(getattr(self, name)))
         s.meta_layer_stride = self.meta_layer_stride
+        s.meta_group_stride = self.meta_group_stride
         s.L, s.cur_frame, s.budget, s.slot = self.L, self.cur_frame, self.budget, self.slot
         return s
 

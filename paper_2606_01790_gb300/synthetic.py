@@ -230,7 +230,9 @@ class SeqInput:
     q: torch.Tensor            # bf16 [n_layers][H][w][d]
     k: torch.Tensor            # bf16 [n_layers][G][L][d]
     v: torch.Tensor            # bf16 [n_layers][G][L][d]
-    layout: List[TokenLayout]  # per layer (identical for a fresh sequence)
+    layout: list               # per layer: a TokenLayout (identical for a fresh
+                               # sequence), or G of them, one per KV group, after
+                               # a per-KV-head compaction
     cur_frame: int
     budget: int
     n_visual_history: int
@@ -324,10 +326,12 @@ def append_step(wl: Workload, prev_k: torch.Tensor, prev_v: torch.Tensor,
     """Trajectory step ``step`` >= 1: append one screenshot (frame = previous
     newest frame + 1) and ``wl.step_text`` text tokens to each layer's compressed
     cache ``prev_k``/``prev_v`` ([n_layers][G][B+w][d]) and draw fresh window
-    queries.  Bump centres drift by one random patch per step."""
+    queries.  Bump centres drift by one random patch per step.  A layer whose
+    ``prev_layout`` is a list of per-group layouts keeps one per group."""
     layers = list(range(wl.n_layers)) if layers is None else list(layers)
+    flat = [x for lay in prev_layout for x in (lay if isinstance(lay, list) else [lay])]
     newest = max(int(lay.frame[lay.is_visual.astype(bool)].max()) if lay.is_visual.any() else -1
-                 for lay in prev_layout)
+                 for lay in flat)
     frame = newest + 1
     R, C = wl.grid_rows, wl.grid_cols
     j = np.arange(R * C, dtype=np.int32)
@@ -344,10 +348,14 @@ def append_step(wl: Workload, prev_k: torch.Tensor, prev_v: torch.Tensor,
         qs.append(q)
         ks.append(torch.cat([prev_k[i], to_bf16(k_new)], dim=1))
         vs.append(torch.cat([prev_v[i], to_bf16(v_new)], dim=1))
-        lays.append(TokenLayout.concat([prev_layout[i], new_lay]))
+        prev = prev_layout[i]
+        if isinstance(prev, list):
+            lays.append([TokenLayout.concat([pg, new_lay]) for pg in prev])
+        else:
+            lays.append(TokenLayout.concat([prev, new_lay]))
     n_vis = n_visual_history + R * C
     pct = wl.budget_pct if budget_pct is None else budget_pct
-    l_past = lays[0].L - wl.window
+    l_past = ks[0].shape[1] - wl.window
     return SeqInput(q=to_bf16(np.stack(qs)), k=torch.stack(ks), v=torch.stack(vs), layout=lays,
                     cur_frame=frame, budget=budget(pct, n_vis, l_past), n_visual_history=n_vis)
 

@@ -32,14 +32,16 @@ def oracle_params(h: Dict) -> O.Params:
     return O.Params(**h)
 
 
-def gpu_config(wl: syn.Workload, h: Dict, n_layers: Optional[int] = None, max_seqs: int = 1) -> sk.Config:
+def gpu_config(wl: syn.Workload, h: Dict, n_layers: Optional[int] = None, max_seqs: int = 1,
+               per_head: bool = False) -> sk.Config:
     return sk.Config(n_layers=n_layers or wl.n_layers, n_heads=wl.n_heads, n_kv_heads=wl.n_kv_heads,
                      head_dim=wl.head_dim, window=wl.window, grid_rows=wl.grid_rows,
                      grid_cols=wl.grid_cols, pool_kernel=h["pool_kernel"], mi_bins=h["mi_bins"],
                      mi_grid=h["mi_grid"], n_warmup=h["n_warmup"], n_ramp=h["n_ramp"],
                      max_seqs=max_seqs, lambda_=h["lam"], tau=h["tau"], rho_mi=h["rho_mi"],
                      rho_t=h["rho_t"], delta=h["delta"], d_min=h["d_min"], t_min=h["t_min"],
-                     t_max=h["t_max"], eps=h["eps"], eps_h=h["eps_h"])
+                     t_max=h["t_max"], eps=h["eps"], eps_h=h["eps_h"],
+                     select_mode=sk.SELECT_PER_HEAD if per_head else sk.SELECT_GLOBAL)
 
 
 @dataclass
@@ -48,28 +50,53 @@ class DevSeq:
     si: syn.SeqInput
 
 
+def _words(lay) -> np.ndarray:
+    """Metadata words of one layer: [L], or [G][L] for per-group layouts."""
+    if isinstance(lay, list):
+        return np.stack([_words(x) for x in lay])
+    return sk.pack_meta(lay.is_visual, lay.frame, lay.row, lay.col)
+
+
+def layer_meta(lay, field: str) -> np.ndarray:
+    """One metadata field of a layer: [L] or [G][L]."""
+    if isinstance(lay, list):
+        return np.stack([getattr(x, field) for x in lay])
+    return getattr(lay, field)
+
+
 def device_seq(si: syn.SeqInput, wl: syn.Workload, slot: int = 0, dev="cuda",
-               with_S: bool = True, with_score: bool = True, with_stats: bool = True) -> DevSeq:
+               with_S: bool = True, with_score: bool = True, with_stats: bool = True,
+               per_head: bool = False) -> DevSeq:
+    """Device buffers of one sequence; per_head sizes idx / score / meta_out with
+    one row per KV group.  Per-group layouts give [n_layers][G][L] metadata."""
     nl, G, w, d = si.k.shape[0], wl.n_kv_heads, wl.window, wl.head_dim
     L, B = si.L, si.budget
     lp = L - w
-    words = np.stack([sk.pack_meta(l.is_visual, l.frame, l.row, l.col) for l in si.layout])
+    P = G if per_head else 1
+    words = np.stack([_words(l) for l in si.layout])
+    grouped = words.ndim == 3
+    if grouped and not per_head:
+        raise ValueError("per-group metadata needs the per-KV-head mode")
     seq = sk.Seq(k=si.k.to(dev), v=si.v.to(dev), q=si.q.to(dev),
-                 meta=sk.meta_tensor(words).to(dev), meta_layer_stride=L, L=L,
+                 meta=sk.meta_tensor(words).to(dev), meta_layer_stride=(G * L if grouped else L),
+                 meta_group_stride=(L if grouped else 0), L=L,
                  cur_frame=si.cur_frame, budget=B, slot=slot,
                  k_out=torch.empty((nl, G, B + w, d), dtype=torch.bfloat16, device=dev),
                  v_out=torch.empty((nl, G, B + w, d), dtype=torch.bfloat16, device=dev),
-                 meta_out=torch.empty((nl, B + w), dtype=torch.int32, device=dev),
-                 idx=torch.empty((nl, max(B, 0)), dtype=torch.int32, device=dev),
+                 meta_out=torch.empty((nl, P, B + w) if per_head else (nl, B + w), dtype=torch.int32,
+                                      device=dev),
+                 idx=torch.empty((nl, P, max(B, 0)) if per_head else (nl, max(B, 0)), dtype=torch.int32,
+                                 device=dev),
                  S=torch.empty((nl, G, lp), dtype=torch.float32, device=dev) if with_S else None,
-                 score=torch.empty((nl, lp), dtype=torch.float32, device=dev) if with_score else None,
+                 score=torch.empty((nl, P, lp) if per_head else (nl, lp), dtype=torch.float32, device=dev)
+                 if with_score else None,
                  stats=torch.empty((nl, sk.stats_stride(G)), dtype=torch.float32, device=dev)
                  if with_stats else None)
     return DevSeq(seq, si)
 
 
 def oracle_layer(si: syn.SeqInput, layer: int, wl: syn.Workload, st: O.LayerState, p: O.Params,
-                 S_override: Optional[np.ndarray] = None) -> Dict:
+                 S_override: Optional[np.ndarray] = None, per_head: bool = False) -> Dict:
     """Algorithm 1 for one layer of one sequence; ``S_override`` skips scoring
     and feeds the given group score map to the calibration/selection steps."""
     lay = si.layout[layer]
@@ -78,8 +105,9 @@ def oracle_layer(si: syn.SeqInput, layer: int, wl: syn.Workload, st: O.LayerStat
         S = O.score_layer(si.q[layer].double().numpy(), si.k[layer].double().numpy(), wl.window, p)
     else:
         S = S_override
-    out = O.select_layer(S, lay.is_visual, lay.frame, lay.row, lay.col, si.cur_frame, si.budget,
-                         wl.grid_rows, wl.grid_cols, st, p)
+    meta = tuple(layer_meta(lay, f) for f in ("is_visual", "frame", "row", "col"))
+    sel = O.select_layer_per_head if per_head else O.select_layer
+    out = sel(S, *meta, si.cur_frame, si.budget, wl.grid_rows, wl.grid_cols, st, p)
     out["S"] = S
     out["lp"] = lp
     return out
@@ -151,3 +179,33 @@ def check_compaction(seq: sk.Seq, si: syn.SeqInput, layer: int, w: int) -> None:
     words = sk.pack_meta(lay.is_visual, lay.frame, lay.row, lay.col)[rows.numpy()]
     got = seq.meta_out[layer].cpu().numpy().view(np.uint32)
     assert np.array_equal(got, words), "meta' is not a bit copy"
+
+
+def check_per_head(seq: sk.Seq, si: syn.SeqInput, layer: int, wl: syn.Workload, ref: Dict,
+                   rtol: float = RTOL) -> Dict:
+    """Per-KV-head mode: each group's fused scores within ``rtol`` relative, its
+    index set equal except ties inside that band, and K', V', meta' of group g
+    bit copies of the rows its own index set names."""
+    G, w, B = wl.n_kv_heads, wl.window, si.budget
+    lp = si.L - w
+    out = dict(max_rel=0.0, n_diff=0)
+    words = _words(si.layout[layer])
+    if words.ndim == 1:
+        words = np.tile(words, (G, 1))
+    score = seq.score[layer].double().cpu().numpy() if seq.score is not None else None
+    for g in range(G):
+        if score is not None:
+            ok = score_tolerance_ok(score[g], ref["score"][g], rtol)
+            assert ok.all(), (layer, g, np.nonzero(~ok)[0][:10])
+            rel = np.abs(score[g] - ref["score"][g]) / np.maximum(np.abs(ref["score"][g]), 1e-30)
+            out["max_rel"] = max(out["max_rel"], float(rel.max()) if rel.size else 0.0)
+        gi = seq.idx[layer][g].cpu().numpy()
+        ix = check_index_set(gi, dict(idx=ref["idx"][g], score=ref["score"][g]), B, rtol)
+        assert ix["ok"], (layer, g, ix)
+        out["n_diff"] += ix["n_diff"]
+        rows = torch.cat([torch.from_numpy(gi.astype(np.int64)), torch.arange(lp, si.L)])
+        assert torch.equal(seq.k_out[layer][g].cpu(), si.k[layer][g].index_select(0, rows)), "K' group copy"
+        assert torch.equal(seq.v_out[layer][g].cpu(), si.v[layer][g].index_select(0, rows)), "V' group copy"
+        got = seq.meta_out[layer][g].cpu().numpy().view(np.uint32)
+        assert np.array_equal(got, words[g][rows.numpy()]), "meta' group copy"
+    return out

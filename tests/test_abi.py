@@ -39,8 +39,18 @@ def test_library_exports_every_declared_symbol(library):
 
 
 def test_struct_layouts_match_header():
-    assert ctypes.sizeof(sk.CConfig) == 13 * 4 + 10 * 4
-    assert ctypes.sizeof(sk.CSeq) == 4 * 8 + 8 + 4 * 4 + 7 * 8
+    assert ctypes.sizeof(sk.CConfig) == 13 * 4 + 10 * 4 + 4
+    assert [f[0] for f in sk.CConfig._fields_][-1] == "select_mode"
+
+
+def test_header_constants_match_binding():
+    import re
+    text = (ROOT / "include" / "starkv.h").read_text()
+    m = re.search(r"#define STARKV_STATS_STRIDE\(G\) \(8 \+ (\d+) \* \(G\)\)", text)
+    assert m and all(sk.stats_stride(g) == 8 + int(m.group(1)) * g for g in range(1, 9))
+    m = re.search(r"STARKV_SELECT_GLOBAL = (\d+), STARKV_SELECT_PER_HEAD = (\d+)", text)
+    assert m and (int(m.group(1)), int(m.group(2))) == (sk.SELECT_GLOBAL, sk.SELECT_PER_HEAD)
+    assert ctypes.sizeof(sk.CSeq) == 4 * 8 + 8 + 4 * 4 + 7 * 8 + 8
 
 
 def test_default_config_matches_paper_defaults(library):
@@ -49,11 +59,12 @@ def test_default_config_matches_paper_defaults(library):
     assert abs(c.lambda_ - 0.5) < 1e-7 and abs(c.delta - 0.2) < 1e-7 and abs(c.d_min - 0.1) < 1e-7
     assert (c.n_warmup, c.n_ramp) == (5, 10)
     assert abs(c.t_min - 0.95) < 1e-7 and abs(c.t_max - 1.05) < 1e-7
+    assert c.select_mode == sk.SELECT_GLOBAL
 
 
 @pytest.mark.parametrize("bad", [dict(head_dim=64), dict(n_heads=30), dict(window=64),
                                  dict(pool_kernel=4), dict(mi_bins=1), dict(t_min=0.0),
-                                 dict(n_kv_heads=0), dict(grid_rows=2000)])
+                                 dict(n_kv_heads=0), dict(grid_rows=2000), dict(select_mode=2)])
 def test_invalid_config_rejected_before_any_device_call(library, bad):
     cfg = sk.Config(**bad)
     with pytest.raises(sk.StarkvError) as e:

@@ -98,6 +98,7 @@ def test_step_matches_oracle(name, sched):
     stats = ds.seq.stats[0].double().cpu().numpy()
     G = wl.n_kv_heads
     assert abs(stats[0] - ref["H"]) < 1e-5 and abs(stats[1] - ref["T"]) < 1e-5
+    assert np.all(stats[8 + 4 * G:8 + 5 * G] == stats[0]) and np.all(stats[8 + 5 * G:8 + 6 * G] == stats[1])
     np.testing.assert_allclose(stats[8:8 + G], ref["mi"], rtol=2e-3, atol=2e-4)
     np.testing.assert_allclose(stats[8 + 2 * G:8 + 3 * G], ref["w"], rtol=2e-3)
 
