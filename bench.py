@@ -47,20 +47,21 @@ def _peaks():
 
 # ----------------------------------------------------------------------------- work accounting
 
-def work_per_step(wl, seqs):
+def work_per_step(wl, seqs, per_head=False):
     """Algorithmic bytes and flops of one step, per kernel kind and in total.
 
     Per scored token and layer: K read once (G * d * 2 B) and 2 * H * w * d
     flop of Q K^T; per (layer, seq): window queries H * w * d * 2 B; the group
     score map written and read (2 * G * 4 B per token); per kept row: K and V
-    read and written (4 * G * d * 2 B)."""
+    read and written (4 * G * d * 2 B) and its metadata word read and written
+    (once, or once per group in the per-KV-head mode)."""
     H, G, w, d, nl = wl.n_heads, wl.n_kv_heads, wl.window, wl.head_dim, wl.n_layers
     tok = sum(s["L"] - w for s in seqs) * nl
     kept = sum(s["B"] + w for s in seqs) * nl
     qk_flops = 2.0 * H * w * d * tok
     k_bytes = G * d * 2.0 * tok + H * w * d * 2.0 * nl * len(seqs)
     s_bytes = 2 * G * 4.0 * tok
-    gather = 4.0 * G * d * 2 * kept + 2 * 4.0 * kept
+    gather = 4.0 * G * d * 2 * kept + 2 * 4.0 * kept * (G if per_head else 1)
     return dict(tokens=tok, qk_flops=qk_flops, k_bytes=k_bytes, s_bytes=s_bytes, gather_bytes=gather,
                 step_bytes=k_bytes + s_bytes + gather)
 
@@ -159,6 +160,7 @@ def oracle_worker(args):
     from paper_2606_01790_gb300 import synthetic as syn
     wl = syn.WORKLOADS[args.workload]
     p = O.Params()
+    per_head = args.select_mode == "per_head"
     spent, tokens = 0.0, 0
     per_call = []
     layers = [0] * args.repeat if args.repeat > 0 else list(range(min(wl.n_layers, args.max_layers)))
@@ -172,7 +174,7 @@ def oracle_worker(args):
         q, k, v = si.q[0].double().numpy(), si.k[0].double().numpy(), si.v[0].double().numpy()
         t = time.perf_counter()
         O.step_layer(q, k, v, lay.is_visual, lay.frame, lay.row, lay.col, si.cur_frame, si.budget,
-                     wl.window, wl.grid_rows, wl.grid_cols, st, p)
+                     wl.window, wl.grid_rows, wl.grid_cols, st, p, per_head=per_head)
         dt = time.perf_counter() - t
         per_call.append(dt)
         spent += dt
@@ -183,13 +185,13 @@ def oracle_worker(args):
                           l_past=syn.make_sequence(wl, seq=0, layers=[0]).L - wl.window)))
 
 
-def run_oracle_subprocess(workload, budget_s=15.0, max_layers=28, repeat=0):
+def run_oracle_subprocess(workload, budget_s=15.0, max_layers=28, repeat=0, select_mode="global"):
     threads = str(os.cpu_count() or 1)
     env = dict(os.environ, OPENBLAS_NUM_THREADS=threads, OMP_NUM_THREADS=threads,
                MKL_NUM_THREADS=threads, CUDA_VISIBLE_DEVICES="")
     r = subprocess.run([sys.executable, str(ROOT / "bench.py"), "--oracle-worker", "--workload", workload,
                         "--budget-s", str(budget_s), "--max-layers", str(max_layers),
-                        "--repeat", str(repeat)],
+                        "--repeat", str(repeat), "--select-mode", select_mode],
                        capture_output=True, text=True, env=env, timeout=3600)
     if r.returncode != 0:
         raise RuntimeError(f"oracle worker failed:\n{r.stderr[-2000:]}")
@@ -205,7 +207,7 @@ def reference_arm(args):
         return
     from paper_2606_01790_gb300 import synthetic as syn
     wl = syn.WORKLOADS[args.workload]
-    d = run_oracle_subprocess(args.workload, repeat=args.warmup + args.steps)
+    d = run_oracle_subprocess(args.workload, repeat=args.warmup + args.steps, select_mode=args.select_mode)
     times = d["per_call"][args.warmup:]
     total = sum(times)
     value = d["l_past"] * len(times) / total
@@ -216,7 +218,7 @@ def reference_arm(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * total / len(times), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": args.workload},
+        "config": {"workload": args.workload, "select_mode": args.select_mode},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": d["cores"], "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -273,9 +275,11 @@ def gpu_arm(args):
     sis = [syn.make_sequence(wl, seq=i, seed=s) for i, s in enumerate(seeds)]
     cfg = sk.Config(n_layers=wl.n_layers, n_heads=wl.n_heads, n_kv_heads=wl.n_kv_heads,
                     head_dim=wl.head_dim, window=wl.window, grid_rows=wl.grid_rows,
-                    grid_cols=wl.grid_cols, max_seqs=len(sis))
+                    grid_cols=wl.grid_cols, max_seqs=len(sis),
+                    select_mode=sk.SELECT_PER_HEAD if args.select_mode == "per_head" else sk.SELECT_GLOBAL)
     st = sk.init_state(cfg)
     G, w, d, nl = wl.n_kv_heads, wl.window, wl.head_dim, wl.n_layers
+    P = sk.sel_rows(cfg)   # rows of idx / meta_out per layer
 
     def make_seq(si, slot, device, pin=False):
         L, B = si.L, si.budget
@@ -292,12 +296,12 @@ def gpu_arm(args):
                       meta_layer_stride=0, L=L, cur_frame=si.cur_frame, budget=B, slot=slot,
                       k_out=alloc((nl, G, B + w, d), torch.bfloat16),
                       v_out=alloc((nl, G, B + w, d), torch.bfloat16),
-                      meta_out=alloc((nl, B + w), torch.int32), idx=alloc((nl, B), torch.int32))
+                      meta_out=alloc((nl, P, B + w), torch.int32), idx=alloc((nl, P, B), torch.int32))
 
     seqs = [make_seq(si, i, dev) for i, si in enumerate(sis)]
     ws = sk.workspace(st, seqs, device=dev)
     stream = torch.cuda.current_stream(dev)
-    work = work_per_step(wl, [dict(L=si.L, B=si.budget) for si in sis])
+    work = work_per_step(wl, [dict(L=si.L, B=si.budget) for si in sis], per_head=P > 1)
 
     def barrier():
         if dist is not None:
@@ -390,7 +394,8 @@ def gpu_arm(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        o = run_oracle_subprocess(args.workload, budget_s=args.cpu_budget_s, max_layers=wl.n_layers)
+        o = run_oracle_subprocess(args.workload, budget_s=args.cpu_budget_s, max_layers=wl.n_layers,
+                                  select_mode=args.select_mode)
         cpu = {"value": o["tokens"] / o["seconds"], "unit": UNIT, "cores": o["cores"], "kind": "oracle",
                "sample": f"{o['calls']} of {wl.n_layers} layers of sequence 0 "
                          f"({o['tokens']} tokens scored in {o['seconds']:.1f} s, "
@@ -401,7 +406,7 @@ def gpu_arm(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": args.workload, "layers": nl, "seqs_per_gpu": len(sis),
+            "config": {"workload": args.workload, "select_mode": args.select_mode, "layers": nl, "seqs_per_gpu": len(sis),
                        "L": [si.L for si in sis], "w": w, "B": [si.budget for si in sis],
                        "H": wl.n_heads, "G": G, "d": d,
                        "l2": f"inputs {2 * sum(s.k.numel() for s in seqs) * 2 / 1e9:.2f} GB per step "
@@ -423,6 +428,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["starkv", "reference"], default="starkv")
     ap.add_argument("--workload", default="uitars_5shot_28l")
+    ap.add_argument("--select-mode", choices=["global", "per_head"], default="global",
+                    help="global top-B per layer (the paper's) or one top-B per KV group")
     ap.add_argument("--soak-s", type=float, default=2.0)
     ap.add_argument("--cpu-budget-s", type=float, default=15.0)
     ap.add_argument("--no-e2e", action="store_true")
