@@ -222,6 +222,12 @@ __device__ __forceinline__ float ex2_approx(float x) {
   return y;
 }
 
+__device__ __forceinline__ float lg2_approx(float x) {
+  float y;
+  asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Named barrier over `nthreads` threads that also ORs `flag` across them.
 __device__ __forceinline__ bool named_bar_any(int id, int nthreads, bool flag) {
   uint32_t res;

@@ -36,6 +36,8 @@ constexpr int kBins1 = 1024;         // second and third digits: bits 19..10 and
 constexpr uint16_t kNoCell = 0xFFFF; // not a (valid) visual token
 constexpr unsigned kFullMask = 0xffffffffu;
 constexpr int kBruteMax = 2048;      // largest boundary bucket ranked pairwise
+constexpr int kCandMax = 2048;       // largest top-B boundary bucket ranked pairwise
+constexpr float kLn2 = 0.6931471805599453f;
 constexpr size_t kSmemMax = 227 * 1024;
 
 // Order-preserving map float -> uint32 (a < b  <=>  key(a) < key(b) for non-NaN).
@@ -160,14 +162,65 @@ struct CalShared {
   float lam;
   int n_old;
   int any_tie;
+  float fredn[4][32];             // multi-value block reductions
+  uint32_t uredn[2][32];
+  float mic[kMaxGroups];          // every group's MI_g (phase 2)
+  float pz[kMaxGroups], pzl[kMaxGroups], pv[kMaxGroups];   // every CTA's phase-2 partials
+  uint32_t pkmin[kMaxGroups], pkmax[kMaxGroups];
+  int pncand[kMaxGroups], pbelow[kMaxGroups];
   // read by the other CTAs of the cluster
   float mi, phi;                  // this CTA's group (phase 1)
-  float zpart, hpart;             // this CTA's token range (phase 2)
-  int vpart, nlt, neq;
-  // top-B radix select
-  uint32_t tprefix;
-  int trank;
+  float zpart, hpart, vpart;      // this CTA's token range (phase 2)
+  uint32_t kminp, kmaxp;
+  int tcand, nbelow;              // top-B boundary-bucket candidates, tokens below it
+  int nlt, neq;
+  // top-B select
+  int tb, tcnt;                   // boundary bucket and its token count
+  uint32_t tprefix, tkey;
+  int trank, tpos;
 };
+
+// Sums of NF floats, the minimum of `mn` and the maximum of `mx` over the
+// 1024 threads with one pair of barriers; every thread gets the results.
+template <int NF>
+__device__ void block_reduce(float (&v)[NF], uint32_t& mn, uint32_t& mx, CalShared& sh) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int k = 0; k < NF; ++k) v[k] = warp_sum(v[k]);
+  mn = __reduce_min_sync(kFullMask, mn);
+  mx = __reduce_max_sync(kFullMask, mx);
+  __syncthreads();
+  if (lane == 0) {
+#pragma unroll
+    for (int k = 0; k < NF; ++k) sh.fredn[k][warp] = v[k];
+    sh.uredn[0][warp] = mn;
+    sh.uredn[1][warp] = mx;
+  }
+  __syncthreads();
+#pragma unroll
+  for (int k = 0; k < NF; ++k) v[k] = warp_sum(sh.fredn[k][lane]);
+  mn = __reduce_min_sync(kFullMask, sh.uredn[0][lane]);
+  mx = __reduce_max_sync(kFullMask, sh.uredn[1][lane]);
+}
+
+// Sum of the int4 at `p` over the CTAs [r_lo, r_hi) of the cluster: every
+// remote load is issued before the first add.
+__device__ __forceinline__ int4 sum_peers_v4(const int* p, int r_lo, int r_hi) {
+  int4 q[kMaxGroups];
+#pragma unroll
+  for (int r = 0; r < kMaxGroups; ++r)
+    if (r < r_hi - r_lo) q[r] = dsmem_ld_v4(dsmem_map(p, r_lo + r));
+  int4 h = make_int4(0, 0, 0, 0);
+#pragma unroll
+  for (int r = 0; r < kMaxGroups; ++r)
+    if (r < r_hi - r_lo) {
+      h.x += q[r].x;
+      h.y += q[r].y;
+      h.z += q[r].z;
+      h.w += q[r].w;
+    }
+  return h;
+}
 
 constexpr size_t align16(size_t x) { return (x + 15) & ~size_t(15); }
 constexpr size_t kCalSharedBytes = align16(sizeof(CalShared));
@@ -403,9 +456,12 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     keys[t] = key;
     cells[t] = cell;
   }
-  const int N = block_sum<int>(nv, sh.ired);
-  kmin = block_min(kmin, sh.ured);
-  kmax = block_max(kmax, sh.ured);
+  int N;
+  {
+    float nvf[1] = {static_cast<float>(nv)};   // counts below 2^24: exact in fp32
+    block_reduce<1>(nvf, kmin, kmax, sh);
+    N = static_cast<int>(nvf[0]);
+  }
   // Sec. 3.4 RankBin, first digit: 4096 buckets spread linearly over the
   // row's key range (monotone in the key, so bucket order is key order)
   const float binv = 4096.f / (static_cast<float>(kmax - kmin) + 1.f);
@@ -562,9 +618,14 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     ncur = fmaf(a, a, ncur);
     nm = fmaf(bm, bm, nm);
   }
-  dot = block_sum<float>(dot, sh.fred);
-  ncur = block_sum<float>(ncur, sh.fred);
-  nm = block_sum<float>(nm, sh.fred);
+  {
+    float r3[3] = {dot, ncur, nm};
+    uint32_t u0 = 0u, u1 = 0u;
+    block_reduce<3>(r3, u0, u1, sh);
+    dot = r3[0];
+    ncur = r3[1];
+    nm = r3[2];
+  }
   float phi = 0.f;
   if (ncur > 0.f) {
     if (nm > 0.f) {
@@ -584,21 +645,26 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   for (int i = tid; i < kBins0; i += kCalThreads) hist[i] = 0;   // top-B digit 1 (below)
   cluster_sync();   // every group's S row, MI_g and phi_g are complete
 
-  // ================= phase 2: tokens [ta, tb) =================
-  float* stats = sv.stats ? sv.stats + static_cast<int64_t>(layer) * (8 + 6 * G) : nullptr;
+  // ================= phase 2 =================
+  // global mode: CTA r scores and selects tokens [r Lp / G, (r + 1) Lp / G) of
+  // s_bar; per-KV-head mode: CTA g its own row S[g, .]
   const bool per_head = kp.per_head != 0;
+  float* stats = sv.stats ? sv.stats + static_cast<int64_t>(layer) * (8 + 6 * G) : nullptr;
   // ---- Eqs. (6)-(7): MI EMA (double state), min-max, softmax prior; lambda
   // schedule.  The same arithmetic in every CTA; CTA 0 stores the new state.
+  if (tid < G) {
+    sh.mic[tid] = dsmem_ld_f32(dsmem_map(&sh.mi, tid));
+    sh.ph[tid] = dsmem_ld_f32(dsmem_map(&sh.phi, tid));
+  }
+  __syncthreads();
   if (tid == 0) {
     const int n = sh.n_old;
     double mib[kMaxGroups];
-    float mic[kMaxGroups], mf[kMaxGroups];
+    float mf[kMaxGroups];
     float lo = 3.4e38f, hi = -3.4e38f;
     for (int gg = 0; gg < G; ++gg) {
-      mic[gg] = dsmem_ld_f32(dsmem_map(&sh.mi, gg));
-      sh.ph[gg] = dsmem_ld_f32(dsmem_map(&sh.phi, gg));
-      mib[gg] = n == 0 ? static_cast<double>(mic[gg])
-                       : kp.rho_mi * sh.mib_old[gg] + (1.0 - kp.rho_mi) * static_cast<double>(mic[gg]);
+      mib[gg] = n == 0 ? static_cast<double>(sh.mic[gg])
+                       : kp.rho_mi * sh.mib_old[gg] + (1.0 - kp.rho_mi) * static_cast<double>(sh.mic[gg]);
       mf[gg] = static_cast<float>(mib[gg]);
       lo = fminf(lo, mf[gg]);
       hi = fmaxf(hi, mf[gg]);
@@ -628,7 +694,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         stats[6] = static_cast<float>(sv.budget);
         stats[7] = 0.f;
         for (int gg = 0; gg < G; ++gg) {
-          stats[8 + gg] = mic[gg];
+          stats[8 + gg] = sh.mic[gg];
           stats[8 + G + gg] = mf[gg];
           stats[8 + 2 * G + gg] = sh.w[gg];
           stats[8 + 3 * G + gg] = sh.ph[gg];
@@ -636,21 +702,40 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       }
     }
   }
-  // global mode: tokens [ta, tb) of the layer; per-KV-head mode: the whole row g
+  __syncthreads();   // w and lambda are read by every thread below
   const int ta = per_head ? 0 : static_cast<int>(static_cast<int64_t>(g) * Lp / G);
   const int tb = per_head ? Lp : static_cast<int>(static_cast<int64_t>(g + 1) * Lp / G);
   const int nr = tb - ta;
   const float* S0 = sv.S + static_cast<int64_t>(layer) * G * Lp;
   const float invG = 1.f / static_cast<float>(G);
-  // ---- Sec. 3.6 in one pass: Z = sum s_bar and sum s_bar log s_bar over the
-  // cluster, then H = -sum p log p / log L_p with p = s_bar / (Z + eps)
-  // (the eps inside the log changes H by less than L_p eps).  The pass stages
-  // s_bar, g* and the metadata word of its tokens for the fused score.
-  float* sbar_s = reinterpret_cast<float*>(cand);   // [nr]
-  float z = 0.f, zl = 0.f;
-  int nvr = 0;
+  const float lam = sh.lam;
+  // ---- one pass over the range: s_bar and g* (Eq. 4; per-KV-head mode:
+  // S[g, t] and g itself); Z = sum s and sum s log2 s (Sec. 3.6, one pass:
+  // H = -sum p log p / log L_p with p = s / (Z + eps), where the eps inside
+  // the log changes H by less than L_p eps); the untempered fused score
+  // x_t = max(s beta D, 0) (Eq. final_score with Eq. 9).  s_t = x_t^(1/T) is
+  // increasing in x_t, so the top-B select ranks the keys of x_t.
+  float* xs = reinterpret_cast<float*>(cand);   // [nr]
+  float z = 0.f, zl = 0.f, nvf = 0.f;
+  uint32_t kmn = 0xFFFFFFFFu, kmx = 0u;
+  auto fuse = [&](int i, float sb, int gs, uint32_t mt) {
+    z += sb;
+    if (sb > 0.f) zl += sb * lg2_approx(sb);
+    const float beta = (1.f - lam) + lam * static_cast<float>(G) * sh.w[gs];
+    float d = 1.f;
+    if (meta_visual(mt)) {
+      nvf += 1.f;
+      const float df = static_cast<float>(sv.cur_frame - meta_frame(mt));
+      d = kp.d_min + (1.f - kp.d_min) * expf(-kp.delta * df * sh.ph[gs]);
+    }
+    const float x = fmaxf(sb * beta * d, 0.f);
+    const uint32_t key = ~order_key(x);   // descending score = ascending key
+    xs[i] = x;
+    keys[i] = key;
+    kmn = min(kmn, key);
+    kmx = max(kmx, key);
+  };
   if (per_head) {
-    // the ranked row is S[g, .] itself; its "governing group" is g
     const float* Sg = S0 + static_cast<int64_t>(g) * Lp;
     for (int i0 = 0; i0 < nr; i0 += 4 * kCalThreads) {
       float v[4];
@@ -668,100 +753,106 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
         const int i = i0 + k * kCalThreads + tid;
-        if (i >= nr) continue;
-        z += v[k];
-        if (v[k] > 0.f) zl += v[k] * logf(v[k]);
-        nvr += meta_visual(mw[k]);
-        sbar_s[i] = v[k];
-        keys[i] = mw[k];
-        cells[i] = static_cast<uint16_t>(g);
+        if (i < nr) fuse(i, v[k], g, mw[k]);
       }
     }
-  }
-  for (int i0 = 0; i0 < (per_head ? 0 : nr); i0 += 2 * kCalThreads) {
-    float v[2][kMaxGroups];
-    uint32_t mw[2];
+  } else {
+    for (int i0 = 0; i0 < nr; i0 += 2 * kCalThreads) {
+      float v[2][kMaxGroups];
+      uint32_t mw[2];
 #pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      const int i = i0 + k * kCalThreads + tid;
-      mw[k] = 0u;
+      for (int k = 0; k < 2; ++k) {
+        const int i = i0 + k * kCalThreads + tid;
+        mw[k] = 0u;
 #pragma unroll
-      for (int gg = 0; gg < kMaxGroups; ++gg) v[k][gg] = 0.f;
-      if (i < nr) {
-        const int t = ta + i;
-        mw[k] = meta[t];
+        for (int gg = 0; gg < kMaxGroups; ++gg) v[k][gg] = 0.f;
+        if (i < nr) {
+          const int t = ta + i;
+          mw[k] = meta[t];
 #pragma unroll
-        for (int gg = 0; gg < kMaxGroups; ++gg)
-          if (gg < G) v[k][gg] = S0[static_cast<int64_t>(gg) * Lp + t];
-      }
-    }
-#pragma unroll
-    for (int k = 0; k < 2; ++k) {
-      const int i = i0 + k * kCalThreads + tid;
-      if (i >= nr) continue;
-      // s_bar (Eq. 4) and its governing group g* (lowest on ties)
-      float best = v[k][0], acc = best;
-      int gs = 0;
-#pragma unroll
-      for (int gg = 1; gg < kMaxGroups; ++gg) {
-        if (gg >= G) break;
-        acc += v[k][gg];
-        if (v[k][gg] > best) {
-          best = v[k][gg];
-          gs = gg;
+          for (int gg = 0; gg < kMaxGroups; ++gg)
+            if (gg < G) v[k][gg] = S0[static_cast<int64_t>(gg) * Lp + t];
         }
       }
-      const float sb = acc * invG;
-      z += sb;
-      if (sb > 0.f) zl += sb * logf(sb);
-      nvr += meta_visual(mw[k]);
-      sbar_s[i] = sb;
-      keys[i] = mw[k];
-      cells[i] = static_cast<uint16_t>(gs);
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const int i = i0 + k * kCalThreads + tid;
+        if (i >= nr) continue;
+        // s_bar (Eq. 4) and its governing group g* (lowest on ties)
+        float best = v[k][0], acc = best;
+        int gs = 0;
+#pragma unroll
+        for (int gg = 1; gg < kMaxGroups; ++gg) {
+          if (gg >= G) break;
+          acc += v[k][gg];
+          if (v[k][gg] > best) {
+            best = v[k][gg];
+            gs = gg;
+          }
+        }
+        fuse(i, acc * invG, gs, mw[k]);
+      }
     }
   }
-  z = block_sum<float>(z, sh.fred);
-  zl = block_sum<float>(zl, sh.fred);
-  nvr = block_sum<int>(nvr, sh.ired);
+  {
+    float r3[3] = {z, zl, nvf};
+    block_reduce<3>(r3, kmn, kmx, sh);
+    z = r3[0];
+    zl = r3[1];
+    nvf = r3[2];
+  }
   if (tid == 0) {
     sh.zpart = z;
     sh.hpart = zl;
-    sh.vpart = nvr;
+    sh.vpart = nvf;
+    sh.kminp = kmn;
+    sh.kmaxp = kmx;
   }
   cluster_sync();
-  auto entropy = [&](float Zr, float ZLr) {
+  if (tid < G) {   // every CTA's partials, one peer per thread
+    sh.pz[tid] = dsmem_ld_f32(dsmem_map(&sh.zpart, tid));
+    sh.pzl[tid] = dsmem_ld_f32(dsmem_map(&sh.hpart, tid));
+    sh.pv[tid] = dsmem_ld_f32(dsmem_map(&sh.vpart, tid));
+    sh.pkmin[tid] = static_cast<uint32_t>(dsmem_ld_s32(dsmem_map(&sh.kminp, tid)));
+    sh.pkmax[tid] = static_cast<uint32_t>(dsmem_ld_s32(dsmem_map(&sh.kmaxp, tid)));
+  }
+  __syncthreads();
+  auto entropy = [&](float Zr, float ZL2r) {   // ZL2r = sum s log2 s
     const float Ze = Zr + kp.eps_h;
-    const float plogp = Zr > 0.f ? ZLr / Ze - (Zr / Ze) * logf(Ze) : 0.f;
+    const float plogp = Zr > 0.f ? kLn2 * ZL2r / Ze - (Zr / Ze) * logf(Ze) : 0.f;
     return Lp > 1 ? -plogp / logf(static_cast<float>(Lp)) : 0.f;
   };
   float Hn, T;
+  uint32_t kmin2 = kmn, kmax2 = kmx;   // key range of the selection
   if (per_head) {
     Hn = entropy(z, zl);   // this CTA's own row
     T = kp.t_min + (kp.t_max - kp.t_min) * Hn;
     if (tid == 0 && g == 0 && stats) {
       float hs = 0.f, ts = 0.f, zs = 0.f;
       for (int r = 0; r < G; ++r) {
-        const float Zr = dsmem_ld_f32(dsmem_map(&sh.zpart, r));
-        const float Hr = entropy(Zr, dsmem_ld_f32(dsmem_map(&sh.hpart, r)));
+        const float Hr = entropy(sh.pz[r], sh.pzl[r]);
         const float Tr = kp.t_min + (kp.t_max - kp.t_min) * Hr;
         stats[8 + 4 * G + r] = Hr;
         stats[8 + 5 * G + r] = Tr;
         hs += Hr;
         ts += Tr;
-        zs += Zr;
+        zs += sh.pz[r];
       }
       stats[0] = hs * invG;
       stats[1] = ts * invG;
       stats[4] = zs * invG;   // sum_t s_bar_t = mean over g of the row sums
-      stats[5] = static_cast<float>(nvr);
+      stats[5] = nvf;
     }
   } else {
-    float Z = 0.f, ZL = 0.f;
-    int nvis = 0;
+    float Z = 0.f, ZL = 0.f, NV = 0.f;
+    kmin2 = 0xFFFFFFFFu;
+    kmax2 = 0u;
     for (int r = 0; r < G; ++r) {
-      Z += dsmem_ld_f32(dsmem_map(&sh.zpart, r));
-      ZL += dsmem_ld_f32(dsmem_map(&sh.hpart, r));
-      nvis += dsmem_ld_s32(dsmem_map(&sh.vpart, r));
+      Z += sh.pz[r];
+      ZL += sh.pzl[r];
+      NV += sh.pv[r];
+      kmin2 = min(kmin2, sh.pkmin[r]);
+      kmax2 = max(kmax2, sh.pkmax[r]);
     }
     Hn = entropy(Z, ZL);
     T = kp.t_min + (kp.t_max - kp.t_min) * Hn;
@@ -769,125 +860,228 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       stats[0] = Hn;
       stats[1] = T;
       stats[4] = Z;
-      stats[5] = static_cast<float>(nvis);
+      stats[5] = NV;
       for (int r = 0; r < G; ++r) {
         stats[8 + 4 * G + r] = Hn;
         stats[8 + 5 * G + r] = T;
       }
     }
   }
+  // ---- Sec. 3.6: s_t = x_t^(1/T) = 2^(log2(x_t) / T) (hardware exp2 / log2,
+  // relative error a few 1e-7); first level of the top-B select: 4096
+  // buckets spread linearly over the selection's key range (monotone in the key)
   const float invT = 1.f / T;
-  // ---- Eq. (final_score) with Eq. (9): fused score, its descending key and
-  // the first digit of the top-B select
-  const float lam = sh.lam;
   float* score = per_head ? sv.score + (static_cast<int64_t>(layer) * G + g) * Lp
                           : sv.score + static_cast<int64_t>(layer) * Lp + ta;
+  const float sbinv = kmax2 >= kmin2 ? 4096.f / (static_cast<float>(kmax2 - kmin2) + 1.f) : 0.f;
+  auto sbucket = [&](uint32_t u) {
+    return min(kBins0 - 1, static_cast<int>(static_cast<float>(u - kmin2) * sbinv));
+  };
   for (int i = tid; i < nr; i += kCalThreads) {
-    const float sb = sbar_s[i];
-    const int gs = cells[i];
-    const uint32_t mt = keys[i];
-    const float beta = (1.f - lam) + lam * static_cast<float>(G) * sh.w[gs];
-    float d = 1.f;
-    if (meta_visual(mt)) {
-      const float df = static_cast<float>(sv.cur_frame - meta_frame(mt));
-      d = kp.d_min + (1.f - kp.d_min) * expf(-kp.delta * df * sh.ph[gs]);
-    }
-    const float s = powf(fmaxf(sb * beta * d, 0.f), invT);
-    score[i] = s;
-    const uint32_t key = ~order_key(s);   // descending score = ascending key
-    keys[i] = key;
-    atomicAdd(&hist[key >> 20], 1);
+    score[i] = ex2_approx(invT * lg2_approx(xs[i]));
+    atomicAdd(&hist[sbucket(keys[i])], 1);
   }
 
-  // ---- Sec. 3.7: global top-B, ties to the lower index (per-KV-head mode:
-  // the histograms and offsets of this CTA's row alone)
+  // ---- Sec. 3.7: top-B, ties to the lower index (global mode: over the
+  // cluster; per-KV-head mode: over this CTA's row, block barriers only)
   const int B = sv.budget;   // the same in every CTA of the cluster
-  const int r_lo = per_head ? g : 0, r_hi = per_head ? g + 1 : G;
   if (B > 0) {
-    cluster_sync();
-    // digit 1 over the cluster: 4 bins per thread
+    const int r_lo = per_head ? g : 0, r_hi = per_head ? g + 1 : G;
+    auto sel_sync = [&]() {
+      if (per_head) __syncthreads();
+      else cluster_sync();
+    };
+    sel_sync();   // every bucket histogram of the selection is complete
     {
-      int4 h = make_int4(0, 0, 0, 0);
-      for (int r = r_lo; r < r_hi; ++r) {
-        const int4 q = dsmem_ld_v4(dsmem_map(hist + 4 * tid, r));
-        h.x += q.x;
-        h.y += q.y;
-        h.z += q.z;
-        h.w += q.w;
-      }
+      int4 h = sum_peers_v4(hist + 4 * tid, r_lo, r_hi);
       const int sum = (h.x + h.y) + (h.z + h.w);
       const int excl = block_excl_scan(sum, sh.scan, nullptr);
       const int rank = B - 1;
       if (rank >= excl && rank < excl + sum) {
-        int c = excl, d = 0;
-        if (rank >= c + h.x) { c += h.x; d = 1; }
-        if (d == 1 && rank >= c + h.y) { c += h.y; d = 2; }
-        if (d == 2 && rank >= c + h.z) { c += h.z; d = 3; }
-        sh.tprefix = static_cast<uint32_t>(tid * 4 + d) << 20;
+        int c = excl, d = 0, n = h.x;
+        if (rank >= c + h.x) { c += h.x; d = 1; n = h.y; }
+        if (d == 1 && rank >= c + h.y) { c += h.y; d = 2; n = h.z; }
+        if (d == 2 && rank >= c + h.z) { c += h.z; d = 3; n = h.w; }
+        sh.tb = tid * 4 + d;
         sh.trank = rank - c;
+        sh.tcnt = n;
       }
     }
     __syncthreads();
-    // digits 2 and 3: histogram B (past the digit-1 bins), then histogram A
-    // again (every CTA has read the peers' digit-1 bins before the barrier)
-    for (int pass = 1; pass <= 2; ++pass) {
-      const int shift = pass == 1 ? 10 : 0;
-      int* hp = pass == 1 ? hist + kBins0 : hist;
-      const uint32_t P = sh.tprefix;
-      const int rk = sh.trank;
-      hp[tid] = 0;
-      __syncthreads();
-      for (int i = tid; i < nr; i += kCalThreads) {
-        const uint32_t u = keys[i];
-        if (((u ^ P) >> (shift + 10)) == 0) atomicAdd(&hp[(u >> shift) & 1023], 1);
-      }
-      cluster_sync();
-      int v = 0;
-      for (int r = r_lo; r < r_hi; ++r) v += dsmem_ld_s32(dsmem_map(hp + tid, r));
-      const int excl = block_excl_scan(v, sh.scan, nullptr);
-      if (rk >= excl && rk < excl + v) {
-        sh.tprefix = P | (static_cast<uint32_t>(tid) << shift);
-        sh.trank = rk - excl;
-      }
-      __syncthreads();
-    }
-    // kept: key < P, or key == P and among the first rk + 1 equal keys in
-    // position order; contiguous spans per thread keep position order
-    const uint32_t P = sh.tprefix;
-    const int rk = sh.trank;
+    const int bstar = sh.tb, rkb = sh.trank, ncb = sh.tcnt;
+    int32_t* idx = sv.idx + (static_cast<int64_t>(layer) * (per_head ? G : 1) + (per_head ? g : 0)) * B;
     const int cs = ceil_div(nr, kCalThreads);
     const int i0 = min(nr, tid * cs), i1 = min(nr, i0 + cs);
-    int nlt = 0, neq = 0;
-    for (int i = i0; i < i1; ++i) {
-      const uint32_t u = keys[i];
-      nlt += u < P;
-      neq += u == P;
-    }
-    int tot_lt, tot_eq;
-    int lt_b = block_excl_scan(nlt, sh.scan, &tot_lt);
-    int eq_b = block_excl_scan(neq, sh.scan, &tot_eq);
-    if (tid == 0) {
-      sh.nlt = tot_lt;
-      sh.neq = tot_eq;
-    }
-    cluster_sync();
-    for (int r = r_lo; r < g; ++r) {
-      lt_b += dsmem_ld_s32(dsmem_map(&sh.nlt, r));
-      eq_b += dsmem_ld_s32(dsmem_map(&sh.neq, r));
-    }
-    int32_t* idx = sv.idx + (static_cast<int64_t>(layer) * (per_head ? G : 1) + (per_head ? g : 0)) * B;
-    for (int i = i0; i < i1; ++i) {
-      const uint32_t u = keys[i];
-      int pos = -1;
-      if (u < P) {
-        pos = lt_b + min(eq_b, rk + 1);
-        ++lt_b;
-      } else if (u == P) {
-        if (eq_b <= rk) pos = lt_b + eq_b;
-        ++eq_b;
+    // the same decision in every CTA: it depends on the summed histogram only
+    if (ncb <= kCandMax && ncb <= capl / 4) {
+      // the boundary bucket's tokens as (key, position) pairs in shared memory
+      // (the cell array is free in this phase), the tokens below it counted
+      uint32_t* clist = reinterpret_cast<uint32_t*>(scells);
+      if (tid == 0) sh.tcand = 0;
+      __syncthreads();
+      float below = 0.f;
+      for (int i = tid; i < nr; i += kCalThreads) {
+        const uint32_t u = keys[i];
+        const int bk = sbucket(u);
+        if (bk < bstar) {
+          below += 1.f;
+        } else if (bk == bstar) {
+          const int j = atomicAdd(&sh.tcand, 1);
+          clist[2 * j] = u;
+          clist[2 * j + 1] = static_cast<uint32_t>(ta + i);
+        }
       }
-      if (pos >= B) atomicOr(st.err, kErrIndex);   // cannot happen for a correct select
-      else if (pos >= 0) idx[pos] = ta + i;
+      {
+        float b1[1] = {below};
+        uint32_t u0 = 0u, u1 = 0u;
+        block_reduce<1>(b1, u0, u1, sh);
+        if (tid == 0) sh.nbelow = static_cast<int>(b1[0]);
+      }
+      sel_sync();   // every candidate list is complete
+      if (tid >= r_lo && tid < r_hi) {
+        sh.pncand[tid] = dsmem_ld_s32(dsmem_map(&sh.tcand, tid));
+        sh.pbelow[tid] = dsmem_ld_s32(dsmem_map(&sh.nbelow, tid));
+      }
+      __syncthreads();
+      // gather the candidates of the selection into the histogram area (no
+      // peer reads it any more), then rank each by (key, position)
+      uint32_t* all = reinterpret_cast<uint32_t*>(hist);
+      int nall = 0, nlow = 0;
+      for (int r = r_lo; r < r_hi; ++r) {
+        const int n = sh.pncand[r];
+        for (int j = tid; j < 2 * n; j += kCalThreads)
+          all[2 * nall + j] = static_cast<uint32_t>(dsmem_ld_s32(dsmem_map(clist + j, r)));
+        nall += n;
+        if (r < g) nlow += sh.pbelow[r];
+      }
+      __syncthreads();
+      for (int i = tid; i < nall; i += kCalThreads) {
+        const uint32_t ki = all[2 * i], ti = all[2 * i + 1];
+        int rank = 0;
+        for (int j = 0; j < nall; ++j) {
+          const uint32_t kj = all[2 * j], tj = all[2 * j + 1];
+          rank += (kj < ki) || (kj == ki && tj < ti);
+        }
+        if (rank == rkb) {
+          sh.tkey = ki;
+          sh.tpos = static_cast<int>(ti);
+        }
+      }
+      __syncthreads();
+      const uint32_t kT = sh.tkey;
+      const uint32_t tT = static_cast<uint32_t>(sh.tpos);
+      auto kept = [&](uint32_t u, uint32_t t) { return u < kT || (u == kT && t <= tT); };
+      // kept tokens of the lower-ranked CTAs: all of their tokens below the
+      // boundary bucket and their kept candidates
+      float lowc = 0.f;
+      for (int i = tid; i < nall; i += kCalThreads) {
+        const uint32_t ti = all[2 * i + 1];
+        if (static_cast<int>(ti) < ta && kept(all[2 * i], ti)) lowc += 1.f;
+      }
+      int nk = 0;
+      for (int i = i0; i < i1; ++i) nk += kept(keys[i], static_cast<uint32_t>(ta + i));
+      {
+        float l1[1] = {lowc};
+        uint32_t u0 = 0u, u1 = 0u;
+        block_reduce<1>(l1, u0, u1, sh);
+        lowc = l1[0];
+      }
+      int pos = nlow + static_cast<int>(lowc) + block_excl_scan(nk, sh.scan, nullptr);
+      for (int i = i0; i < i1; ++i) {
+        if (!kept(keys[i], static_cast<uint32_t>(ta + i))) continue;
+        if (pos >= B) atomicOr(st.err, kErrIndex);   // cannot happen for a correct select
+        else idx[pos] = ta + i;
+        ++pos;
+      }
+    } else {
+      // many equal keys around the boundary: an exact radix select over the
+      // keys (12 + 10 + 10-bit digits), then ordered compaction
+      sel_sync();   // the peers have read this CTA's bucket histogram
+      for (int i = tid; i < kBins0; i += kCalThreads) hist[i] = 0;
+      __syncthreads();
+      for (int i = tid; i < nr; i += kCalThreads) atomicAdd(&hist[keys[i] >> 20], 1);
+      sel_sync();
+      {
+        int4 h = sum_peers_v4(hist + 4 * tid, r_lo, r_hi);
+        const int sum = (h.x + h.y) + (h.z + h.w);
+        const int excl = block_excl_scan(sum, sh.scan, nullptr);
+        const int rank = B - 1;
+        if (rank >= excl && rank < excl + sum) {
+          int c = excl, d = 0;
+          if (rank >= c + h.x) { c += h.x; d = 1; }
+          if (d == 1 && rank >= c + h.y) { c += h.y; d = 2; }
+          if (d == 2 && rank >= c + h.z) { c += h.z; d = 3; }
+          sh.tprefix = static_cast<uint32_t>(tid * 4 + d) << 20;
+          sh.trank = rank - c;
+        }
+      }
+      __syncthreads();
+      // digits 2 and 3: histogram B (past the digit-1 bins), then histogram A
+      // again (every CTA has read the peers' digit-1 bins before the barrier)
+      for (int pass = 1; pass <= 2; ++pass) {
+        const int shift = pass == 1 ? 10 : 0;
+        int* hp = pass == 1 ? hist + kBins0 : hist;
+        const uint32_t P = sh.tprefix;
+        const int rk = sh.trank;
+        hp[tid] = 0;
+        __syncthreads();
+        for (int i = tid; i < nr; i += kCalThreads) {
+          const uint32_t u = keys[i];
+          if (((u ^ P) >> (shift + 10)) == 0) atomicAdd(&hp[(u >> shift) & 1023], 1);
+        }
+        sel_sync();
+        int v = 0;
+        {
+          int q[kMaxGroups];
+#pragma unroll
+          for (int r = 0; r < kMaxGroups; ++r)
+            if (r < r_hi - r_lo) q[r] = dsmem_ld_s32(dsmem_map(hp + tid, r_lo + r));
+#pragma unroll
+          for (int r = 0; r < kMaxGroups; ++r)
+            if (r < r_hi - r_lo) v += q[r];
+        }
+        const int excl = block_excl_scan(v, sh.scan, nullptr);
+        if (rk >= excl && rk < excl + v) {
+          sh.tprefix = P | (static_cast<uint32_t>(tid) << shift);
+          sh.trank = rk - excl;
+        }
+        __syncthreads();
+      }
+      // kept: key < P, or key == P and among the first rk + 1 equal keys in
+      // position order; contiguous spans per thread keep position order
+      const uint32_t P = sh.tprefix;
+      const int rk = sh.trank;
+      int nlt = 0, neq = 0;
+      for (int i = i0; i < i1; ++i) {
+        const uint32_t u = keys[i];
+        nlt += u < P;
+        neq += u == P;
+      }
+      int tot_lt, tot_eq;
+      int lt_b = block_excl_scan(nlt, sh.scan, &tot_lt);
+      int eq_b = block_excl_scan(neq, sh.scan, &tot_eq);
+      if (tid == 0) {
+        sh.nlt = tot_lt;
+        sh.neq = tot_eq;
+      }
+      sel_sync();
+      for (int r = r_lo; r < g; ++r) {
+        lt_b += dsmem_ld_s32(dsmem_map(&sh.nlt, r));
+        eq_b += dsmem_ld_s32(dsmem_map(&sh.neq, r));
+      }
+      for (int i = i0; i < i1; ++i) {
+        const uint32_t u = keys[i];
+        int pos = -1;
+        if (u < P) {
+          pos = lt_b + min(eq_b, rk + 1);
+          ++lt_b;
+        } else if (u == P) {
+          if (eq_b <= rk) pos = lt_b + eq_b;
+          ++eq_b;
+        }
+        if (pos >= B) atomicOr(st.err, kErrIndex);   // cannot happen for a correct select
+        else if (pos >= 0) idx[pos] = ta + i;
+      }
     }
   }
   cluster_sync();   // the peers' shared memory stays valid until every remote read is done
