@@ -152,6 +152,24 @@ __device__ __forceinline__ uint64_t sdesc_k_sw128(uint32_t saddr) {
   return d;
 }
 
+// Shared-memory matrix descriptor of a K-major operand without swizzling:
+// 8-row x 16-byte core matrices, `lbo` bytes between the two core matrices of
+// a 16-element K slice, `sbo` bytes between consecutive 8-row groups.
+__device__ __forceinline__ uint64_t sdesc_k_none(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);         // start address (16 B units)
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;     // leading (K) byte offset
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;     // stride (M / N) byte offset
+  d |= static_cast<uint64_t>(1) << 46;                        // descriptor version (tcgen05)
+  return d;                                                    // swizzle mode 0: none
+}
+
+// Makes this thread's generic-proxy shared-memory writes visible to later
+// async-proxy reads (tensor-core operands).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 // Instruction descriptor of tcgen05.mma kind::f16 with bf16 A and B (both
 // K-major), fp32 accumulator, shape M x N.
 __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N) {

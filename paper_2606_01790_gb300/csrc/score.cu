@@ -11,11 +11,13 @@
 //                           sum of exp2) pair for its row over its keys and
 //                           one partial per (row, piece) is written.
 //   pass 2 (k_score_accum): keys on TMEM lanes (M = 128), the group's window
-//                           rows on columns (N <= 256); each thread sums
-//                           exp2(z * log2e/sqrt(d) - lse2[col]) over its
-//                           columns, so the per-key group sum needs no
-//                           cross-lane reduction.  The score matrix never
-//                           leaves the chip.
+//                           rows on columns (N <= 256); one extra K step adds
+//                           -lse2[col] sqrt(d)/log2e to every logit (a ones
+//                           operand against the rows' -lse as three bf16
+//                           parts), and each thread sums exp2(acc log2e/sqrt(d))
+//                           over its columns, so the per-key group sum needs
+//                           no cross-lane reduction and no per-column operand.
+//                           The score matrix never leaves the chip.
 // Both passes split the flattened (seq, layer, group, key tile) space into one
 // contiguous range per CTA (persistent grid <= #SMs), so a CTA reloads the
 // group's queries only when its range crosses into a new (seq, layer, group)
@@ -25,6 +27,7 @@
 // warps.  Two 256-column TMEM accumulator stages let the MMA of tile i+1 run
 // under the epilogue of tile i; TMEM is read in 16-column loads with the next
 // load in flight under the arithmetic, which runs on packed fp32 pairs.
+#include <algorithm>
 #include <utility>
 
 #include "common.cuh"
@@ -35,7 +38,7 @@ namespace starkv {
 
 namespace {
 
-constexpr int kMaxStages = 5;                 // K-tile pipeline depth (at most)
+constexpr int kMaxStages = 4;                 // K-tile pipeline depth (at most)
 constexpr size_t kSmemLimit = 227 * 1024;
 constexpr int kTileBytes = kTileKeys * 256;   // 128 keys x 128 bf16
 constexpr int kHalfBytes = kTileKeys * 128;   // one 64-column swizzled half
@@ -45,6 +48,8 @@ constexpr int kEpiWarp0 = 4;                  // first epilogue warp (warpgroup 
 constexpr int kEpiWarps = 16;
 constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr uint32_t kFull = 0xffffffffu;
+constexpr int kXOnesBytes = 256;              // pass 2: the ones operand (two 8 x 16 B core matrices)
+constexpr int kXRowBytes = 32;                // pass 2: one window row of the -lse operand (16 bf16)
 
 struct TileCoord {
   int s, l, g, j;
@@ -112,10 +117,13 @@ struct SmemCtl {
   uint64_t t_empty[2];
   uint64_t q_full;
   uint64_t q_empty;
+  uint64_t x_full[2];   // pass 2: a piece's -lse operand is in its buffer
   uint64_t drain;
   uint32_t tmem_base;
   volatile int abort;
 };
+
+static_assert(sizeof(SmemCtl) <= 256, "the control block has 256 bytes");
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
@@ -137,6 +145,7 @@ __device__ __forceinline__ void ctl_init(SmemCtl* ctl, int kstages) {
   }
   mbar_init(&ctl->q_full, 1);
   mbar_init(&ctl->q_empty, kMmaThreads);   // each MMA thread commits once per piece
+  for (int i = 0; i < 2; ++i) mbar_init(&ctl->x_full[i], 1);
   mbar_init(&ctl->drain, kMmaThreads);
   ctl->abort = 0;
   fence_mbar_init();
@@ -203,13 +212,19 @@ __device__ void producer_loop(const ScoreParams& p, SmemCtl* ctl, uint8_t* sQ, u
 // for its own MMAs.
 template <int PASS>
 __device__ void mma_loop(const ScoreParams& p, SmemCtl* ctl, const uint8_t* sQ, const uint8_t* sK,
-                         uint32_t tmem, int64_t fb, int64_t fe, int who) {
+                         const uint8_t* sX, uint32_t tmem, int64_t fb, int64_t fe, int who) {
   const uint32_t idesc = PASS == 1 ? idesc_bf16(128, kTileKeys) : idesc_bf16(128, p.n2);
   // shared-memory descriptors are built once; an MMA only adds its operand's
   // offset (in 16-byte units) to the start-address field, which cannot carry
   // out of the field inside the 227 KB window
   const uint64_t dq0 = sdesc_k_sw128(smem_u32(sQ)), dk0 = sdesc_k_sw128(smem_u32(sK));
   const uint32_t qhalf16 = (p.q_rows * 128) >> 4;
+  // pass 2, one more K step per tile: a constant operand of ones (every 8-key
+  // group shares one core matrix) times each window row's -lse2 / scale as
+  // three bf16 parts, so that the accumulator holds z - lse2 / scale
+  const uint64_t dax = sdesc_k_none(smem_u32(sX), 128, 0);
+  const uint64_t dbx0 = sdesc_k_none(smem_u32(sX) + kXOnesBytes, 128, 256);
+  uint64_t dbx = dbx0;
   // K stage and phase of tile jt = who, who + 2, ...
   int stage = who % p.kstages, phase = 0, pc = 0, own = 0;
   const uint32_t d0 = tmem + who * 256;
@@ -219,6 +234,10 @@ __device__ void mma_loop(const ScoreParams& p, SmemCtl* ctl, const uint8_t* sQ, 
     if (ctl->abort) break;
     if (c.first(fb)) {
       if (!mbar_wait(&ctl->q_full, pc & 1, p.wait_ns)) { fail(ctl, p.err); break; }
+      if (PASS == 2) {
+        if (!mbar_wait(&ctl->x_full[pc & 1], (pc >> 1) & 1, p.wait_ns)) { fail(ctl, p.err); break; }
+        dbx = dbx0 + static_cast<uint64_t>((pc & 1) * ((p.q_rows * kXRowBytes) >> 4));
+      }
       ++pc;
     }
     if ((jt & 1) == who) {
@@ -248,6 +267,7 @@ __device__ void mma_loop(const ScoreParams& p, SmemCtl* ctl, const uint8_t* sQ, 
           const uint32_t qoff16 = (kk >> 2) * qhalf16 + (kk & 3) * 2;
           mma_bf16(d0, dk + koff16, dq0 + qoff16, idesc, kk > 0);
         }
+        mma_bf16(d0, dax, dbx, idesc, 1);
       }
       mma_commit(&ctl->k_empty[stage]);
       mma_commit(&ctl->t_full[who]);
@@ -396,22 +416,6 @@ __device__ __forceinline__ void lse_tile(uint32_t base, int nch, int lim, float 
   }
 }
 
-// sum over 16 columns of exp2(z * sc + nl[col]), nl = -lse2 of the columns
-__device__ __forceinline__ void accum16(const uint32_t (&r)[16], const float4* nl, float sc, float2& a0,
-                                        float2& a1) {
-  const float2 sc2 = make_float2(sc, sc);
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float4 l = nl[i];
-    const float2 t0 = ffma2(make_float2(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1])), sc2,
-                            make_float2(l.x, l.y));
-    const float2 t1 = ffma2(make_float2(__uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3])), sc2,
-                            make_float2(l.z, l.w));
-    a0 = fadd2(a0, make_float2(ex2_approx(t0.x), ex2_approx(t0.y)));
-    a1 = fadd2(a1, make_float2(ex2_approx(t1.x), ex2_approx(t1.y)));
-  }
-}
-
 }  // namespace
 
 // 20 warps share the register file: at most 96 registers a thread.
@@ -443,7 +447,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_lse(const __grid_con
   if (warp == 0) {
     if (lane == 0) producer_loop<1>(p, ctl, sQ, sK, fb, fe);
   } else if (warp == 1 || warp == 2) {
-    if (lane == 0) mma_loop<1>(p, ctl, sQ, sK, tmem, fb, fe, warp - 1);
+    if (lane == 0) mma_loop<1>(p, ctl, sQ, sK, nullptr, tmem, fb, fe, warp - 1);
   } else if (warp >= kEpiWarp0) {
     const int wg = (warp - kEpiWarp0) >> 2;  // epilogue warpgroup 0..3
     const int quad = warp & 3;              // TMEM lane quadrant
@@ -521,7 +525,8 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
   uint8_t* sQ = smem;                          // [2 halves][q_rows][128 B]
   uint8_t* sK = smem + 2 * p.q_rows * 128;     // [kstages][2 halves][128][128 B]
   SmemCtl* ctl = reinterpret_cast<SmemCtl*>(sK + p.kstages * kTileBytes);
-  float* nlse = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(ctl) + 256);  // [256] -lse2
+  // ones operand [256 B], then two buffers of the -lse operand [q_rows][32 B]
+  uint8_t* sX = reinterpret_cast<uint8_t*>(ctl) + 256;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) ctl_init(ctl, p.kstages);
@@ -543,7 +548,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
   if (warp == 0) {
     if (lane == 0) producer_loop<2>(p, ctl, sQ, sK, fb, fe);
   } else if (warp == 1 || warp == 2) {
-    if (lane == 0) mma_loop<2>(p, ctl, sQ, sK, tmem, fb, fe, warp - 1);
+    if (lane == 0) mma_loop<2>(p, ctl, sQ, sK, sX, tmem, fb, fe, warp - 1);
   } else if (warp >= kEpiWarp0) {
     const int et = threadIdx.x - 32 * kEpiWarp0;   // 0..511
     const int wg = et >> 7;                 // column quarter
@@ -553,21 +558,59 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
     const int ch0 = wg * (nc >> 2) + min(wg, nc & 3);
     const int nch = (nc >> 2) + (wg < (nc & 3) ? 1 : 0);
     const uint32_t base0 = tmem + (static_cast<uint32_t>(quad * 32) << 16) + ch0 * 16;
-    const float4* nl = reinterpret_cast<const float4*>(nlse + ch0 * 16);
-    const float sc = p.scale2;
-    int jt = 0;
+    const float sc = p.scale2, isc = 1.f / p.scale2;
+    // the -lse operand of the piece whose row starts at flat tile r0, into
+    // buffer `buf`: window row et holds x = -lse2 / scale as three bf16 parts
+    // (x = hi + mid + lo to about 2^-24 relative) in its K columns 0..2;
+    // rows past the group's window rows get a large negative x (exp2 -> 0)
+    auto write_x = [&](int64_t r0, int nt, int buf) {
+      if (et < p.n2) {
+        float x = -3.0e38f;
+        if (et < p.rows) x = -combine_lse2(p, r0, nt, et) * isc;
+        const __nv_bfloat16 hi = __float2bfloat16_rn(x);
+        const float r1 = x - __bfloat162float(hi);
+        const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
+        const __nv_bfloat16 lo = __float2bfloat16_rn(r1 - __bfloat162float(mid));
+        uint8_t* row = sX + kXOnesBytes + buf * (p.q_rows * kXRowBytes) + (et >> 3) * 256 + (et & 7) * 16;
+        *reinterpret_cast<uint4*>(row) =
+            make_uint4(static_cast<uint32_t>(__bfloat16_as_ushort(hi)) | (static_cast<uint32_t>(__bfloat16_as_ushort(mid)) << 16),
+                       static_cast<uint32_t>(__bfloat16_as_ushort(lo)), 0u, 0u);
+        *reinterpret_cast<uint4*>(row + 128) = make_uint4(0u, 0u, 0u, 0u);
+      }
+      fence_proxy_async_smem();
+      named_bar_sync(1, kEpiThreads);
+      if (et == 0) mbar_arrive(&ctl->x_full[buf]);
+    };
+    int jt = 0, kp = 0;
     bool dead = false;
     float* dst = nullptr;   // this thread's copy of the piece's unpooled row
     int lp = 0;
     TileIter c;
-    for (c.init(p, fb, fe); c.valid(); c.next(p)) {
+    c.init(p, fb, fe);
+    if (c.valid()) {
+      // the ones operand: bf16 1.0 in K columns 0..2 of core matrix 0, zeros elsewhere
+      if (et < 16) {
+        *reinterpret_cast<uint4*>(sX + et * 16) =
+            et < 8 ? make_uint4(0x3F803F80u, 0x00003F80u, 0u, 0u) : make_uint4(0u, 0u, 0u, 0u);
+      }
+      write_x(c.f - c.j, c.nt, 0);
+    }
+    const float2 sc2 = make_float2(sc, sc), zero2 = make_float2(0.f, 0.f);
+    for (; c.valid(); c.next(p)) {
       if (c.first(fb)) {
-        named_bar_sync(1, kEpiThreads);   // the previous piece's readers are done
-        if (et < kMaxRows) nlse[et] = et < p.rows ? -combine_lse2(p, c.f - c.j, c.nt, et) : -INFINITY;
+        // the next piece's operand goes to the other buffer now, one piece
+        // ahead of its MMAs (this piece's buffer was written one piece earlier;
+        // the other one's readers, the previous piece's MMAs, are done)
+        const int64_t fn = c.f + (c.nt - c.j);
+        if (fn < fe) {
+          TileIter n;
+          n.init(p, fn, fe);
+          write_x(fn, n.nt, (kp + 1) & 1);
+        }
+        ++kp;
         const ScoreSeq& sq = p.seq[c.s];
         lp = sq.Lp;
         dst = sq.s_raw + (static_cast<int64_t>(c.l * p.G + c.g) * kRawCopies + wg) * lp + q;
-        named_bar_sync(1, kEpiThreads);
       }
       const int ts = jt & 1;
       if (!dead) {
@@ -578,7 +621,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
           tc_fence_after();
           float2 a0 = make_float2(0.f, 0.f), a1 = make_float2(0.f, 0.f);
           if (nch > 0)
-            stream16(base0 + ts * 256, nch, [&](const uint32_t(&v)[16], int ch) { accum16(v, nl + ch * 4, sc, a0, a1); });
+            stream16(base0 + ts * 256, nch, [&](const uint32_t(&v)[16], int) { exp2_acc16(v, sc2, zero2, a0, a1); });
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(&ctl->t_empty[ts]);
@@ -622,10 +665,11 @@ __global__ void k_pool(const __grid_constant__ SeqBatch b, int G, int H, int poo
   s.S[(static_cast<int64_t>(layer) * G + g) * s.Lp + t] = acc * scale;
 }
 
-// alignment slack + Q + K stages + control block + pass-1 merge buffer
+// alignment slack + Q + K stages + control block + the larger of the pass-1
+// merge buffer and the pass-2 -lse operands (ones + two row buffers)
 size_t score_smem_bytes(int q_rows, int kstages) {
-  return 1024 + static_cast<size_t>(2 * q_rows * 128) + static_cast<size_t>(kstages) * kTileBytes + 256 +
-         4 * 128 * sizeof(float2);
+  const size_t aux = std::max<size_t>(4 * 128 * sizeof(float2), kXOnesBytes + 2 * static_cast<size_t>(q_rows) * kXRowBytes);
+  return 1024 + static_cast<size_t>(2 * q_rows * 128) + static_cast<size_t>(kstages) * kTileBytes + 256 + aux;
 }
 
 int score_kstages(int q_rows) {
