@@ -287,27 +287,35 @@ __device__ void mma_loop(const ScoreParams& p, SmemCtl* ctl, const uint8_t* sQ, 
 
 // log2-domain log-sum-exp of window row `col` of the (seq, layer, group) row
 // whose first flat tile is `r0`, from the pass-1 partials of every CTA piece
-// that covered the row.
+// that covered the row: one pass, eight partials loaded at a time, each batch
+// merged into the running (maximum, sum).
 __device__ float combine_lse2(const ScoreParams& p, int64_t r0, int nt, int col) {
   const int64_t T = p.total_tiles;
   const int P = p.grid1;
   const int64_t r1 = r0 + nt - 1;
   const int c0 = static_cast<int>(((r0 + 1) * P - 1) / T);
   const int c1 = static_cast<int>(((r1 + 1) * P - 1) / T);
-  float mx = -INFINITY;
-  for (int c = c0; c <= c1; ++c) {
-    const int64_t ps = max(range_begin(T, c, P), r0);
-    mx = fmaxf(mx, p.partials[ps * kMaxRows + col].x);
-  }
-  float sum = 0.f;
-  for (int c = c0; c <= c1; ++c) {
-    const int64_t ps = max(range_begin(T, c, P), r0);
-    const float2 v = p.partials[ps * kMaxRows + col];
-    sum += v.y * exp2f(v.x - mx);
+  float mx = -INFINITY, sum = 0.f;
+  for (int cb = c0; cb <= c1; cb += 8) {
+    float2 v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      v[k] = make_float2(-INFINITY, 0.f);
+      if (cb + k <= c1) v[k] = p.partials[max(range_begin(T, cb + k, P), r0) * kMaxRows + col];
+    }
+    float bm = mx;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) bm = fmaxf(bm, v[k].x);
+    if (bm == -INFINITY) continue;
+    float bs = mx == -INFINITY ? 0.f : sum * exp2f(mx - bm);
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (v[k].x != -INFINITY) bs += v[k].y * exp2f(v[k].x - bm);
+    mx = bm;
+    sum = bs;
   }
   return mx + log2f(sum);
 }
-
 
 // Streams `n` 16-column chunks of this thread's TMEM lane from `base`, one
 // load in flight under the arithmetic of the previous chunk.
