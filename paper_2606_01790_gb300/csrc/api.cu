@@ -249,7 +249,7 @@ void plan_ws(const starkv_state* st, const starkv_seq* seqs, int nseq, int nlaye
       off += align256(static_cast<size_t>(nlayers) * G * lp * 3 * sizeof(uint32_t));
     }
     p->raw_off[i] = off;
-    off += align256(static_cast<size_t>(nlayers) * G * kRawCopies * lp * sizeof(float));
+    off += align256(static_cast<size_t>(nlayers) * G * kRawCopies * raw_stride(static_cast<int>(lp)) * sizeof(float));
     if (ws_S && !seqs[i].S) {
       p->S_off[i] = off;
       off += align256(static_cast<size_t>(c.n_layers) * G * lp * sizeof(float));

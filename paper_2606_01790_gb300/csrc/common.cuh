@@ -62,7 +62,7 @@ struct SeqView {
   uint32_t* meta_out;
   int32_t* idx;    // [n_layers][P][B]
   float* S;        // [n_layers][G][Lp] (a workspace region when the caller passed NULL)
-  float* s_raw;    // [n_layers_in_launch][G][kRawCopies][Lp] unpooled sums (workspace) or NULL
+  float* s_raw;    // [n_layers_in_launch][G][kRawCopies][raw_stride(Lp)] unpooled sums (workspace) or NULL
   float* score;    // [n_layers][P][Lp] fused score, P = 1 or G (a workspace region when NULL)
   float* stats;    // optional
   uint32_t* vis;   // [n_layers_in_launch][G][3 Lp] keys, candidate list and cells of
@@ -77,5 +77,9 @@ struct SeqBatch {
 };
 
 __host__ __device__ __forceinline__ int ceil_div(int a, int b) { return (a + b - 1) / b; }
+
+// Row stride (floats) of the unpooled group sums: L_p rounded up to 4, so that
+// every row starts on a 16-byte boundary.
+__host__ __device__ __forceinline__ int raw_stride(int lp) { return (lp + 3) & ~3; }
 
 }  // namespace starkv

@@ -618,7 +618,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
         ++kp;
         const ScoreSeq& sq = p.seq[c.s];
         lp = sq.Lp;
-        dst = sq.s_raw + (static_cast<int64_t>(c.l * p.G + c.g) * kRawCopies + wg) * lp + q;
+        dst = sq.s_raw + (static_cast<int64_t>(c.l * p.G + c.g) * kRawCopies + wg) * raw_stride(lp) + q;
       }
       const int ts = jt & 1;
       if (!dead) {
@@ -658,14 +658,15 @@ __global__ void k_pool(const __grid_constant__ SeqBatch b, int G, int H, int poo
   if (t >= s.Lp) return;
   const int lg = blockIdx.y;                  // launch-local layer * G + g
   const int layer = b.layer0 + lg / G, g = lg % G;
-  const float* src = s.s_raw + static_cast<int64_t>(lg) * kRawCopies * s.Lp;
+  const int rs = raw_stride(s.Lp);
+  const float* src = s.s_raw + static_cast<int64_t>(lg) * kRawCopies * rs;
   const int half = pool >> 1;
   float acc = 0.f;
   for (int j = -half; j <= half; ++j) {
     const int u = t + j;
     if (u >= 0 && u < s.Lp) {
       float r = 0.f;
-      for (int c = 0; c < kRawCopies; ++c) r += src[c * s.Lp + u];
+      for (int c = 0; c < kRawCopies; ++c) r += src[c * rs + u];
       acc += r;
     }
   }

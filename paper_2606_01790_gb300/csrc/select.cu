@@ -380,34 +380,79 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   // given S, into the candidate region; the metadata words into the key region
   const float pscale = static_cast<float>(G) / static_cast<float>(kp.H) / static_cast<float>(kp.pool);
   const int half = kp.pool >> 1;
-  const float* raw = FROM_RAW ? sv.s_raw + static_cast<int64_t>(ll * G + g) * kRawCopies * Lp : nullptr;
+  const int rs = raw_stride(Lp);
+  const float* raw = FROM_RAW ? sv.s_raw + static_cast<int64_t>(ll * G + g) * kRawCopies * rs : nullptr;
   float* stage = reinterpret_cast<float*>(cand);
-  for (int t0 = 0; t0 < Lp; t0 += 4 * kCalThreads) {
-    float v[4];
-    uint32_t mw[4];
+  // the step's rows held on chip: four consecutive tokens per thread and
+  // 16-byte accesses (unpooled rows are 16-byte aligned; the metadata row is
+  // read in 16 bytes when its address allows)
+  const bool vec = FROM_RAW && in_smem;
+  if (vec) {
+    const bool meta16 = (reinterpret_cast<uintptr_t>(meta) & 15) == 0;
+    for (int t00 = 4 * tid; t00 < Lp; t00 += 8 * kCalThreads) {
+      float4 v[2];
+      uint4 mw[2];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int t = t0 + k * kCalThreads + tid;
-      v[k] = 0.f;
-      mw[k] = 0u;
-      if (t < Lp) {
-        mw[k] = meta[t];
-        if (FROM_RAW) {
-          float r = 0.f;
+      for (int k = 0; k < 2; ++k) {
+        const int t0 = t00 + 4 * k * kCalThreads;
+        v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        mw[k] = make_uint4(0u, 0u, 0u, 0u);
+        if (t0 < Lp) {
 #pragma unroll
-          for (int c = 0; c < kRawCopies; ++c) r += raw[c * Lp + t];
-          v[k] = r;
-        } else {
-          v[k] = S[t];
+          for (int c = 0; c < kRawCopies; ++c) {   // copies added in order, as in the scalar path
+            const float4 q = *reinterpret_cast<const float4*>(raw + c * rs + t0);
+            v[k].x += q.x;
+            v[k].y += q.y;
+            v[k].z += q.z;
+            v[k].w += q.w;
+          }
+          if (meta16 && t0 + 3 < Lp) {
+            mw[k] = *reinterpret_cast<const uint4*>(meta + t0);
+          } else {
+            mw[k].x = meta[t0];
+            if (t0 + 1 < Lp) mw[k].y = meta[t0 + 1];
+            if (t0 + 2 < Lp) mw[k].z = meta[t0 + 2];
+            if (t0 + 3 < Lp) mw[k].w = meta[t0 + 3];
+          }
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 2; ++k) {
+        const int t0 = t00 + 4 * k * kCalThreads;
+        if (t0 < Lp) {   // the arrays hold capl >= Lp rounded up to 16 entries
+          reinterpret_cast<float4*>(stage)[t0 >> 2] = v[k];
+          reinterpret_cast<uint4*>(keys)[t0 >> 2] = mw[k];
         }
       }
     }
+  } else {
+    for (int t0 = 0; t0 < Lp; t0 += 4 * kCalThreads) {
+      float v[4];
+      uint32_t mw[4];
 #pragma unroll
-    for (int k = 0; k < 4; ++k) {
-      const int t = t0 + k * kCalThreads + tid;
-      if (t < Lp) {
-        stage[t] = v[k];
-        keys[t] = mw[k];
+      for (int k = 0; k < 4; ++k) {
+        const int t = t0 + k * kCalThreads + tid;
+        v[k] = 0.f;
+        mw[k] = 0u;
+        if (t < Lp) {
+          mw[k] = meta[t];
+          if (FROM_RAW) {
+            float r = 0.f;
+#pragma unroll
+            for (int c = 0; c < kRawCopies; ++c) r += raw[c * rs + t];
+            v[k] = r;
+          } else {
+            v[k] = S[t];
+          }
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int t = t0 + k * kCalThreads + tid;
+        if (t < Lp) {
+          stage[t] = v[k];
+          keys[t] = mw[k];
+        }
       }
     }
   }
@@ -429,17 +474,10 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     }
     return acc * pscale;
   };
-  for (int t = tid; t < Lp; t += kCalThreads) {
-    float s;
-    if (FROM_RAW) {
-      s = pooled(t);
-      S[t] = s;
-    } else {
-      s = stage[t];
-    }
-    const uint32_t mt = keys[t];
-    uint16_t cell = kNoCell;
-    uint32_t key = 0;
+  // key and cell of one token; the current frame's tokens go onto the grid
+  auto classify = [&](float s, uint32_t mt, uint32_t& key, uint16_t& cell) {
+    cell = kNoCell;
+    key = 0;
     if (meta_visual(mt)) {
       const int r = meta_row(mt), c = meta_col(mt);
       if (r < R && c < C) {
@@ -453,8 +491,54 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         atomicOr(st.err, kErrMeta);
       }
     }
-    keys[t] = key;
-    cells[t] = cell;
+  };
+  if (vec) {
+    const float4* st4 = reinterpret_cast<const float4*>(stage);
+    for (int t0 = 4 * tid; t0 < Lp; t0 += 4 * kCalThreads) {
+      float sv4[4];
+      if (half == 2 && t0 >= 4 && t0 + 8 <= Lp) {   // x[t0 - 4 .. t0 + 7] in three 16-byte loads
+        const float4 a = st4[(t0 >> 2) - 1], b = st4[t0 >> 2], c = st4[(t0 >> 2) + 1];
+        const float x[12] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w, c.x, c.y, c.z, c.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          sv4[k] = ((((x[k + 2] + x[k + 3]) + x[k + 4]) + x[k + 5]) + x[k + 6]) * pscale;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) sv4[k] = t0 + k < Lp ? pooled(t0 + k) : 0.f;
+      }
+      const uint4 m4 = reinterpret_cast<const uint4*>(keys)[t0 >> 2];
+      const uint32_t mts[4] = {m4.x, m4.y, m4.z, m4.w};
+      uint32_t ks[4];
+      uint16_t cs[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        ks[k] = 0u;
+        cs[k] = kNoCell;
+        if (t0 + k < Lp) {
+          S[t0 + k] = sv4[k];
+          classify(sv4[k], mts[k], ks[k], cs[k]);
+        }
+      }
+      reinterpret_cast<uint4*>(keys)[t0 >> 2] = make_uint4(ks[0], ks[1], ks[2], ks[3]);
+      reinterpret_cast<uint2*>(cells)[t0 >> 2] =
+          make_uint2(static_cast<uint32_t>(cs[0]) | (static_cast<uint32_t>(cs[1]) << 16),
+                     static_cast<uint32_t>(cs[2]) | (static_cast<uint32_t>(cs[3]) << 16));
+    }
+  } else {
+    for (int t = tid; t < Lp; t += kCalThreads) {
+      float s;
+      if (FROM_RAW) {
+        s = pooled(t);
+        S[t] = s;
+      } else {
+        s = stage[t];
+      }
+      uint32_t key;
+      uint16_t cell;
+      classify(s, keys[t], key, cell);
+      keys[t] = key;
+      cells[t] = cell;
+    }
   }
   int N;
   {
