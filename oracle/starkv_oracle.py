@@ -88,6 +88,43 @@ def head_group(h: int, n_heads: int, n_kv_heads: int) -> int:
 
 # ---------------------------------------------------------------- Sec. 3.3
 
+def window_lse(q: np.ndarray, k: np.ndarray, window: int) -> np.ndarray:
+    """Sec. 3.3, Eq. (2): the softmax normaliser of each window row, as the
+    natural-log log-sum-exp of z = Q_{-i,h} . K_past[g(h), t] / sqrt(d) over
+    the L_past past keys.  [H][w]; -inf when L_past = 0."""
+    H, w, d = q.shape
+    G, L, _ = k.shape
+    assert w == window
+    lp = L - w
+    out = np.full((H, w), -np.inf)
+    if lp == 0:
+        return out
+    for h in range(H):
+        g = head_group(h, H, G)
+        z = (q[h].astype(np.float64) @ k[g, :lp].astype(np.float64).T) / math.sqrt(d)
+        m = z.max(axis=1)
+        out[h] = m + np.log(np.exp(z - m[:, None]).sum(axis=1))
+    return out
+
+
+def window_attention_given_lse(q: np.ndarray, k: np.ndarray, window: int, lse: np.ndarray) -> np.ndarray:
+    """Eq. (2) with the softmax normaliser supplied (the log-sum-exp of each
+    window row over K_past, as the layer's own prefill attention pass produces
+    it): A_raw[h, t] = sum_i exp(z_{h,i,t} - lse[h, i])."""
+    H, w, d = q.shape
+    G, L, _ = k.shape
+    assert w == window
+    lp = L - w
+    a_raw = np.zeros((H, lp), np.float64)
+    if lp == 0:
+        return a_raw
+    for h in range(H):
+        g = head_group(h, H, G)
+        z = (q[h].astype(np.float64) @ k[g, :lp].astype(np.float64).T) / math.sqrt(d)
+        a_raw[h] = np.exp(z - lse[h][:, None]).sum(axis=0)
+    return a_raw
+
+
 def window_attention(q: np.ndarray, k: np.ndarray, window: int) -> np.ndarray:
     """Sec. 3.3, Eq. (2) / Algorithm 1 first step: A_raw[h, t] = sum over the w
     window queries of softmax_t(Q_{-i,h} . K_past[g(h), t] / sqrt(d)).
@@ -306,9 +343,11 @@ class LayerState:
         return LayerState(self.n, self.mi_bar.copy(), self.m.copy())
 
 
-def score_layer(q: np.ndarray, k: np.ndarray, window: int, p: Params) -> np.ndarray:
-    """Algorithm 1, first two steps: S = group-mean of Pool(sum_i softmax(Q_{-i} K^T / sqrt d))."""
-    a_raw = window_attention(q, k, window)
+def score_layer(q: np.ndarray, k: np.ndarray, window: int, p: Params,
+                lse: Optional[np.ndarray] = None) -> np.ndarray:
+    """Algorithm 1, first two steps: S = group-mean of Pool(sum_i softmax(Q_{-i} K^T / sqrt d)).
+    ``lse`` [H][w], when given, is the softmax normaliser of each window row."""
+    a_raw = window_attention(q, k, window) if lse is None else window_attention_given_lse(q, k, window, lse)
     a = avg_pool(a_raw, p.pool_kernel)
     return group_scores(a, k.shape[0])
 

@@ -509,3 +509,29 @@ def test_per_head_per_group_metadata_follows_each_groups_tokens():
         assert sorted(perms[g][o["idx"][g]].tolist()) == shared["idx"][g].tolist()
     np.testing.assert_allclose(o["mi"], shared["mi"], rtol=1e-12)
     np.testing.assert_allclose(o["phi"], shared["phi"], rtol=1e-12)
+
+
+# ------------------------------------------------------------------ normaliser supplied by the prefill pass
+
+def test_window_lse_vs_torch_logsumexp():
+    r = _rng(60)
+    H, G, w, L, d = 8, 2, 4, 50, 16
+    q = r.standard_normal((H, w, d)) * 3
+    k = r.standard_normal((G, L, d))
+    got = O.window_lse(q, k, w)
+    kk = torch.from_numpy(k[:, :L - w]).repeat_interleave(H // G, dim=0)
+    z = torch.einsum("hid,htd->hit", torch.from_numpy(q), kk) / math.sqrt(d)
+    np.testing.assert_allclose(got, torch.logsumexp(z, dim=-1).numpy(), rtol=1e-13, atol=1e-13)
+    assert np.all(O.window_lse(q, k[:, :w], w) == -np.inf)   # no past keys
+
+
+def test_attention_with_the_exact_normaliser_is_the_softmax_sum():
+    r = _rng(61)
+    q = r.standard_normal((6, 5, 16))
+    k = r.standard_normal((3, 40, 16))
+    lse = O.window_lse(q, k, 5)
+    np.testing.assert_allclose(O.window_attention_given_lse(q, k, 5, lse), O.window_attention(q, k, 5),
+                               rtol=1e-12, atol=1e-15)
+    # a normaliser larger by c scales every row's contribution by exp(-c)
+    shifted = O.window_attention_given_lse(q, k, 5, lse + 0.5)
+    np.testing.assert_allclose(shifted, O.window_attention(q, k, 5) * math.exp(-0.5), rtol=1e-12)
