@@ -254,6 +254,24 @@ def job_throughput(tokens_per_rank_step, world, steps, ms_max):
 
 # ----------------------------------------------------------------------------- GPU arm
 
+def window_lse_torch(si, wl, dev):
+    """[n_layers][H][w] natural-log log-sum-exp of each window row over the
+    past keys, in fp32 with torch (input preparation for --lse given)."""
+    import math
+    import torch
+    nl, H, G, w = si.k.shape[0], wl.n_heads, wl.n_kv_heads, wl.window
+    lp = si.L - w
+    out = torch.empty((nl, H, w), dtype=torch.float32, device=dev)
+    for l in range(nl):
+        q = si.q[l].to(dev).float()                      # [H][w][d]
+        k = si.k[l, :, :lp].to(dev).float()              # [G][lp][d]
+        for g in range(G):
+            hs = slice(g * (H // G), (g + 1) * (H // G))
+            z = torch.einsum("hid,td->hit", q[hs], k[g]) / math.sqrt(wl.head_dim)
+            out[l, hs] = torch.logsumexp(z, dim=-1)
+    return out
+
+
 def gpu_arm(args):
     import numpy as np
     import torch
@@ -299,6 +317,11 @@ def gpu_arm(args):
                       meta_out=alloc((nl, P, B + w), torch.int32), idx=alloc((nl, P, B), torch.int32))
 
     seqs = [make_seq(si, i, dev) for i, si in enumerate(sis)]
+    if args.lse == "given":
+        # the softmax normaliser of each window row over the past keys, as the
+        # layer's prefill attention pass supplies it (input preparation, torch)
+        for s_, si in zip(seqs, sis):
+            s_.lse = window_lse_torch(si, wl, dev)
     ws = sk.workspace(st, seqs, device=dev)
     stream = torch.cuda.current_stream(dev)
     work = work_per_step(wl, [dict(L=si.L, B=si.budget) for si in sis], per_head=P > 1)
@@ -370,10 +393,15 @@ def gpu_arm(args):
     e2e = None
     if not args.no_e2e:
         hseqs = [make_seq(si, i, None, pin=True) for i, si in enumerate(sis)]
+        if args.lse == "given":
+            for hs_, s_ in zip(hseqs, seqs):
+                hs_.lse = torch.empty(s_.lse.shape, dtype=torch.float32, pin_memory=True)
+                hs_.lse.copy_(s_.lse)
         hws = sk.workspace(st, hseqs, host=True, device=dev)
         # K, Q and metadata are uploaded; V is page-locked, so the gather reads
         # only its kept rows in place (the same bytes as V')
-        h2d = sum(s.k.numel() * 2 + s.v_out.numel() * 2 + s.q.numel() * 2 + s.meta.numel() * 4 for s in hseqs)
+        h2d = sum(s.k.numel() * 2 + s.v_out.numel() * 2 + s.q.numel() * 2 + s.meta.numel() * 4 +
+                  (s.lse.numel() * 4 if s.lse is not None else 0) for s in hseqs)
         d2h = sum(s.k_out.numel() * 2 + s.v_out.numel() * 2 + s.meta_out.numel() * 4 + s.idx.numel() * 4
                   for s in hseqs)
         for _ in range(2):
@@ -406,7 +434,9 @@ def gpu_arm(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": args.workload, "select_mode": args.select_mode, "layers": nl, "seqs_per_gpu": len(sis),
+            "config": {"workload": args.workload, "select_mode": args.select_mode,
+                       "lse": "supplied (prefill attention); first scoring pass skipped" if args.lse == "given"
+                       else "computed (both scoring passes)", "layers": nl, "seqs_per_gpu": len(sis),
                        "L": [si.L for si in sis], "w": w, "B": [si.budget for si in sis],
                        "H": wl.n_heads, "G": G, "d": d,
                        "l2": f"inputs {2 * sum(s.k.numel() for s in seqs) * 2 / 1e9:.2f} GB per step "
@@ -430,6 +460,9 @@ def main():
     ap.add_argument("--workload", default="uitars_5shot_28l")
     ap.add_argument("--select-mode", choices=["global", "per_head"], default="global",
                     help="global top-B per layer (the paper's) or one top-B per KV group")
+    ap.add_argument("--lse", choices=["computed", "given"], default="computed",
+                    help="given: the window rows' softmax normalisers are inputs (from the prefill "
+                         "attention pass), so the first scoring pass is skipped")
     ap.add_argument("--soak-s", type=float, default=2.0)
     ap.add_argument("--cpu-budget-s", type=float, default=15.0)
     ap.add_argument("--no-e2e", action="store_true")

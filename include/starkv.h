@@ -142,6 +142,15 @@ typedef struct {
                                    its own tokens after a compaction); with a
                                    nonzero meta_layer_stride it must be
                                    >= (G - 1) * meta_group_stride + L                */
+  const float* lse;             /* f32 [n_layers][H][w], optional: the softmax
+                                   normaliser of each window row (Eq. 2), as the
+                                   natural-log log-sum-exp over the past keys t < L_p
+                                   of z = Q_{-i,h} . K[g(h), t] / sqrt(d) (the window
+                                   keys excluded), e.g. from the layer's own prefill
+                                   attention pass, which computes these logits.  When
+                                   every sequence of a call gives it, the first
+                                   scoring pass (a whole read of K) is skipped.
+                                   NULL = computed.                                 */
 } starkv_seq;
 
 /* Per-layer diagnostics written to starkv_seq.stats (floats):
@@ -190,7 +199,8 @@ starkv_status starkv_workspace_bytes(const starkv_state* st, const starkv_seq* s
  * every sequence, writes S[g][t] = (G/H) * sum_{h in g} AvgPool1D(
  * sum_{i<w} softmax_t(Q_{-i,h} K_past[g]^T / sqrt(d)))[t]  for t < L_p,
  * softmax over K_past only.  Reads k, q; writes S.  Uses tcgen05 tensor cores
- * (bf16 in, fp32 accumulate) in two passes (log-sum-exp, then normalised sums). */
+ * (bf16 in, fp32 accumulate) in two passes (log-sum-exp, then normalised sums);
+ * the first is skipped when every sequence supplies `lse`. */
 starkv_status starkv_score_layer(starkv_state* st, int32_t layer, const starkv_seq* seqs,
                                  int32_t nseq, void* workspace, size_t workspace_bytes,
                                  void* stream);

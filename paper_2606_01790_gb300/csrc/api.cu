@@ -309,6 +309,7 @@ starkv_status run_score(starkv_state* st, const starkv_seq* seqs, int i0, int i1
   if (p.kstages < 2) return set_error(STARKV_ERR_UNSUPPORTED, "window rows per group too large for shared memory");
   p.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(kHeadDim)));
   int64_t tiles = 0;
+  bool need_lse = false;   // the first pass runs unless every sequence supplies its normalisers
   for (int i = i0; i < i1; ++i) {
     const starkv_seq& q = seqs[i];
     const int lp = q.L - w;
@@ -317,6 +318,8 @@ starkv_status run_score(starkv_state* st, const starkv_seq* seqs, int i0, int i1
     ss.nt = tiles_of(lp);
     ss.tile_base = tiles;
     ss.s_raw = reinterpret_cast<float*>(ws + plan.raw_off[i]);
+    ss.lse = q.lse;
+    if (!q.lse && ss.nt > 0) need_lse = true;
     tiles += static_cast<int64_t>(nlayers) * G * ss.nt;
     if (ss.nt == 0) continue;
     if ((s = encode_3d(&p.tmk[i - i0], q.k, kHeadDim, q.L, static_cast<uint64_t>(c.n_layers) * G, kTileKeys)) != STARKV_OK) return s;
@@ -335,7 +338,8 @@ starkv_status run_score(starkv_state* st, const starkv_seq* seqs, int i0, int i1
   *partial_cursor += tiles;
   p.err = st->dev.err;
   p.wait_ns = st->wait_ns;
-  CUDA_TRY(launch(st, STARKV_KERNEL_SCORE_LSE, stream, [&] { return score_lse_launch(p, p.grid1, stream); }));
+  if (need_lse)
+    CUDA_TRY(launch(st, STARKV_KERNEL_SCORE_LSE, stream, [&] { return score_lse_launch(p, p.grid1, stream); }));
   CUDA_TRY(launch(st, STARKV_KERNEL_SCORE_ACCUM, stream, [&] { return score_accum_launch(p, p.grid1, stream); }));
   return STARKV_OK;
 }
@@ -420,7 +424,8 @@ size_t seq_bytes_in(const starkv_config& c, const starkv_seq& s) {
   const size_t kv = static_cast<size_t>(c.n_layers) * c.n_kv_heads * s.L * kHeadDim * 2;
   const size_t q = static_cast<size_t>(c.n_layers) * c.n_heads * c.window * kHeadDim * 2;
   const size_t meta = meta_elems(c, s, c.n_layers) * 4;
-  return align256(kv) * 2 + align256(q) + align256(meta);
+  const size_t lse = s.lse ? align256(static_cast<size_t>(c.n_layers) * c.n_heads * c.window * 4) : 0;
+  return align256(kv) * 2 + align256(q) + align256(meta) + lse;
 }
 
 size_t seq_bytes_out(const starkv_config& c, const starkv_seq& s) {
@@ -653,7 +658,7 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
     cur += align256(bytes);
     return p;
   };
-  struct Rows { size_t kv_layer, q_layer, meta_layer, out_layer, sel_layer, meta_out_layer, lp; bool v_in_place; };
+  struct Rows { size_t kv_layer, q_layer, lse_layer, meta_layer, out_layer, sel_layer, meta_out_layer, lp; bool v_in_place; };
   const size_t P = sel_rows(c);
   std::vector<starkv_seq> dev(seqs, seqs + nseq);
   std::vector<Rows> rows(nseq);
@@ -663,6 +668,7 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
     Rows& r = rows[i];
     r.kv_layer = static_cast<size_t>(G) * h.L * kHeadDim * 2;
     r.q_layer = static_cast<size_t>(c.n_heads) * c.window * kHeadDim * 2;
+    r.lse_layer = static_cast<size_t>(c.n_heads) * c.window * 4;
     r.meta_layer = static_cast<size_t>(h.meta_layer_stride) * 4;
     r.lp = static_cast<size_t>(h.L - c.window);
     r.out_layer = static_cast<size_t>(h.budget + c.window);
@@ -686,6 +692,7 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
     d.S = h.S ? reinterpret_cast<float*>(take(NL * static_cast<size_t>(G) * r.lp * 4)) : nullptr;
     d.score = h.score ? reinterpret_cast<float*>(take(NL * P * r.lp * 4)) : nullptr;
     d.stats = h.stats ? reinterpret_cast<float*>(take(static_cast<size_t>(NL) * stats_bytes(c))) : nullptr;
+    d.lse = h.lse ? reinterpret_cast<const float*>(take(NL * r.lse_layer)) : nullptr;
   }
   const size_t used = static_cast<size_t>(cur - static_cast<char*>(workspace));
   // the uploads may start once earlier work on the caller's stream (which may
@@ -709,6 +716,7 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
       CUDA_TRY(h2d(d.k, h.k, l0 * r.kv_layer, nl * r.kv_layer));
       if (!r.v_in_place) CUDA_TRY(h2d(d.v, h.v, l0 * r.kv_layer, nl * r.kv_layer));
       CUDA_TRY(h2d(d.q, h.q, l0 * r.q_layer, nl * r.q_layer));
+      if (h.lse) CUDA_TRY(h2d(d.lse, h.lse, l0 * r.lse_layer, nl * r.lse_layer));
       if (h.meta_layer_stride) CUDA_TRY(h2d(d.meta, h.meta, l0 * r.meta_layer, nl * r.meta_layer));
       else if (k == 0) CUDA_TRY(h2d(d.meta, h.meta, 0, meta_elems(c, h, NL) * 4));
     }

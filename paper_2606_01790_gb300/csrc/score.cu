@@ -566,15 +566,20 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
     const int ch0 = wg * (nc >> 2) + min(wg, nc & 3);
     const int nch = (nc >> 2) + (wg < (nc & 3) ? 1 : 0);
     const uint32_t base0 = tmem + (static_cast<uint32_t>(quad * 32) << 16) + ch0 * 16;
-    const float sc = p.scale2, isc = 1.f / p.scale2;
-    // the -lse operand of the piece whose row starts at flat tile r0, into
-    // buffer `buf`: window row et holds x = -lse2 / scale as three bf16 parts
-    // (x = hi + mid + lo to about 2^-24 relative) in its K columns 0..2;
-    // rows past the group's window rows get a large negative x (exp2 -> 0)
-    auto write_x = [&](int64_t r0, int nt, int buf) {
+    const float sc = p.scale2, isc = 1.f / p.scale2, sqd = sqrtf(static_cast<float>(kHeadDim));
+    // the -lse operand of the piece `it` (whose row starts at flat tile r0),
+    // into buffer `buf`: window row et holds x = -lse2 / scale (= -lse sqrt(d)
+    // for a supplied natural-log normaliser) as three bf16 parts (x = hi + mid
+    // + lo to about 2^-24 relative) in its K columns 0..2; rows past the
+    // group's window rows get a large negative x (exp2 -> 0)
+    auto write_x = [&](const TileIter& it, int64_t r0, int buf) {
       if (et < p.n2) {
         float x = -3.0e38f;
-        if (et < p.rows) x = -combine_lse2(p, r0, nt, et) * isc;
+        if (et < p.rows) {
+          const float* lse = p.seq[it.s].lse;
+          x = lse ? -lse[(static_cast<int64_t>(p.layer0 + it.l) * p.G + it.g) * p.rows + et] * sqd
+                  : -combine_lse2(p, r0, it.nt, et) * isc;
+        }
         const __nv_bfloat16 hi = __float2bfloat16_rn(x);
         const float r1 = x - __bfloat162float(hi);
         const __nv_bfloat16 mid = __float2bfloat16_rn(r1);
@@ -601,7 +606,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
         *reinterpret_cast<uint4*>(sX + et * 16) =
             et < 8 ? make_uint4(0x3F803F80u, 0x00003F80u, 0u, 0u) : make_uint4(0u, 0u, 0u, 0u);
       }
-      write_x(c.f - c.j, c.nt, 0);
+      write_x(c, c.f - c.j, 0);
     }
     const float2 sc2 = make_float2(sc, sc), zero2 = make_float2(0.f, 0.f);
     for (; c.valid(); c.next(p)) {
@@ -613,7 +618,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
         if (fn < fe) {
           TileIter n;
           n.init(p, fn, fe);
-          write_x(fn, n.nt, (kp + 1) & 1);
+          write_x(n, fn, (kp + 1) & 1);
         }
         ++kp;
         const ScoreSeq& sq = p.seq[c.s];

@@ -11,7 +11,8 @@ struct ScoreSeq {
   int Lp;              // scored (historical) keys
   int nt;              // ceil(Lp / 128) key tiles per (layer, group) row
   int64_t tile_base;   // flat index of this sequence's first tile in the launch
-  float* s_raw;        // [nlayers][G][kRawCopies][Lp] unpooled group sums, one copy per column quarter
+  float* s_raw;        // [nlayers][G][kRawCopies][raw_stride(Lp)] unpooled group sums, one copy per column quarter
+  const float* lse;    // [n_layers][H][w] supplied row normalisers (natural log) or NULL
 };
 
 struct ScoreParams {

@@ -55,7 +55,7 @@ class CSeq(C.Structure):
                 ("budget", C.c_int32), ("slot", C.c_int32), ("k_out", C.c_void_p),
                 ("v_out", C.c_void_p), ("meta_out", C.c_void_p), ("idx", C.c_void_p),
                 ("S", C.c_void_p), ("score", C.c_void_p), ("stats", C.c_void_p),
-                ("meta_group_stride", C.c_int64)]
+                ("meta_group_stride", C.c_int64), ("lse", C.c_void_p)]
 
 
 _lib: Optional[C.CDLL] = None
@@ -206,10 +206,11 @@ class Seq:
     score: Optional[torch.Tensor] = None
     stats: Optional[torch.Tensor] = None
     meta_group_stride: int = 0              # per-KV-head mode: one metadata row per group
+    lse: Optional[torch.Tensor] = None      # f32 [n_layers][H][w] supplied row normalisers
 
     def to_c(self) -> CSeq:
         s = CSeq()
-        for name in ("k", "v", "q", "meta", "k_out", "v_out", "meta_out", "idx", "S", "score", "stats"):
+        for name in ("k", "v", "q", "meta", "k_out", "v_out", "meta_out", "idx", "S", "score", "stats", "lse"):
             setattr(s, name, _ptr(getattr(self, name)))
         s.meta_layer_stride = self.meta_layer_stride
         s.meta_group_stride = self.meta_group_stride
