@@ -31,6 +31,14 @@ parameter with the stated default):
   with no visual tokens: phi_g = 0 and m_g unchanged.
 * Top-B (Sec. 3.7, Algorithm 1 "Sort(TopK)"): one global token-level set per
   layer, ties to the lower index, returned ascending.
+* Method variants of the ablations (Table 3 and the AEB ablation), off by
+  default; the paper names them but prints no formula, so each is a reading:
+  decay_mode 1 "linear": D = D_min + (1 - D_min) max(0, 1 - delta Df phi);
+  decay_mode 2 "gamma" (power law): D = D_min + (1 - D_min) (1 + Df phi)^(-delta)
+  (at the defaults it keeps more of old frames than Eq. 9, linear less, as the
+  ablation describes them); aeb_mode 1 "confidence": T = T_min + (T_max -
+  T_min)(1 - p_max) with p_max = max_t p_t, the peak attention mass;
+  mi_span 1: the MI of Sec. 3.4 over the newest frame's visual tokens only.
 * Per-KV-head selection (an optional mode; the paper's method is the global
   set above; App. A.3 names head-wise top-K as the SnapKV-style alternative):
   each group g ranks its own row s_{g,t} = max(S[g,t] beta_g D_{g,t}, 0)^(1/T_g)
@@ -75,6 +83,9 @@ class Params:
     mi_grid: int = 8          # M, reading
     eps: float = 1e-6         # epsilon of the min-max prior, reading
     eps_h: float = 1e-12      # epsilon of the AEB entropy, reading
+    decay_mode: int = 0       # 0 exponential (Eq. 9), 1 linear, 2 power law (readings)
+    aeb_mode: int = 0         # 0 entropy (Sec. 3.6), 1 peak confidence (reading)
+    mi_span: int = 0          # 0 every historical visual token, 1 the newest frame's
 
 
 # ---------------------------------------------------------------- Sec. 3.1
@@ -201,6 +212,23 @@ def entropy_temperature(sbar: np.ndarray, t_min: float, t_max: float,
 
 # ---------------------------------------------------------------- Sec. 3.4
 
+def confidence_temperature(sbar: np.ndarray, t_min: float, t_max: float, eps_h: float) -> tuple:
+    """The AEB ablation's confidence variant (reading): p_t = s_bar_t /
+    (sum s_bar + eps), p_max = max_t p_t, T = T_min + (T_max - T_min)(1 - p_max).
+    Returns (p_max, T); no tokens gives p_max = 0."""
+    if sbar.shape[0] == 0:
+        return 0.0, t_max
+    pmax = float(sbar.max() / (sbar.sum() + eps_h))
+    return pmax, t_min + (t_max - t_min) * (1.0 - pmax)
+
+
+def layer_temperature(s: np.ndarray, p: "Params") -> tuple:
+    """(H or p_max, T) of one score row by the configured AEB mode."""
+    if p.aeb_mode == 1:
+        return confidence_temperature(s, p.t_min, p.t_max, p.eps_h)
+    return entropy_temperature(s, p.t_min, p.t_max, p.eps_h)
+
+
 def rank_bins(values: np.ndarray, n_bins: int) -> np.ndarray:
     """Sec. 3.4 RankBin: K equal-frequency bins of the values; ties in value
     broken by position; bin(rho) = floor(rho K / N)."""
@@ -290,11 +318,19 @@ def temporal_stability(cur: np.ndarray, m: np.ndarray, rho_t: float) -> tuple:
 
 
 def temporal_decay(is_visual: np.ndarray, frame: np.ndarray, cur_frame: int,
-                   phi_gstar: np.ndarray, delta: float, d_min: float) -> np.ndarray:
+                   phi_gstar: np.ndarray, delta: float, d_min: float, mode: int = 0) -> np.ndarray:
     """Sec. 3.5, Eq. (9): D_t = D_min + (1 - D_min) exp(-delta Delta_f(t) phi_{g*(t)})
-    for visual t with Delta_f = F - f(t); D_t = 1 for non-visual tokens."""
+    for visual t with Delta_f = F - f(t); D_t = 1 for non-visual tokens.
+    mode 1 / 2: the linear and power-law readings of Table 3's variants."""
     dist = (cur_frame - frame).astype(np.float64)
-    d = d_min + (1.0 - d_min) * np.exp(-delta * dist * phi_gstar)
+    x = dist * phi_gstar
+    if mode == 1:
+        shape = np.maximum(0.0, 1.0 - delta * x)
+    elif mode == 2:
+        shape = (1.0 + x) ** (-delta)
+    else:
+        shape = np.exp(-delta * x)
+    d = d_min + (1.0 - d_min) * shape
     return np.where(is_visual != 0, d, 1.0)
 
 
@@ -374,6 +410,8 @@ def calibrate_layer(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarray, row
     for g in range(G):
         vis_g, fr_g, row_g, col_g = (_group_meta(a, g)[:lp] for a in (is_visual, frame, row, col))
         vis = vis_g != 0
+        if p.mi_span == 1:   # the newest frame's visual tokens only
+            vis = vis & (fr_g == cur_frame)
         cells = spatial_cells(row_g[vis], col_g[vis], R, C, p.mi_grid)
         mi[g] = mutual_information(rank_bins(s[g][vis], p.mi_bins), cells, p.mi_bins, n_cells)
         cur = current_row(s[g], vis_g, fr_g, row_g, col_g, cur_frame, R, C)
@@ -405,9 +443,10 @@ def select_layer(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarray, row: n
     # online MI prior (Sec. 3.4)
     beta = mi_weight(gstar, cal["w"], cal["lam"])
     # temporal discount (Sec. 3.5)
-    d = temporal_decay(is_visual[:lp], frame[:lp], cur_frame, cal["phi"][gstar], p.delta, p.d_min)
+    d = temporal_decay(is_visual[:lp], frame[:lp], cur_frame, cal["phi"][gstar], p.delta, p.d_min,
+                       p.decay_mode)
     # entropy temperature (Sec. 3.6) and fused score
-    h, temp = entropy_temperature(sbar, p.t_min, p.t_max, p.eps_h)
+    h, temp = layer_temperature(sbar, p)
     score = final_score(sbar, beta, d, temp)
     idx = top_b(score, budget)
     _advance(st, cal)
@@ -427,9 +466,9 @@ def select_layer_per_head(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarra
     own = np.arange(G)
     beta = mi_weight(own, cal["w"], cal["lam"])                       # [G]
     d = np.stack([temporal_decay(_group_meta(is_visual, g)[:lp], _group_meta(frame, g)[:lp], cur_frame,
-                                 np.full(lp, cal["phi"][g]), p.delta, p.d_min)
+                                 np.full(lp, cal["phi"][g]), p.delta, p.d_min, p.decay_mode)
                   for g in range(G)])                                  # [G][L_past]
-    ht = [entropy_temperature(s[g], p.t_min, p.t_max, p.eps_h) for g in range(G)]
+    ht = [layer_temperature(s[g], p) for g in range(G)]
     h = np.array([x[0] for x in ht])
     temp = np.array([x[1] for x in ht])
     score = np.stack([final_score(s[g], beta[g], d[g], temp[g]) for g in range(G)])

@@ -535,3 +535,65 @@ def test_attention_with_the_exact_normaliser_is_the_softmax_sum():
     # a normaliser larger by c scales every row's contribution by exp(-c)
     shifted = O.window_attention_given_lse(q, k, 5, lse + 0.5)
     np.testing.assert_allclose(shifted, O.window_attention(q, k, 5) * math.exp(-0.5), rtol=1e-12)
+
+
+# ------------------------------------------------------------------ ablation variants (readings)
+
+def test_decay_variants_limits_and_ordering():
+    """All three shapes give D = 1 at Delta_f phi = 0 and for text tokens; the
+    linear one reaches D_min at delta Delta_f phi = 1 and stays there; at the
+    defaults linear < exponential < power law for old frames (the order in
+    which the ablation says they keep history); each decreases with age."""
+    dist = np.arange(0, 12)
+    vis = np.ones_like(dist)
+    cur = 11
+    frame = cur - dist
+    phi = np.full(dist.shape, 0.8)
+    ds = [O.temporal_decay(vis, frame, cur, phi, 0.2, 0.1, m) for m in (0, 1, 2)]
+    for d in ds:
+        assert d[0] == 1.0 and np.all(np.diff(d) <= 0)
+        np.testing.assert_array_equal(O.temporal_decay(vis * 0, frame, cur, phi, 0.2, 0.1), 1.0)
+        np.testing.assert_array_equal(O.temporal_decay(vis, frame, cur, phi * 0, 0.2, 0.1), 1.0)
+    lin = ds[1]
+    floor = dist * 0.8 * 0.2 >= 1.0
+    assert floor.any() and np.all(lin[floor] == 0.1) and np.all(lin[~floor] > 0.1)
+    old = dist >= 2
+    assert np.all(ds[1][old] < ds[0][old]) and np.all(ds[0][old] < ds[2][old])
+
+
+def test_confidence_temperature_closed_forms_and_rank_preservation():
+    L = 50
+    pm, t = O.confidence_temperature(np.full(L, 0.3), 0.75, 1.25, 1e-12)
+    assert abs(pm - 1 / L) < 1e-12 and abs(t - (0.75 + 0.5 * (1 - 1 / L))) < 1e-12
+    pm, t = O.confidence_temperature(np.eye(L)[3] * 2.0, 0.75, 1.25, 1e-12)
+    assert abs(pm - 1.0) < 1e-12 and abs(t - 0.75) < 1e-12
+    q, k, meta, F_ = _small_case(62)
+    sets = []
+    for mode in (0, 1):
+        p = O.Params(aeb_mode=mode, n_warmup=0, n_ramp=0, t_min=0.5, t_max=2.0)
+        o = O.select_layer(O.score_layer(q, k, q.shape[1], p), *meta, F_, 17, 4, 5,
+                           O.LayerState.fresh(k.shape[0], 4, 5), p)
+        sets.append(o["idx"].tolist())
+    assert sets[0] == sets[1]
+
+
+def test_mi_over_the_newest_frame_vs_sklearn():
+    """mi_span = 1: MI_g from the newest frame's visual tokens alone, checked
+    against scikit-learn's mutual_info_score on that subset (scipy ordinal ranks
+    for the rank bins)."""
+    metrics = pytest.importorskip("sklearn.metrics")
+    q, k, meta, F_ = _small_case(63, G=2, shots=3, n_text=20)
+    is_vis, frame, row, col = meta
+    p = O.Params(mi_span=1, n_warmup=0, n_ramp=0, pool_kernel=1, mi_bins=4, mi_grid=2)
+    s = O.score_layer(q, k, q.shape[1], p)
+    lp = s.shape[1]
+    o = O.select_layer(s, *meta, F_, 9, 4, 5, O.LayerState.fresh(2, 4, 5), p)
+    sel = (is_vis[:lp] != 0) & (frame[:lp] == F_)
+    cells = (row[:lp][sel] * 2 // 4) * 2 + (col[:lp][sel] * 2 // 5)
+    for g in range(2):
+        v = s[g][sel]
+        bins = (scipy.stats.rankdata(v, method="ordinal").astype(np.int64) - 1) * 4 // v.size
+        assert abs(o["mi"][g] - metrics.mutual_info_score(bins, cells)) < 1e-12
+    full = O.select_layer(s, *meta, F_, 9, 4, 5, O.LayerState.fresh(2, 4, 5),
+                          O.Params(n_warmup=0, n_ramp=0, pool_kernel=1, mi_bins=4, mi_grid=2))
+    assert not np.allclose(full["mi"], o["mi"])   # the span matters
