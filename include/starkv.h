@@ -109,6 +109,18 @@ typedef struct {
   float eps_h;          /* epsilon of the AEB entropy (Algorithm 1)                */
   int32_t select_mode;  /* STARKV_SELECT_GLOBAL (the paper's, default) or
                            STARKV_SELECT_PER_HEAD (one top-B set per KV group)     */
+  /* Variants of the paper's ablations (Table 3, the AEB ablation), 0 = the
+   * method as defined.  The paper names them without a formula; this
+   * library's readings, with x = Delta_f phi:
+   *   decay_mode 1 (linear):    D = D_min + (1 - D_min) max(0, 1 - delta x)
+   *   decay_mode 2 (power law): D = D_min + (1 - D_min) (1 + x)^(-delta)
+   *   aeb_mode 1 (confidence):  T = T_min + (T_max - T_min)(1 - p_max), with
+   *                             p_max = max_t s_bar_t / (sum_t s_bar_t + eps_h)
+   *   mi_span 1:                the MI of Sec. 3.4 over the newest frame's
+   *                             visual tokens only                              */
+  int32_t decay_mode;
+  int32_t aeb_mode;
+  int32_t mi_span;
 } starkv_config;
 
 /* Values of starkv_config.select_mode. */
@@ -154,7 +166,7 @@ typedef struct {
 } starkv_seq;
 
 /* Per-layer diagnostics written to starkv_seq.stats (floats):
- *   [0] H_hat  [1] T  [2] lambda_n  [3] n (steps seen before this one)
+ *   [0] H_hat (p_max with aeb_mode 1)  [1] T  [2] lambda_n  [3] n (steps seen before this one)
  *   [4] sum_t s_bar_t  [5] visual tokens in L_p  [6] kept count  [7] 0
  *   [8 + g]       MI_g of this step            (Eq. 5)
  *   [8 + G + g]   MI_bar_g after the EMA       (Eq. 6)

@@ -144,6 +144,8 @@ starkv_status validate_config(const starkv_config& c) {
   if (c.n_warmup < 0 || c.n_ramp < 0) return set_error(STARKV_ERR_INVALID_ARG, "config: negative schedule");
   if (!(c.t_min > 0.f) || !(c.t_max > 0.f) || !(c.tau > 0.f))
     return set_error(STARKV_ERR_INVALID_ARG, "config: t_min, t_max and tau must be > 0");
+  if (c.decay_mode < 0 || c.decay_mode > 2 || c.aeb_mode < 0 || c.aeb_mode > 1 || c.mi_span < 0 || c.mi_span > 1)
+    return set_error(STARKV_ERR_INVALID_ARG, "config: decay_mode in 0..2, aeb_mode and mi_span in 0..1");
   if (c.select_mode != STARKV_SELECT_GLOBAL && c.select_mode != STARKV_SELECT_PER_HEAD)
     return set_error(STARKV_ERR_INVALID_ARG, "config: select_mode must be 0 (global) or 1 (per KV head)");
   if (!(c.rho_mi >= 0.f && c.rho_mi <= 1.f) || !(c.rho_t >= 0.f && c.rho_t <= 1.f) ||
@@ -207,6 +209,9 @@ KParams make_kparams(const starkv_state* st) {
   k.lambda = c.lambda; k.tau = c.tau; k.rho_mi = c.rho_mi; k.rho_t = c.rho_t; k.delta = c.delta;
   k.d_min = c.d_min; k.t_min = c.t_min; k.t_max = c.t_max; k.eps = c.eps; k.eps_h = c.eps_h;
   k.per_head = c.select_mode == STARKV_SELECT_PER_HEAD;
+  k.decay_mode = c.decay_mode;
+  k.aeb_mode = c.aeb_mode;
+  k.mi_span = c.mi_span;
   k.wait_ns = st->wait_ns;
   return k;
 }

@@ -46,6 +46,9 @@ struct KParams {
   int n_layers, H, G, w, R, C, pool, K, M, n_warmup, n_ramp;
   float lambda, tau, rho_mi, rho_t, delta, d_min, t_min, t_max, eps, eps_h;
   int per_head;        // selection mode: 0 = one global top-B per layer, 1 = one per KV group
+  int decay_mode;      // 0 exponential (Eq. 9), 1 linear, 2 power law
+  int aeb_mode;        // 0 entropy (Sec. 3.6), 1 peak confidence
+  int mi_span;         // 0 every historical visual token, 1 the newest frame's
   uint64_t wait_ns;    // bounded-wait limit
 };
 

@@ -163,15 +163,15 @@ struct CalShared {
   int n_old;
   int any_tie;
   float fredn[4][32];             // multi-value block reductions
-  uint32_t uredn[2][32];
+  uint32_t uredn[3][32];
   float mic[kMaxGroups];          // every group's MI_g (phase 2)
   float pz[kMaxGroups], pzl[kMaxGroups], pv[kMaxGroups];   // every CTA's phase-2 partials
-  uint32_t pkmin[kMaxGroups], pkmax[kMaxGroups];
+  uint32_t pkmin[kMaxGroups], pkmax[kMaxGroups], psmax[kMaxGroups];
   int pncand[kMaxGroups], pbelow[kMaxGroups];
   // read by the other CTAs of the cluster
   float mi, phi;                  // this CTA's group (phase 1)
   float zpart, hpart, vpart;      // this CTA's token range (phase 2)
-  uint32_t kminp, kmaxp;
+  uint32_t kminp, kmaxp, smaxp;
   int tcand, nbelow;              // top-B boundary-bucket candidates, tokens below it
   int nlt, neq;
   // top-B select
@@ -183,24 +183,27 @@ struct CalShared {
 // Sums of NF floats, the minimum of `mn` and the maximum of `mx` over the
 // 1024 threads with one pair of barriers; every thread gets the results.
 template <int NF>
-__device__ void block_reduce(float (&v)[NF], uint32_t& mn, uint32_t& mx, CalShared& sh) {
+__device__ void block_reduce(float (&v)[NF], uint32_t& mn, uint32_t& mx, CalShared& sh, uint32_t* mx2 = nullptr) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
 #pragma unroll
   for (int k = 0; k < NF; ++k) v[k] = warp_sum(v[k]);
   mn = __reduce_min_sync(kFullMask, mn);
   mx = __reduce_max_sync(kFullMask, mx);
+  if (mx2) *mx2 = __reduce_max_sync(kFullMask, *mx2);
   __syncthreads();
   if (lane == 0) {
 #pragma unroll
     for (int k = 0; k < NF; ++k) sh.fredn[k][warp] = v[k];
     sh.uredn[0][warp] = mn;
     sh.uredn[1][warp] = mx;
+    if (mx2) sh.uredn[2][warp] = *mx2;
   }
   __syncthreads();
 #pragma unroll
   for (int k = 0; k < NF; ++k) v[k] = warp_sum(sh.fredn[k][lane]);
   mn = __reduce_min_sync(kFullMask, sh.uredn[0][lane]);
   mx = __reduce_max_sync(kFullMask, sh.uredn[1][lane]);
+  if (mx2) *mx2 = __reduce_max_sync(kFullMask, sh.uredn[2][lane]);
 }
 
 // Sum of the int4 at `p` over the CTAs [r_lo, r_hi) of the cluster: every
@@ -481,12 +484,15 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     if (meta_visual(mt)) {
       const int r = meta_row(mt), c = meta_col(mt);
       if (r < R && c < C) {
-        key = order_key(s);
-        cell = static_cast<uint16_t>(rowc[r] * M + colc[c]);
-        ++nv;
-        kmin = min(kmin, key);
-        kmax = max(kmax, key);
-        if (meta_frame(mt) == sv.cur_frame) atomicAdd(&cur[r * C + c], s);
+        const bool newest = meta_frame(mt) == sv.cur_frame;
+        if (newest) atomicAdd(&cur[r * C + c], s);
+        if (kp.mi_span == 0 || newest) {   // a token of the MI span (Sec. 3.4)
+          key = order_key(s);
+          cell = static_cast<uint16_t>(rowc[r] * M + colc[c]);
+          ++nv;
+          kmin = min(kmin, key);
+          kmax = max(kmax, key);
+        }
       } else {
         atomicOr(st.err, kErrMeta);
       }
@@ -802,15 +808,21 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   float* xs = reinterpret_cast<float*>(cand);   // [nr]
   float z = 0.f, zl = 0.f, nvf = 0.f;
   uint32_t kmn = 0xFFFFFFFFu, kmx = 0u;
+  uint32_t smx = 0u;   // the largest s (non-negative: its bits order like the values)
   auto fuse = [&](int i, float sb, int gs, uint32_t mt) {
     z += sb;
+    smx = max(smx, __float_as_uint(fmaxf(sb, 0.f)));
     if (sb > 0.f) zl += sb * lg2_approx(sb);
     const float beta = (1.f - lam) + lam * static_cast<float>(G) * sh.w[gs];
     float d = 1.f;
     if (meta_visual(mt)) {
       nvf += 1.f;
       const float df = static_cast<float>(sv.cur_frame - meta_frame(mt));
-      d = kp.d_min + (1.f - kp.d_min) * expf(-kp.delta * df * sh.ph[gs]);
+      float shape;
+      if (kp.decay_mode == 1) shape = fmaxf(0.f, 1.f - kp.delta * (df * sh.ph[gs]));
+      else if (kp.decay_mode == 2) shape = powf(1.f + df * sh.ph[gs], -kp.delta);
+      else shape = expf(-kp.delta * df * sh.ph[gs]);
+      d = kp.d_min + (1.f - kp.d_min) * shape;
     }
     const float x = fmaxf(sb * beta * d, 0.f);
     const uint32_t key = ~order_key(x);   // descending score = ascending key
@@ -880,7 +892,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   }
   {
     float r3[3] = {z, zl, nvf};
-    block_reduce<3>(r3, kmn, kmx, sh);
+    block_reduce<3>(r3, kmn, kmx, sh, &smx);
     z = r3[0];
     zl = r3[1];
     nvf = r3[2];
@@ -891,6 +903,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     sh.vpart = nvf;
     sh.kminp = kmn;
     sh.kmaxp = kmx;
+    sh.smaxp = smx;
   }
   cluster_sync();
   if (tid < G) {   // every CTA's partials, one peer per thread
@@ -899,23 +912,31 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     sh.pv[tid] = dsmem_ld_f32(dsmem_map(&sh.vpart, tid));
     sh.pkmin[tid] = static_cast<uint32_t>(dsmem_ld_s32(dsmem_map(&sh.kminp, tid)));
     sh.pkmax[tid] = static_cast<uint32_t>(dsmem_ld_s32(dsmem_map(&sh.kmaxp, tid)));
+    sh.psmax[tid] = static_cast<uint32_t>(dsmem_ld_s32(dsmem_map(&sh.smaxp, tid)));
   }
   __syncthreads();
-  auto entropy = [&](float Zr, float ZL2r) {   // ZL2r = sum s log2 s
+  // the AEB signal of a row from its sums: the normalised entropy (Sec. 3.6)
+  // or, with aeb_mode 1, the peak mass p_max = max s / (sum s + eps); T grows
+  // with the entropy and falls with the peak mass
+  auto entropy = [&](float Zr, float ZL2r, uint32_t smaxr) {   // ZL2r = sum s log2 s
     const float Ze = Zr + kp.eps_h;
+    if (kp.aeb_mode == 1) return __uint_as_float(smaxr) / Ze;
     const float plogp = Zr > 0.f ? kLn2 * ZL2r / Ze - (Zr / Ze) * logf(Ze) : 0.f;
     return Lp > 1 ? -plogp / logf(static_cast<float>(Lp)) : 0.f;
+  };
+  auto temperature = [&](float sig) {
+    return kp.t_min + (kp.t_max - kp.t_min) * (kp.aeb_mode == 1 ? 1.f - sig : sig);
   };
   float Hn, T;
   uint32_t kmin2 = kmn, kmax2 = kmx;   // key range of the selection
   if (per_head) {
-    Hn = entropy(z, zl);   // this CTA's own row
-    T = kp.t_min + (kp.t_max - kp.t_min) * Hn;
+    Hn = entropy(z, zl, smx);   // this CTA's own row
+    T = temperature(Hn);
     if (tid == 0 && g == 0 && stats) {
       float hs = 0.f, ts = 0.f, zs = 0.f;
       for (int r = 0; r < G; ++r) {
-        const float Hr = entropy(sh.pz[r], sh.pzl[r]);
-        const float Tr = kp.t_min + (kp.t_max - kp.t_min) * Hr;
+        const float Hr = entropy(sh.pz[r], sh.pzl[r], sh.psmax[r]);
+        const float Tr = temperature(Hr);
         stats[8 + 4 * G + r] = Hr;
         stats[8 + 5 * G + r] = Tr;
         hs += Hr;
@@ -929,17 +950,19 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     }
   } else {
     float Z = 0.f, ZL = 0.f, NV = 0.f;
+    uint32_t SM = 0u;
     kmin2 = 0xFFFFFFFFu;
     kmax2 = 0u;
     for (int r = 0; r < G; ++r) {
       Z += sh.pz[r];
       ZL += sh.pzl[r];
       NV += sh.pv[r];
+      SM = max(SM, sh.psmax[r]);
       kmin2 = min(kmin2, sh.pkmin[r]);
       kmax2 = max(kmax2, sh.pkmax[r]);
     }
-    Hn = entropy(Z, ZL);
-    T = kp.t_min + (kp.t_max - kp.t_min) * Hn;
+    Hn = entropy(Z, ZL, SM);
+    T = temperature(Hn);
     if (tid == 0 && g == 0 && stats) {
       stats[0] = Hn;
       stats[1] = T;

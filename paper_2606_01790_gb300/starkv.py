@@ -46,7 +46,7 @@ class CConfig(C.Structure):
         "pool_kernel", "mi_bins", "mi_grid", "n_warmup", "n_ramp", "max_seqs")] + \
         [(n, C.c_float) for n in (
             "lambda_", "tau", "rho_mi", "rho_t", "delta", "d_min", "t_min", "t_max", "eps", "eps_h")] + \
-        [("select_mode", C.c_int32)]
+        [(n, C.c_int32) for n in ("select_mode", "decay_mode", "aeb_mode", "mi_span")]
 
 
 class CSeq(C.Structure):
@@ -130,6 +130,9 @@ class Config:
     eps: float = 1e-6
     eps_h: float = 1e-12
     select_mode: int = 0    # SELECT_GLOBAL (the paper's) or SELECT_PER_HEAD
+    decay_mode: int = 0     # 0 exponential (Eq. 9), 1 linear, 2 power law (readings)
+    aeb_mode: int = 0       # 0 entropy, 1 peak confidence (reading)
+    mi_span: int = 0        # 0 every historical visual token, 1 the newest frame's
 
     def to_c(self) -> CConfig:
         c = CConfig()

@@ -23,7 +23,7 @@ def hyper(**over) -> Dict:
     """One set of hyper-parameters, given to both sides explicitly."""
     h = dict(lam=0.5, tau=1.0, rho_mi=0.9, n_warmup=5, n_ramp=10, delta=0.2, d_min=0.1,
              rho_t=0.9, t_min=0.95, t_max=1.05, pool_kernel=5, mi_bins=8, mi_grid=8,
-             eps=1e-6, eps_h=1e-12)
+             eps=1e-6, eps_h=1e-12, decay_mode=0, aeb_mode=0, mi_span=0)
     h.update(over)
     return h
 
@@ -40,7 +40,8 @@ def gpu_config(wl: syn.Workload, h: Dict, n_layers: Optional[int] = None, max_se
                      mi_grid=h["mi_grid"], n_warmup=h["n_warmup"], n_ramp=h["n_ramp"],
                      max_seqs=max_seqs, lambda_=h["lam"], tau=h["tau"], rho_mi=h["rho_mi"],
                      rho_t=h["rho_t"], delta=h["delta"], d_min=h["d_min"], t_min=h["t_min"],
-                     t_max=h["t_max"], eps=h["eps"], eps_h=h["eps_h"],
+                     t_max=h["t_max"], eps=h["eps"], eps_h=h["eps_h"], decay_mode=h["decay_mode"],
+                     aeb_mode=h["aeb_mode"], mi_span=h["mi_span"],
                      select_mode=sk.SELECT_PER_HEAD if per_head else sk.SELECT_GLOBAL)
 
 

@@ -39,8 +39,8 @@ def test_library_exports_every_declared_symbol(library):
 
 
 def test_struct_layouts_match_header():
-    assert ctypes.sizeof(sk.CConfig) == 13 * 4 + 10 * 4 + 4
-    assert [f[0] for f in sk.CConfig._fields_][-1] == "select_mode"
+    assert ctypes.sizeof(sk.CConfig) == 13 * 4 + 10 * 4 + 4 * 4
+    assert [f[0] for f in sk.CConfig._fields_][-4:] == ["select_mode", "decay_mode", "aeb_mode", "mi_span"]
 
 
 def test_header_constants_match_binding():
@@ -64,7 +64,8 @@ def test_default_config_matches_paper_defaults(library):
 
 @pytest.mark.parametrize("bad", [dict(head_dim=64), dict(n_heads=30), dict(window=64),
                                  dict(pool_kernel=4), dict(mi_bins=1), dict(t_min=0.0),
-                                 dict(n_kv_heads=0), dict(grid_rows=2000), dict(select_mode=2)])
+                                 dict(n_kv_heads=0), dict(grid_rows=2000), dict(select_mode=2),
+                                 dict(decay_mode=3), dict(aeb_mode=2), dict(mi_span=-1)])
 def test_invalid_config_rejected_before_any_device_call(library, bad):
     cfg = sk.Config(**bad)
     with pytest.raises(sk.StarkvError) as e:
