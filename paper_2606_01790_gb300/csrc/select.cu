@@ -164,7 +164,6 @@ struct CalShared {
   int any_tie;
   float fredn[4][32];             // multi-value block reductions
   uint32_t uredn[3][32];
-  float mic[kMaxGroups];          // every group's MI_g (phase 2)
   float pz[kMaxGroups], pzl[kMaxGroups], pv[kMaxGroups];   // every CTA's phase-2 partials
   uint32_t pkmin[kMaxGroups], pkmax[kMaxGroups], psmax[kMaxGroups];
   int pncand[kMaxGroups], pbelow[kMaxGroups];
@@ -688,13 +687,12 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     __syncthreads();
     const float fN = static_cast<float>(N);
     float acc = 0.f;
-    for (int bb = 0; bb < K; ++bb) {
-      for (int c = tid; c < MM; c += kCalThreads) {
-        const int n = joint[bb * MM + c];
-        if (n == 0) continue;
-        const float fn = static_cast<float>(n);
-        acc += fn * logf(fn * fN / (static_cast<float>(sh.nb[bb]) * static_cast<float>(ncell[c])));
-      }
+    for (int i = tid; i < K * MM; i += kCalThreads) {   // one (bin, cell) term per thread
+      const int bb = i / MM, c = i - bb * MM;
+      const int n = joint[i];
+      if (n == 0) continue;
+      const float fn = static_cast<float>(n);
+      acc += fn * logf(fn * fN / (static_cast<float>(sh.nb[bb]) * static_cast<float>(ncell[c])));
     }
     mi = block_sum<float>(acc, sh.fred) / fN;
   }
@@ -742,52 +740,55 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   float* stats = sv.stats ? sv.stats + static_cast<int64_t>(layer) * (8 + 6 * G) : nullptr;
   // ---- Eqs. (6)-(7): MI EMA (double state), min-max, softmax prior; lambda
   // schedule.  The same arithmetic in every CTA; CTA 0 stores the new state.
-  if (tid < G) {
-    sh.mic[tid] = dsmem_ld_f32(dsmem_map(&sh.mi, tid));
-    sh.ph[tid] = dsmem_ld_f32(dsmem_map(&sh.phi, tid));
-  }
-  __syncthreads();
-  if (tid == 0) {
+  // warp 0, lane gg < G: group gg's MI (from CTA gg), its EMA, then the
+  // min-max and the softmax over the groups by warp reductions
+  if (warp == 0) {
     const int n = sh.n_old;
-    double mib[kMaxGroups];
-    float mf[kMaxGroups];
-    float lo = 3.4e38f, hi = -3.4e38f;
-    for (int gg = 0; gg < G; ++gg) {
-      mib[gg] = n == 0 ? static_cast<double>(sh.mic[gg])
-                       : kp.rho_mi * sh.mib_old[gg] + (1.0 - kp.rho_mi) * static_cast<double>(sh.mic[gg]);
-      mf[gg] = static_cast<float>(mib[gg]);
-      lo = fminf(lo, mf[gg]);
-      hi = fmaxf(hi, mf[gg]);
+    const bool on = lane < G;
+    double mib = 0.0;
+    float mic = 0.f, mf = 0.f;
+    if (on) {
+      mic = dsmem_ld_f32(dsmem_map(&sh.mi, lane));
+      sh.ph[lane] = dsmem_ld_f32(dsmem_map(&sh.phi, lane));
+      mib = n == 0 ? static_cast<double>(mic)
+                   : kp.rho_mi * sh.mib_old[lane] + (1.0 - kp.rho_mi) * static_cast<double>(mic);
+      mf = static_cast<float>(mib);
     }
-    float e[kMaxGroups], zmax = -3.4e38f, zs = 0.f;
+    float lo = on ? mf : 3.4e38f, hi = on ? mf : -3.4e38f;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      lo = fminf(lo, __shfl_xor_sync(kFullMask, lo, o));
+      hi = fmaxf(hi, __shfl_xor_sync(kFullMask, hi, o));
+    }
     const float inv = 1.f / (((hi - lo) + kp.eps) * kp.tau);
-    for (int gg = 0; gg < G; ++gg) {
-      e[gg] = (mf[gg] - lo) * inv;
-      zmax = fmaxf(zmax, e[gg]);
-    }
-    for (int gg = 0; gg < G; ++gg) {
-      e[gg] = expf(e[gg] - zmax);
-      zs += e[gg];
-    }
-    for (int gg = 0; gg < G; ++gg) sh.w[gg] = e[gg] / zs;
+    const float e = on ? (mf - lo) * inv : -3.4e38f;
+    float zmax = e;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) zmax = fmaxf(zmax, __shfl_xor_sync(kFullMask, zmax, o));
+    const float ex = on ? expf(e - zmax) : 0.f;
+    const float zs = warp_sum(ex);
+    const float wg = ex / zs;
+    if (on) sh.w[lane] = wg;
     float lam = 0.f;
     if (n >= kp.n_warmup)
       lam = kp.n_ramp <= 0 ? kp.lambda
                            : kp.lambda * fminf(1.f, static_cast<float>(n - kp.n_warmup) / kp.n_ramp);
-    sh.lam = lam;
+    if (lane == 0) sh.lam = lam;
     if (g == 0) {
-      for (int gg = 0; gg < G; ++gg) st.mi_bar[sl * G + gg] = mib[gg];
-      st.n[sl] = n + 1;
+      if (on) st.mi_bar[sl * G + lane] = mib;
+      if (lane == 0) st.n[sl] = n + 1;
       if (stats) {
-        stats[2] = lam;
-        stats[3] = static_cast<float>(n);
-        stats[6] = static_cast<float>(sv.budget);
-        stats[7] = 0.f;
-        for (int gg = 0; gg < G; ++gg) {
-          stats[8 + gg] = sh.mic[gg];
-          stats[8 + G + gg] = mf[gg];
-          stats[8 + 2 * G + gg] = sh.w[gg];
-          stats[8 + 3 * G + gg] = sh.ph[gg];
+        if (lane == 0) {
+          stats[2] = lam;
+          stats[3] = static_cast<float>(n);
+          stats[6] = static_cast<float>(sv.budget);
+          stats[7] = 0.f;
+        }
+        if (on) {
+          stats[8 + lane] = mic;
+          stats[8 + G + lane] = mf;
+          stats[8 + 2 * G + lane] = wg;
+          stats[8 + 3 * G + lane] = sh.ph[lane];
         }
       }
     }
