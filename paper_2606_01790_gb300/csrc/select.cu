@@ -592,41 +592,62 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         }
       }
       __syncthreads();
-      if (tid == 0) {
+      if (warp == 0) {
         // boundaries are in rank order, so their buckets are non-decreasing;
-        // a slot is one boundary bucket with its candidate tokens
-        int slot = -1, prev = -1, off = 0, nmax = 0;
-        for (int j = 0; j < nt; ++j) {
-          if (!sh.reach[j]) continue;
-          if (sh.dig[j] != prev) {
-            ++slot;
-            prev = sh.dig[j];
-            const int n = hist[prev];
-            sh.slot_off[slot] = off;
-            sh.slot_n[slot] = n;
-            sh.slot_j0[slot] = j;
-            off += n;
-            nmax = max(nmax, n);
-          }
-          sh.slot_of[j] = slot;
-          sh.rem[j] -= sh.below[j];   // rank inside the bucket
+        // a slot is one boundary bucket with its candidate tokens.  Lane j is
+        // boundary j (nt <= 15; the reachable ones are a prefix).
+        const bool rj = lane < nt && sh.reach[lane];
+        const int dj = lane < nt ? sh.dig[lane] : -1;
+        const int dprev = __shfl_up_sync(kFullMask, dj, 1);
+        const bool isnew = rj && (lane == 0 || dj != dprev);
+        const unsigned newmask = __ballot_sync(kFullMask, isnew);
+        const int slot = __popc(newmask & ((2u << lane) - 1u)) - 1;   // slots opened at lanes <= this one
+        const int n = isnew ? hist[dj] : 0;
+        int incl = n;   // running candidate offset over the slots
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int y = __shfl_up_sync(kFullMask, incl, o);
+          if (lane >= o) incl += y;
         }
-        sh.nslot = slot + 1;
-        sh.ncand_all = off;
-        sh.brute = off <= Lp / 2 && nmax <= kBruteMax;
+        if (isnew) {
+          sh.slot_off[slot] = incl - n;
+          sh.slot_n[slot] = n;
+          sh.slot_j0[slot] = lane;
+        }
+        if (rj) {
+          sh.slot_of[lane] = slot;
+          sh.rem[lane] -= sh.below[lane];   // rank inside the bucket
+        }
+        const int total = __shfl_sync(kFullMask, incl, 31);
+        const int nmax = __reduce_max_sync(kFullMask, static_cast<unsigned>(n));
+        if (lane == 0) {
+          sh.nslot = __popc(newmask);
+          sh.ncand_all = total;
+          sh.brute = total <= Lp / 2 && nmax <= kBruteMax;
+        }
       }
       __syncthreads();
     }
     // ---- bucket table: a bucket without a boundary puts all its tokens in
     // one rank bin (the boundaries below it); a boundary bucket is refined
-    for (int bk = tid; bk < kBins0; bk += kCalThreads) {
-      int below = 0, slot = -1;
+    static_assert(kBins0 == 4 * kCalThreads, "four buckets per thread");
+    {
+      const int bk0 = 4 * tid;   // this thread's four consecutive buckets, each boundary read once
+      int below[4] = {0, 0, 0, 0}, slot[4] = {-1, -1, -1, -1};
       for (int j = 0; j < nt; ++j) {
         if (!sh.reach[j]) break;
-        below += sh.dig[j] < bk;
-        if (sh.dig[j] == bk) slot = sh.slot_of[j];
+        const int d = sh.dig[j], so = sh.slot_of[j];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          below[k] += d < bk0 + k;
+          if (d == bk0 + k) slot[k] = so;
+        }
       }
-      btab[bk] = static_cast<uint8_t>(slot >= 0 ? (0x80 | slot) : below);
+      uint32_t packed = 0u;
+#pragma unroll
+      for (int k = 0; k < 4; ++k)
+        packed |= static_cast<uint32_t>(static_cast<uint8_t>(slot[k] >= 0 ? (0x80 | slot[k]) : below[k])) << (8 * k);
+      reinterpret_cast<uint32_t*>(btab)[tid] = packed;
     }
     __syncthreads();
     const bool brute = sh.brute;
