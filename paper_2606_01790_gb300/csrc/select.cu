@@ -499,6 +499,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   };
   if (vec) {
     const float4* st4 = reinterpret_cast<const float4*>(stage);
+    const bool s16 = (reinterpret_cast<uintptr_t>(S) & 15) == 0;   // S row on a 16-byte boundary
     for (int t0 = 4 * tid; t0 < Lp; t0 += 4 * kCalThreads) {
       float sv4[4];
       if (half == 2 && t0 >= 4 && t0 + 8 <= Lp) {   // x[t0 - 4 .. t0 + 7] in three 16-byte loads
@@ -515,12 +516,13 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       const uint32_t mts[4] = {m4.x, m4.y, m4.z, m4.w};
       uint32_t ks[4];
       uint16_t cs[4];
+      if (s16 && t0 + 3 < Lp) *reinterpret_cast<float4*>(S + t0) = make_float4(sv4[0], sv4[1], sv4[2], sv4[3]);
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
         ks[k] = 0u;
         cs[k] = kNoCell;
         if (t0 + k < Lp) {
-          S[t0 + k] = sv4[k];
+          if (!s16 || t0 + 3 >= Lp) S[t0 + k] = sv4[k];
           classify(sv4[k], mts[k], ks[k], cs[k]);
         }
       }
@@ -815,8 +817,13 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     }
   }
   __syncthreads();   // w and lambda are read by every thread below
-  const int ta = per_head ? 0 : static_cast<int>(static_cast<int64_t>(g) * Lp / G);
-  const int tb = per_head ? Lp : static_cast<int>(static_cast<int64_t>(g + 1) * Lp / G);
+  // (range boundaries on multiples of 4 tokens, so that the ranges can be read in 16 bytes)
+  auto split = [&](int r) {
+    const int64_t t = (static_cast<int64_t>(r) * Lp / G + 3) & ~static_cast<int64_t>(3);
+    return static_cast<int>(t < Lp ? t : Lp);
+  };
+  const int ta = per_head ? 0 : split(g);
+  const int tb = per_head ? Lp : split(g + 1);
   const int nr = tb - ta;
   const float* S0 = sv.S + static_cast<int64_t>(layer) * G * Lp;
   const float invG = 1.f / static_cast<float>(G);
@@ -873,6 +880,32 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         const int i = i0 + k * kCalThreads + tid;
         if (i < nr) fuse(i, v[k], g, mw[k]);
       }
+    }
+  } else if ((Lp & 3) == 0 && ((reinterpret_cast<uintptr_t>(S0) | reinterpret_cast<uintptr_t>(meta)) & 15) == 0) {
+    // four consecutive tokens per thread, every group's row and the metadata
+    // read in 16 bytes (ta and Lp are multiples of 4)
+    for (int i0 = 4 * tid; i0 < nr; i0 += 4 * kCalThreads) {
+      const int t = ta + i0;
+      const uint4 m4 = *reinterpret_cast<const uint4*>(meta + t);
+      float4 acc = *reinterpret_cast<const float4*>(S0 + t), best = acc;
+      int gs[4] = {0, 0, 0, 0};
+#pragma unroll
+      for (int gg = 1; gg < kMaxGroups; ++gg) {
+        if (gg >= G) break;
+        const float4 q = *reinterpret_cast<const float4*>(S0 + static_cast<int64_t>(gg) * Lp + t);
+        acc.x += q.x;
+        acc.y += q.y;
+        acc.z += q.z;
+        acc.w += q.w;
+        if (q.x > best.x) { best.x = q.x; gs[0] = gg; }
+        if (q.y > best.y) { best.y = q.y; gs[1] = gg; }
+        if (q.z > best.z) { best.z = q.z; gs[2] = gg; }
+        if (q.w > best.w) { best.w = q.w; gs[3] = gg; }
+      }
+      fuse(i0, acc.x * invG, gs[0], m4.x);
+      fuse(i0 + 1, acc.y * invG, gs[1], m4.y);
+      fuse(i0 + 2, acc.z * invG, gs[2], m4.z);
+      fuse(i0 + 3, acc.w * invG, gs[3], m4.w);
     }
   } else {
     for (int i0 = 0; i0 < nr; i0 += 2 * kCalThreads) {
