@@ -369,6 +369,9 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   for (int i = tid; i < RC; i += kCalThreads) cur[i] = 0.f;
   for (int r = tid; r < R; r += kCalThreads) rowc[r] = static_cast<uint8_t>(r * M / R);
   for (int c = tid; c < C; c += kCalThreads) colc[c] = static_cast<uint8_t>(c * M / C);
+  // this group's temporal EMA row (state of the previous step, read after
+  // phase 1) on its way into L2
+  if (tid * 32 < RC) prefetch_l2(st.m + static_cast<int64_t>(sl * G + g) * RC + tid * 32);
   __syncthreads();
   // the set-up above overlaps the previous kernel's tail; its outputs are read below
   griddep_launch_dependents();
@@ -573,10 +576,28 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
 
   float mi = 0.f;
   if (N > 0) {
-    for (int base = s0; base < s1; base += 32) {
-      const int t = base + lane;
-      if (t < s1 && cells[t] != kNoCell) atomicAdd(&hist[bucket_of(keys[t])], 1);
-    }
+    // (token order does not matter here: four consecutive tokens per thread
+    // when the row is on chip, else the warp segments)
+    auto each_visual = [&](auto&& f) {
+      if (in_smem) {
+        for (int t0 = 4 * tid; t0 < Lp; t0 += 4 * kCalThreads) {
+          const uint4 k4 = reinterpret_cast<const uint4*>(keys)[t0 >> 2];
+          const uint2 c2 = reinterpret_cast<const uint2*>(cells)[t0 >> 2];
+          const uint32_t ku[4] = {k4.x, k4.y, k4.z, k4.w};
+          const uint32_t cu[4] = {c2.x & 0xFFFFu, c2.x >> 16, c2.y & 0xFFFFu, c2.y >> 16};
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            if (t0 + k < Lp && cu[k] != kNoCell) f(t0 + k, ku[k], static_cast<int>(cu[k]));
+        }
+      } else {
+        for (int base = s0; base < s1; base += 32) {
+          const int t = base + lane;
+          const int cell = t < s1 ? cells[t] : kNoCell;
+          if (cell != kNoCell) f(t, keys[t], cell);
+        }
+      }
+    };
+    each_visual([&](int, uint32_t u, int) { atomicAdd(&hist[bucket_of(u)], 1); });
     __syncthreads();
     {
       const int4 h = reinterpret_cast<const int4*>(hist)[tid];
@@ -656,11 +677,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     // ---- joint histogram of the settled tokens; boundary-bucket tokens go
     // to their slot's (key, position) pool
     uint32_t* pool = cand;   // [2 * candidates]
-    for (int base = s0; base < s1; base += 32) {
-      const int t = base + lane;
-      const int cell = t < s1 ? cells[t] : kNoCell;
-      if (cell == kNoCell) continue;
-      const uint32_t u = keys[t];
+    each_visual([&](int t, uint32_t u, int cell) {
       const int v = btab[bucket_of(u)];
       if (!(v & 0x80)) {
         atomicAdd(&joint[v * MM + cell], 1);
@@ -670,7 +687,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         pool[2 * i] = u;
         pool[2 * i + 1] = static_cast<uint32_t>(t);
       }
-    }
+    });
     __syncthreads();
     if (brute) {
       // exact rank of each candidate inside its bucket by (key, position),
