@@ -153,9 +153,9 @@ class ClockSampler:
 def oracle_worker(args):
     """Times the fp64 oracle on the workload; prints one JSON line.
 
-    Budget mode (``--repeat 0``): layers 0, 1, ... of sequence 0 until
-    ``--budget-s`` seconds of oracle work have run.  Repeat mode: layer 0,
-    ``--repeat`` times (the reference arm's steps)."""
+    Budget mode (``--repeat 0``): layers 0, 1, ... of sequence 0, cycled,
+    until ``--budget-s`` seconds of oracle work have run.  Repeat mode: layer
+    0, ``--repeat`` times (the reference arm's steps)."""
     from oracle import starkv_oracle as O
     from paper_2606_01790_gb300 import synthetic as syn
     wl = syn.WORKLOADS[args.workload]
@@ -163,7 +163,10 @@ def oracle_worker(args):
     per_head = args.select_mode == "per_head"
     spent, tokens = 0.0, 0
     per_call = []
-    layers = [0] * args.repeat if args.repeat > 0 else list(range(min(wl.n_layers, args.max_layers)))
+    nl = min(wl.n_layers, args.max_layers)
+    # repeat mode: layer 0, --repeat times; budget mode: layers 0, 1, ... cycled
+    # until --budget-s seconds of oracle work have run
+    layers = [0] * args.repeat if args.repeat > 0 else (i % nl for i in range(1 << 30))
     cache = {}
     for layer in layers:
         if layer not in cache:
@@ -425,8 +428,8 @@ def gpu_arm(args):
         o = run_oracle_subprocess(args.workload, budget_s=args.cpu_budget_s, max_layers=wl.n_layers,
                                   select_mode=args.select_mode)
         cpu = {"value": o["tokens"] / o["seconds"], "unit": UNIT, "cores": o["cores"], "kind": "oracle",
-               "sample": f"{o['calls']} of {wl.n_layers} layers of sequence 0 "
-                         f"({o['tokens']} tokens scored in {o['seconds']:.1f} s, "
+               "sample": f"{o['calls']} layer compressions of sequence 0 (layers 0..{wl.n_layers - 1} "
+                         f"cycled; {o['tokens']} tokens scored in {o['seconds']:.1f} s, "
                          f"numpy BLAS on {o['cores']} threads)"}
 
     if rank == 0:
