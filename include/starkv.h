@@ -59,7 +59,8 @@
  *   0 <= B <= L_p; L < 2^24; 1 <= R, C <= 1024; R * C <= 16384;
  *   2 <= mi_bins <= 16; mi_bins * mi_grid^2 <= 4096; odd pool_kernel <= 31;
  *   frame ids 0..2047.  Other shapes return STARKV_ERR_UNSUPPORTED.
- *   k, v, q, k_out and v_out must be 16-byte aligned.
+ *   k, v, q, k_out and v_out must be 16-byte aligned, every other array
+ *   4-byte aligned (STARKV_ERR_INVALID_ARG otherwise).
  */
 #ifndef STARKV_H
 #define STARKV_H

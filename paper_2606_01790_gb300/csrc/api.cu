@@ -159,6 +159,7 @@ enum Need : unsigned {
 };
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+bool aligned4(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 3) == 0; }
 
 starkv_status validate_seqs(const starkv_state* st, const starkv_seq* seqs, int nseq, unsigned need) {
   if (!st) return set_error(STARKV_ERR_INVALID_ARG, "state is NULL");
@@ -190,6 +191,10 @@ starkv_status validate_seqs(const starkv_state* st, const starkv_seq* seqs, int 
       if (s.meta_layer_stride != 0 && s.meta_layer_stride < span)
         return set_error(STARKV_ERR_INVALID_ARG, "seq %d: meta_layer_stride must be 0 or >= (G-1)*meta_group_stride + L", i);
     }
+    // 4-byte words: a misaligned pointer is an argument error, not a device fault
+    const void* words[] = {s.meta, s.meta_out, s.idx, s.S, s.score, s.stats, s.lse};
+    for (const void* w : words)
+      if (w && !aligned4(w)) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: a 4-byte array is not 4-byte aligned", i);
     if ((need & kNeedS) && !s.S && lp > 0) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: S is NULL", i);
     if ((need & kNeedIdx) && !s.idx && s.budget > 0) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: idx is NULL", i);
     if (need & kNeedOut) {

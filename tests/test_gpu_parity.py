@@ -274,3 +274,10 @@ def test_invalid_arguments_rejected():
         sk.step(st, [ds.seq], ws[:1024])           # workspace too small
     with pytest.raises(sk.StarkvError):
         sk.score_layer(st, 5, [ds.seq], ws)        # layer out of range
+    # a 4-byte array at an odd address is refused before any launch
+    mis = H.device_seq(si, wl).seq
+    raw = torch.zeros(mis.meta.numel() * 4 + 4, dtype=torch.uint8, device="cuda")
+    mis.meta = raw[2:2 + mis.meta.numel() * 4]
+    with pytest.raises(sk.StarkvError) as e:
+        sk.step(st, [mis], ws)
+    assert e.value.status == sk.ERR_INVALID_ARG
