@@ -66,9 +66,16 @@ def work_per_step(wl, seqs, per_head=False):
                 step_bytes=k_bytes + s_bytes + gather)
 
 
-def kernel_work(kind, work):
-    """(bound, algorithmic units per step, unit) of one kernel kind."""
+def kernel_work(kind, work, peaks):
+    """(bound, algorithmic units per step, unit) of one kernel kind.  A scoring
+    pass reads K once and does the Q K^T flops; its bound is whichever of the
+    two takes longer at the measured peaks (224 flop per byte at the UI-TARS
+    shape, below the HBM / bf16 ridge, so HBM)."""
     if kind in ("score_lse", "score_accum"):
+        t_hbm = work["k_bytes"] / (peaks["hbm"] * 1e9)
+        t_tc = work["qk_flops"] / (peaks["tc_sus"] * 1e12)
+        if t_hbm >= t_tc:
+            return "hbm", work["k_bytes"] / 1e9, "GB/s"
         return "tensor", work["qk_flops"] / 1e12, "TFLOP/s"
     if kind == "compact":
         return "hbm", work["gather_bytes"] / 1e9, "GB/s"
@@ -379,7 +386,7 @@ def gpu_arm(args):
             continue
         kernels[kind] = {"launches": n, "avg_us": 1e3 * tms / n, "share": tms / max(1e-9, sum(v[1] for v in kt.values()))}
     dom = max(kernels, key=lambda k: kernels[k]["avg_us"] * kernels[k]["launches"])
-    bound, units_per_step, unit = kernel_work(dom, work)
+    bound, units_per_step, unit = kernel_work(dom, work, peaks)
     per_launch = units_per_step * n_kt / kernels[dom]["launches"]
     achieved = per_launch / (kernels[dom]["avg_us"] * 1e-6)
     peak = peaks["tc_sus"] if bound == "tensor" else peaks["hbm"]
