@@ -154,3 +154,39 @@ def test_meta_group_stride_needs_the_per_head_mode():
     with pytest.raises(sk.StarkvError) as e:
         sk.step(st, [ds.seq], sk.workspace(st, [ds.seq]))
     assert e.value.status == sk.ERR_INVALID_ARG
+
+
+def test_per_head_with_supplied_normalisers():
+    """Per-KV-head selection on top of the supplied-normaliser path (first
+    scoring pass skipped)."""
+    wl = syn.WORKLOADS["uitars_layer"]
+    si = syn.make_sequence(wl)
+    h = H.hyper(n_warmup=0, n_ramp=0)
+    p = H.oracle_params(h)
+    lse = O.window_lse(si.q[0].double().numpy(), si.k[0].double().numpy(), wl.window)
+    st = sk.init_state(H.gpu_config(wl, h, per_head=True))
+    ds = H.device_seq(si, wl, per_head=True)
+    ds.seq.lse = torch.from_numpy(lse.astype(np.float32))[None].cuda()
+    sk.kernel_times(st)
+    _step(st, [ds])
+    assert sk.kernel_times(st)["score_lse"][0] == 0
+    S = O.score_layer(si.q[0].double().numpy(), si.k[0].double().numpy(), wl.window, p,
+                      lse=lse.astype(np.float32).astype(np.float64))
+    ref = H.oracle_layer(si, 0, wl, _fresh(wl), p, S_override=S, per_head=True)
+    H.check_per_head(ds.seq, si, 0, wl, ref)
+
+
+def test_per_head_sixteen_ragged_trajectories():
+    """16 independent sequences of different lengths and budgets in one
+    batched per-KV-head step over 28 layers; sampled (sequence, layer) pairs."""
+    wl = syn.WORKLOADS["ragged"]
+    h = H.hyper(n_warmup=0, n_ramp=0)
+    p = H.oracle_params(h)
+    sis = [syn.make_sequence(wl, seq=i) for i in range(wl.n_seqs)]
+    st = sk.init_state(H.gpu_config(wl, h, max_seqs=wl.n_seqs, per_head=True))
+    dss = [H.device_seq(si, wl, slot=i, per_head=True) for i, si in enumerate(sis)]
+    _step(st, dss)
+    lens = [si.L for si in sis]
+    for i, layer in ((int(np.argmin(lens)), 5), (int(np.argmax(lens)), 22)):
+        ref = H.oracle_layer(sis[i], layer, wl, _fresh(wl), p, per_head=True)
+        H.check_per_head(dss[i].seq, sis[i], layer, wl, ref)

@@ -57,3 +57,27 @@ def test_variant_matches_oracle_over_two_calls(variant, per_head):
     if "decay_mode" in variant:
         d = ref["D"]
         assert np.ptp(d) > 1e-3        # the decay shape took part
+
+
+def test_variants_on_a_row_longer_than_shared_memory():
+    """20 screenshots + 2,048 text tokens (L_p = 56,096): the calibration keeps
+    its per-token arrays in the workspace; the decay and MI-span switches on
+    that path, over two calls."""
+    wl = syn.WORKLOADS["long_layer"]
+    si = syn.make_sequence(wl)
+    h = H.hyper(n_warmup=0, n_ramp=0, decay_mode=1, mi_span=1, aeb_mode=1)
+    p = H.oracle_params(h)
+    S = O.score_layer(si.q[0].double().numpy(), si.k[0].double().numpy(), wl.window, p)
+    st = sk.init_state(H.gpu_config(wl, h))
+    ost = O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols)
+    for call in range(2):
+        ds = H.device_seq(si, wl)
+        sk.step(st, [ds.seq], sk.workspace(st, [ds.seq]))
+        torch.cuda.synchronize()
+        sk.check_device_error(st)
+        ref = H.oracle_layer(si, 0, wl, ost, p, S_override=S)
+        sc = H.check_scores(ds.seq.score[0].double().cpu().numpy(), ref, S, si, 0, wl, p)
+        assert sc["ok"], (call, sc)
+        assert H.check_index_set(ds.seq.idx[0].cpu().numpy(), ref, si.budget)["ok"]
+        H.check_compaction(ds.seq, si, 0, wl.window)
+    assert np.max(ref["phi"]) > 0.0
