@@ -38,7 +38,7 @@ namespace starkv {
 
 namespace {
 
-constexpr int kMaxStages = 4;                 // K-tile pipeline depth (at most)
+constexpr int kMaxStages = 4;                 // K-tile pipeline depth (at most; even, see score_kstages)
 constexpr size_t kSmemLimit = 227 * 1024;
 constexpr int kTileBytes = kTileKeys * 256;   // 128 keys x 128 bf16
 constexpr int kHalfBytes = kTileKeys * 128;   // one 64-column swizzled half
@@ -686,9 +686,14 @@ size_t score_smem_bytes(int q_rows, int kstages) {
   return 1024 + static_cast<size_t>(2 * q_rows * 128) + static_cast<size_t>(kstages) * kTileBytes + 256 + aux;
 }
 
+// The K-stage count is even: MMA issuer `who` takes tiles who, who + 2, ..., so
+// with an even count every stage belongs to one issuer, which consumes its
+// phases in order.  With an odd count consecutive uses of a stage alternate
+// between the issuers, and one can wait on the stage's next phase while the
+// other's load of it is still in flight (the parity wait then passes early).
 int score_kstages(int q_rows) {
-  int k = kMaxStages;
-  while (k > 0 && score_smem_bytes(q_rows, k) > kSmemLimit) --k;
+  int k = kMaxStages & ~1;
+  while (k > 0 && score_smem_bytes(q_rows, k) > kSmemLimit) k -= 2;
   return k;
 }
 
