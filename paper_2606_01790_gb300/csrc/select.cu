@@ -92,24 +92,6 @@ __device__ int block_excl_scan(int v, int* tmp, int* total) {
   return tmp[warp] + incl - v;
 }
 
-__device__ uint32_t block_min(uint32_t v, uint32_t* red) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  v = __reduce_min_sync(kFullMask, v);
-  __syncthreads();
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  return __reduce_min_sync(kFullMask, red[lane]);
-}
-
-__device__ uint32_t block_max(uint32_t v, uint32_t* red) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  v = __reduce_max_sync(kFullMask, v);
-  __syncthreads();
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  return __reduce_max_sync(kFullMask, red[lane]);
-}
-
 // One warp: the bin of a 256-bin histogram that holds rank `rank` (0-based)
 // and the count of keys in lower bins; written by the lane that finds it.
 __device__ void warp_find_256(const int* hist, int rank, int* digit, int* below) {
@@ -150,13 +132,11 @@ struct CalShared {
   int slot_j0[kMaxTargets];       // slot -> first boundary in it (= boundaries in lower buckets)
   int slot_cnt[kMaxTargets];      // slot -> candidates placed so far
   int nslot, ncand_all, brute;
-  uint32_t ured[32];
   int ncand[32];                  // boundary-bucket tokens of each warp's segment
   int eqw[32][kMaxTargets];       // keys equal to each boundary before each warp's segment
   int nb[16];                     // rank-bin marginals
   int scan[33];
   float fred[32];
-  int ired[32];
   double mib_old[kMaxGroups];     // MI EMA before this step
   float w[kMaxGroups], ph[kMaxGroups];
   float lam;
