@@ -107,3 +107,30 @@ def test_supplied_normalisers_at_an_odd_shape():
     S = O.score_layer(si.q[0].double().numpy(), si.k[0].double().numpy(), wl.window, p, lse=lse.astype(np.float64))
     S_gpu = ds.seq.S[0].double().cpu().numpy()
     assert (np.abs(S_gpu - S) / np.abs(S)).max() < 1e-3
+
+
+def test_forty_sequences_span_two_launch_batches():
+    """40 ragged sequences in one step: a launch carries at most 32 sequences,
+    so the call runs two batches of every kernel (the second with its own
+    tensor maps, partial-sum offsets and state slots).  Sampled sequences on
+    both sides of the batch boundary against the oracle, in both layers."""
+    wl = dataclasses.replace(syn.WORKLOADS["tiny"], n_layers=2, n_seqs=40, ragged=True,
+                             shots_range=(1, 3), text_range=(16, 160))
+    h = H.hyper(n_warmup=0, n_ramp=0, t_min=0.75, t_max=1.25)
+    p = H.oracle_params(h)
+    sis = [syn.make_sequence(wl, seq=i) for i in range(wl.n_seqs)]
+    assert len({si.L for si in sis}) > 10
+    st = sk.init_state(H.gpu_config(wl, h, max_seqs=wl.n_seqs))
+    dss = [H.device_seq(si, wl, slot=i) for i, si in enumerate(sis)]
+    sk.step(st, [d.seq for d in dss], sk.workspace(st, [d.seq for d in dss]))
+    torch.cuda.synchronize()
+    sk.check_device_error(st)
+    for i in (0, 31, 32, 39):
+        for layer in (0, 1):
+            ref = H.oracle_layer(sis[i], layer, wl,
+                                 O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols), p)
+            sc = H.check_scores(dss[i].seq.score[layer].double().cpu().numpy(), ref, ref["S"], sis[i], layer, wl, p)
+            assert sc["ok"], (i, layer, sc)
+            ix = H.check_index_set(dss[i].seq.idx[layer].cpu().numpy(), ref, sis[i].budget)
+            assert ix["ok"], (i, layer, ix)
+            H.check_compaction(dss[i].seq, sis[i], layer, wl.window)
