@@ -82,12 +82,40 @@ def kernel_work(kind, work, peaks):
     return "hbm", work["s_bytes"] / 1e9, "GB/s"
 
 
-def kernel_src_hash(kind):
+def code_only(text):
+    """C/C++ source without its comments and with whitespace runs collapsed,
+    so that an edit of comments alone keeps a kernel's recorded counters."""
+    out, i, n = [], 0, len(text)
+    while i < n:
+        c = text[i]
+        if c in "\"'":   # string or character literal, copied as is
+            j = i + 1
+            while j < n and text[j] != c:
+                j += 2 if text[j] == "\\" else 1
+            out.append(text[i:j + 1])
+            i = j + 1
+        elif text.startswith("//", i):
+            j = text.find("\n", i)
+            i = n if j < 0 else j
+        elif text.startswith("/*", i):
+            j = text.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+            out.append(" ")
+        else:
+            out.append(c)
+            i += 1
+    return " ".join("".join(out).split())
+
+
+def kernel_src_hash(kind, read=None):
+    """Hash of the code (comments excluded) that a kernel is built from;
+    ``read(name)`` returns a source file's text (default: the working tree)."""
     files = {"score_lse": "score.cu", "score_accum": "score.cu", "pool": "score.cu",
              "calibrate": "select.cu", "compact": "compact.cu"}[kind]
+    read = read or (lambda f: (ROOT / "paper_2606_01790_gb300" / "csrc" / f).read_text())
     h = hashlib.sha256()
     for f in (files, "ptx.cuh", "common.cuh"):
-        h.update((ROOT / "paper_2606_01790_gb300" / "csrc" / f).read_bytes())
+        h.update(code_only(read(f)).encode())
     return h.hexdigest()[:16]
 
 

@@ -21,12 +21,14 @@
 // Both passes split the flattened (seq, layer, group, key tile) space into one
 // contiguous range per CTA (persistent grid <= #SMs), so a CTA reloads the
 // group's queries only when its range crosses into a new (seq, layer, group)
-// row ("piece").  Warp roles: warp 0 TMA producer, warp 1 MMA issuer (+ TMEM
-// owner), warps 4..19 epilogue: four warpgroups that all work on every tile,
-// so the 32-bit exp2 stream (the bound of both passes) is spread over 16
-// warps.  Two 256-column TMEM accumulator stages let the MMA of tile i+1 run
-// under the epilogue of tile i; TMEM is read in 16-column loads with the next
-// load in flight under the arithmetic, which runs on packed fp32 pairs.
+// row ("piece").  Warp roles: warp 0 TMA producer, warps 1 and 2 MMA issuers
+// (even / odd tiles; warp 1 also owns the TMEM allocation), warps 4..19
+// epilogue: four warpgroups that all work on every tile, so the per-element
+// exp2 and sums are spread over 16 warps.  Two 256-column TMEM accumulator
+// stages let the MMA of tile i+1 run under the epilogue of tile i; TMEM is
+// read in 16-column loads with the next load in flight under the arithmetic,
+// which runs on packed fp32 pairs.  Each pass is bounded below by its K
+// stream and, at nearly the same level, by the epilogue's per-tile cost.
 #include <algorithm>
 #include <utility>
 

@@ -60,3 +60,21 @@ def test_reference_arm_prints_on_rank_zero_only():
                        timeout=120)
     assert r.returncode == 0, r.stderr
     assert r.stdout.strip() == ""
+
+
+def test_recorded_traffic_follows_the_kernel_code_not_its_comments():
+    """The DRAM bytes a committed ncu capture recorded are reported only for
+    the code they were measured on: the key ignores comments and layout, and
+    changes with any code token."""
+    a = "int f(int x) {\n  return x + 1;  // one more\n}\n/* note */\n"
+    b = "int f(int x) {   return x + 1; }\n// another note\n"
+    c = "int f(int x) {\n  return x + 2;\n}\n"
+    assert bench.code_only(a) == bench.code_only(b) != bench.code_only(c)
+    assert bench.code_only('s = "a // b"; // tail') == 's = "a // b";'
+    tree = {f: open(os.path.join(ROOT, "paper_2606_01790_gb300", "csrc", f)).read()
+            for f in ("score.cu", "ptx.cuh", "common.cuh")}
+    edited = dict(tree, **{"score.cu": "// a new comment line\n" + tree["score.cu"]})
+    changed = dict(tree, **{"score.cu": tree["score.cu"] + "\nstatic int extra_symbol;\n"})
+    h = bench.kernel_src_hash("score_lse", tree.__getitem__)
+    assert bench.kernel_src_hash("score_lse", edited.__getitem__) == h
+    assert bench.kernel_src_hash("score_lse", changed.__getitem__) != h
