@@ -276,9 +276,19 @@ starkv_status starkv_check_device_error(starkv_state* st, void* stream);
 
 /* Limit, in nanoseconds, of every bounded device-side wait of this state's
  * kernels (default 1e9).  A wait that runs out stops its kernel early and
- * latches STARKV_ERR_TIMEOUT in the device error word.  A debugging and test
- * knob: 0 makes the first wait that does not succeed at once run out. */
+ * latches STARKV_ERR_TIMEOUT in the device error word; before it exits or
+ * releases tensor memory the kernel still waits for the copies and MMAs it
+ * has already issued, for max(limit, 2 s). */
 starkv_status starkv_set_wait_limit(starkv_state* st, uint64_t limit_ns);
+
+/* Self-test of the failure path that every bounded device wait shares: one
+ * thread of a one-block kernel waits on a shared-memory barrier that nothing
+ * completes; after `limit_ns` (1e3 .. 1e9) the wait gives up, latches
+ * STARKV_ERR_TIMEOUT in the state's device error word and the kernel
+ * returns, so the context stays usable.  Stream-ordered; the next
+ * starkv_check_device_error reports STARKV_ERR_TIMEOUT (and clears it).
+ * STARKV_ERR_INVALID_ARG for a NULL state or a limit out of range. */
+starkv_status starkv_selftest_wait(starkv_state* st, uint64_t limit_ns, void* stream);
 
 /* Kernels of the library, for starkv_kernel_times. */
 enum {

@@ -773,6 +773,16 @@ starkv_status starkv_check_device_error(starkv_state* st, void* stream) {
   return STARKV_OK;
 }
 
+starkv_status starkv_selftest_wait(starkv_state* st, uint64_t limit_ns, void* stream) {
+  if (!st) return set_error(STARKV_ERR_INVALID_ARG, "state is NULL");
+  if (limit_ns < 1000ull || limit_ns > 1000000000ull)
+    return set_error(STARKV_ERR_INVALID_ARG, "limit_ns must be in [1 us, 1 s]");
+  starkv_status s = check_device(st);
+  if (s != STARKV_OK) return s;
+  CUDA_TRY(wait_probe_launch(st->dev.err, limit_ns, static_cast<cudaStream_t>(stream)));
+  return STARKV_OK;
+}
+
 starkv_status starkv_set_timing(starkv_state* st, int32_t on) {
   if (!st) return set_error(STARKV_ERR_INVALID_ARG, "state is NULL");
   st->timing = on != 0;

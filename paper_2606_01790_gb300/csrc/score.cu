@@ -52,6 +52,14 @@ constexpr int kEpiThreads = 32 * kEpiWarps;
 constexpr uint32_t kFull = 0xffffffffu;
 constexpr int kXOnesBytes = 256;              // pass 2: the ones operand (two 8 x 16 B core matrices)
 constexpr int kXRowBytes = 32;                // pass 2: one window row of the -lse operand (16 bf16)
+// Limit of the waits for copies and MMAs this CTA has already issued, before
+// it exits or releases TMEM: those complete in microseconds, so the limit only
+// guards against a broken memory system, whatever the configured wait limit.
+constexpr uint64_t kDrainWaitNs = 2000000000ull;
+
+__device__ __forceinline__ uint64_t drain_limit(uint64_t wait_ns) {
+  return wait_ns > kDrainWaitNs ? wait_ns : kDrainWaitNs;
+}
 
 struct TileCoord {
   int s, l, g, j;
@@ -200,8 +208,8 @@ __device__ void producer_loop(const ScoreParams& p, SmemCtl* ctl, uint8_t* sQ, u
   if (ctl->abort) {
     // bring every issued copy to completion before the CTA can exit
     for (int i = 0; i < p.kstages; ++i)
-      if (last_ph[i] >= 0) mbar_wait(&ctl->k_full[i], last_ph[i], p.wait_ns);
-    if (last_q_pc >= 0) mbar_wait(&ctl->q_full, last_q_pc & 1, p.wait_ns);
+      if (last_ph[i] >= 0) mbar_wait(&ctl->k_full[i], last_ph[i], drain_limit(p.wait_ns));
+    if (last_q_pc >= 0) mbar_wait(&ctl->q_full, last_q_pc & 1, drain_limit(p.wait_ns));
   }
 }
 
@@ -284,7 +292,7 @@ __device__ void mma_loop(const ScoreParams& p, SmemCtl* ctl, const uint8_t* sQ, 
   }
   // every MMA issued above must be complete before TMEM is released
   mma_commit(&ctl->drain);
-  mbar_wait(&ctl->drain, 0, p.wait_ns);
+  mbar_wait(&ctl->drain, 0, drain_limit(p.wait_ns));
 }
 
 // log2-domain log-sum-exp of window row `col` of the (seq, layer, group) row
@@ -741,6 +749,22 @@ cudaError_t pool_launch(const SeqBatch& b, int G, int H, int pool, int lp_max, c
   if (lp_max <= 0) return cudaSuccess;
   dim3 grid(ceil_div(lp_max, 256), b.nlayers * G, b.nseq);
   return launch_pdl(k_pool, grid, dim3(256), 0, stream, b, G, H, pool);
+}
+
+// Self-test of the failure path that every bounded wait above shares: one
+// thread waits on a shared-memory barrier that nothing arrives on; the wait
+// gives up after `limit_ns`, latches the timeout code and the kernel returns.
+__global__ void k_wait_probe(uint32_t* err, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  fence_mbar_init();
+  if (!mbar_wait(&bar, 0, limit_ns)) atomicOr(err, kErrTimeout);
+}
+
+cudaError_t wait_probe_launch(uint32_t* err, uint64_t limit_ns, cudaStream_t stream) {
+  k_wait_probe<<<1, 32, 0, stream>>>(err, limit_ns);
+  return cudaGetLastError();
 }
 
 }  // namespace starkv

@@ -41,5 +41,6 @@ cudaError_t score_configure();
 cudaError_t score_lse_launch(const ScoreParams& p, int grid, cudaStream_t stream);
 cudaError_t score_accum_launch(const ScoreParams& p, int grid, cudaStream_t stream);
 cudaError_t pool_launch(const SeqBatch& b, int G, int H, int pool, int lp_max, cudaStream_t stream);
+cudaError_t wait_probe_launch(uint32_t* err, uint64_t limit_ns, cudaStream_t stream);
 
 }  // namespace starkv

@@ -25,7 +25,7 @@ ABI_FUNCTIONS = [
     "starkv_get_config", "starkv_workspace_bytes", "starkv_score_layer", "starkv_select",
     "starkv_compact", "starkv_step", "starkv_step_host", "starkv_check_device_error",
     "starkv_set_wait_limit", "starkv_set_timing", "starkv_kernel_times", "starkv_last_error",
-    "starkv_score_layer_noalloc",
+    "starkv_score_layer_noalloc", "starkv_selftest_wait",
 ]
 
 KERNELS = ["score_lse", "score_accum", "pool", "calibrate", "compact"]
@@ -86,6 +86,7 @@ def lib() -> C.CDLL:
                                              C.POINTER(C.c_size_t)]
         L.starkv_check_device_error.argtypes = [st, C.c_void_p]
         L.starkv_set_wait_limit.argtypes = [st, C.c_uint64]
+        L.starkv_selftest_wait.argtypes = [st, C.c_uint64, C.c_void_p]
         L.starkv_set_timing.argtypes = [st, C.c_int32]
         L.starkv_kernel_times.argtypes = [st, C.POINTER(C.c_int64), C.POINTER(C.c_float)]
         L.starkv_last_error.argtypes = []
@@ -270,6 +271,13 @@ def reset_seq(st: State, slot: int, stream=None) -> None:
 
 def set_wait_limit(st: State, limit_ns: int) -> None:
     _check(lib().starkv_set_wait_limit(st.handle, int(limit_ns)))
+
+
+def selftest_wait(st: State, limit_ns: int, stream=None) -> None:
+    """Runs the bounded-wait failure path once: a device wait that nothing
+    completes gives up after ``limit_ns`` and latches ERR_TIMEOUT, which the
+    next ``check_device_error`` raises."""
+    _check(lib().starkv_selftest_wait(st.handle, int(limit_ns), _stream(stream)))
 
 
 def workspace_bytes(st: State, seqs: Sequence[Seq], host: bool = False) -> int:

@@ -84,3 +84,7 @@ def test_meta_packing_roundtrip():
     assert r2[1:].tolist() == row[1:].tolist() and c2[1:].tolist() == col[1:].tolist()
     with pytest.raises(ValueError):
         sk.pack_meta([1], [4096], [0], [0])
+
+
+def test_wait_selftest_checks_its_arguments_on_the_host(library):
+    assert library.starkv_selftest_wait(None, 1000000, None) == sk.ERR_INVALID_ARG
