@@ -199,6 +199,42 @@ starkv_status starkv_reset_seq(starkv_state* st, int32_t slot, void* stream);
 /* Frees the state (synchronises the device first).  NULL is accepted. */
 starkv_status starkv_destroy_state(starkv_state* st);
 
+/* Checkpoint / resume of one slot's carried state (the step counters n, the
+ * MI EMAs MI_bar of Eq. 6 and the temporal EMAs m_g of Eq. 8 of every layer),
+ * e.g. to continue a trajectory in another process or on another device.
+ * Host buffer layout, STARKV_SLOT_STATE_BYTES(n_layers, G, R*C) bytes:
+ *   starkv_slot_header (32 B), then
+ *   int32  n[n_layers]                 padded to a multiple of 8 bytes
+ *   f64    mi_bar[n_layers][G]
+ *   f32    m[n_layers][G][R*C]
+ * The header records the shape; an import whose header does not match the
+ * state's (magic, version, n_layers, G, R, C) or whose buffer is too small is
+ * rejected with STARKV_ERR_INVALID_ARG before any copy. */
+typedef struct {
+  uint32_t magic;       /* STARKV_SLOT_MAGIC */
+  uint32_t version;     /* 1 */
+  int32_t n_layers, n_kv_heads, grid_rows, grid_cols;
+  uint32_t reserved[2]; /* zero */
+} starkv_slot_header;
+
+#define STARKV_SLOT_MAGIC 0x31564B53u   /* "SKV1" */
+#define STARKV_SLOT_STATE_BYTES(n_layers, G, RC)                              \
+  (sizeof(starkv_slot_header) + (((size_t)(n_layers) * 4 + 7) & ~(size_t)7) + \
+   (size_t)(n_layers) * (G) * 8 + (size_t)(n_layers) * (G) * (RC) * 4)
+
+/* Bytes of one slot's exported state for this state's shape. */
+starkv_status starkv_slot_state_bytes(const starkv_state* st, size_t* bytes);
+
+/* Writes slot `slot`'s state into the HOST buffer `host` (>= the size above):
+ * the header at once, the arrays by stream-ordered copies (valid after the
+ * stream is synchronised; page-locked memory keeps them asynchronous). */
+starkv_status starkv_export_slot(starkv_state* st, int32_t slot, void* host, size_t bytes, void* stream);
+
+/* Replaces slot `slot`'s state with the one in the HOST buffer `host`, written
+ * by starkv_export_slot for the same shape (stream-ordered copies; the buffer
+ * may be reused once the stream has passed them). */
+starkv_status starkv_import_slot(starkv_state* st, int32_t slot, const void* host, size_t bytes, void* stream);
+
 /* Copies the config the state was created with. */
 starkv_status starkv_get_config(const starkv_state* st, starkv_config* out);
 

@@ -559,6 +559,100 @@ starkv_status starkv_destroy_state(starkv_state* st) {
   return STARKV_OK;
 }
 
+starkv_status starkv_slot_state_bytes(const starkv_state* st, size_t* bytes) {
+  if (!st || !bytes) return set_error(STARKV_ERR_INVALID_ARG, "NULL state or output pointer");
+  const starkv_config& c = st->cfg;
+  *bytes = STARKV_SLOT_STATE_BYTES(c.n_layers, c.n_kv_heads, static_cast<size_t>(c.grid_rows) * c.grid_cols);
+  return STARKV_OK;
+}
+
+namespace {
+
+// Offsets of the three arrays of one slot in an exported buffer, and their
+// sources in the device state.
+struct SlotLayout {
+  size_t o_n, o_mi, o_m, n_bytes, mi_bytes, m_bytes;
+  int32_t* dn;
+  double* dmi;
+  float* dm;
+};
+
+SlotLayout slot_layout(const starkv_state* st, int slot) {
+  const starkv_config& c = st->cfg;
+  const size_t L = c.n_layers, G = c.n_kv_heads, RC = static_cast<size_t>(c.grid_rows) * c.grid_cols;
+  SlotLayout s;
+  s.n_bytes = L * sizeof(int32_t);
+  s.mi_bytes = L * G * sizeof(double);
+  s.m_bytes = L * G * RC * sizeof(float);
+  s.o_n = sizeof(starkv_slot_header);
+  s.o_mi = s.o_n + ((s.n_bytes + 7) & ~static_cast<size_t>(7));
+  s.o_m = s.o_mi + s.mi_bytes;
+  s.dn = st->dev.n + slot * L;
+  s.dmi = st->dev.mi_bar + slot * L * G;
+  s.dm = st->dev.m + slot * L * G * RC;
+  return s;
+}
+
+starkv_status check_slot_buffer(const starkv_state* st, int slot, const void* host, size_t bytes) {
+  if (!st) return set_error(STARKV_ERR_INVALID_ARG, "state is NULL");
+  if (!host) return set_error(STARKV_ERR_INVALID_ARG, "host buffer is NULL");
+  if (slot < 0 || slot >= st->cfg.max_seqs) return set_error(STARKV_ERR_INVALID_ARG, "slot out of range");
+  size_t need = 0;
+  starkv_slot_state_bytes(st, &need);
+  if (bytes < need) return set_error(STARKV_ERR_INVALID_ARG, "slot buffer of %zu bytes, %zu needed", bytes, need);
+  if (reinterpret_cast<uintptr_t>(host) & 7) return set_error(STARKV_ERR_INVALID_ARG, "slot buffer not 8-byte aligned");
+  return STARKV_OK;
+}
+
+}  // namespace
+
+starkv_status starkv_export_slot(starkv_state* st, int32_t slot, void* host, size_t bytes, void* stream) {
+  starkv_status s = check_slot_buffer(st, slot, host, bytes);
+  if (s != STARKV_OK) return s;
+  if ((s = check_device(st)) != STARKV_OK) return s;
+  const starkv_config& c = st->cfg;
+  starkv_slot_header h;
+  memset(&h, 0, sizeof(h));
+  h.magic = STARKV_SLOT_MAGIC;
+  h.version = 1;
+  h.n_layers = c.n_layers;
+  h.n_kv_heads = c.n_kv_heads;
+  h.grid_rows = c.grid_rows;
+  h.grid_cols = c.grid_cols;
+  char* b = static_cast<char*>(host);
+  memcpy(b, &h, sizeof(h));
+  const SlotLayout l = slot_layout(st, slot);
+  memset(b + l.o_n + l.n_bytes, 0, l.o_mi - l.o_n - l.n_bytes);   // padding
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  CUDA_TRY(cudaMemcpyAsync(b + l.o_n, l.dn, l.n_bytes, cudaMemcpyDeviceToHost, cs));
+  CUDA_TRY(cudaMemcpyAsync(b + l.o_mi, l.dmi, l.mi_bytes, cudaMemcpyDeviceToHost, cs));
+  CUDA_TRY(cudaMemcpyAsync(b + l.o_m, l.dm, l.m_bytes, cudaMemcpyDeviceToHost, cs));
+  return STARKV_OK;
+}
+
+starkv_status starkv_import_slot(starkv_state* st, int32_t slot, const void* host, size_t bytes, void* stream) {
+  starkv_status s = check_slot_buffer(st, slot, host, bytes);
+  if (s != STARKV_OK) return s;
+  if ((s = check_device(st)) != STARKV_OK) return s;
+  const starkv_config& c = st->cfg;
+  starkv_slot_header h;
+  memcpy(&h, host, sizeof(h));
+  if (h.magic != STARKV_SLOT_MAGIC || h.version != 1)
+    return set_error(STARKV_ERR_INVALID_ARG, "not an exported slot state (magic / version)");
+  if (h.n_layers != c.n_layers || h.n_kv_heads != c.n_kv_heads || h.grid_rows != c.grid_rows ||
+      h.grid_cols != c.grid_cols)
+    return set_error(STARKV_ERR_INVALID_ARG, "slot state of shape (layers %d, G %d, grid %d x %d), state has (%d, %d, %d x %d)",
+                     h.n_layers, h.n_kv_heads, h.grid_rows, h.grid_cols, c.n_layers, c.n_kv_heads, c.grid_rows,
+                     c.grid_cols);
+  const char* b = static_cast<const char*>(host);
+  const SlotLayout l = slot_layout(st, slot);
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  CUDA_TRY(cudaMemcpyAsync(l.dn, b + l.o_n, l.n_bytes, cudaMemcpyHostToDevice, cs));
+  CUDA_TRY(cudaMemcpyAsync(l.dmi, b + l.o_mi, l.mi_bytes, cudaMemcpyHostToDevice, cs));
+  CUDA_TRY(cudaMemcpyAsync(l.dm, b + l.o_m, l.m_bytes, cudaMemcpyHostToDevice, cs));
+  return STARKV_OK;
+}
+
 starkv_status starkv_get_config(const starkv_state* st, starkv_config* out) {
   if (!st || !out) return set_error(STARKV_ERR_INVALID_ARG, "NULL argument");
   *out = st->cfg;

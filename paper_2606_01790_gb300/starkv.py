@@ -25,7 +25,8 @@ ABI_FUNCTIONS = [
     "starkv_get_config", "starkv_workspace_bytes", "starkv_score_layer", "starkv_select",
     "starkv_compact", "starkv_step", "starkv_step_host", "starkv_check_device_error",
     "starkv_set_wait_limit", "starkv_set_timing", "starkv_kernel_times", "starkv_last_error",
-    "starkv_score_layer_noalloc", "starkv_selftest_wait",
+    "starkv_score_layer_noalloc", "starkv_selftest_wait", "starkv_slot_state_bytes", "starkv_export_slot",
+    "starkv_import_slot",
 ]
 
 KERNELS = ["score_lse", "score_accum", "pool", "calibrate", "compact"]
@@ -61,6 +62,21 @@ class CSeq(C.Structure):
 _lib: Optional[C.CDLL] = None
 
 
+class CSlotHeader(C.Structure):
+    """``starkv_slot_header``: the first 32 bytes of an exported slot state."""
+    _fields_ = [("magic", C.c_uint32), ("version", C.c_uint32), ("n_layers", C.c_int32),
+                ("n_kv_heads", C.c_int32), ("grid_rows", C.c_int32), ("grid_cols", C.c_int32),
+                ("reserved", C.c_uint32 * 2)]
+
+
+SLOT_MAGIC = 0x31564B53
+
+
+def slot_state_bytes_for(n_layers: int, G: int, RC: int) -> int:
+    """STARKV_SLOT_STATE_BYTES of the header."""
+    return C.sizeof(CSlotHeader) + ((n_layers * 4 + 7) & ~7) + n_layers * G * 8 + n_layers * G * RC * 4
+
+
 def lib() -> C.CDLL:
     """The loaded library (raises if it has not been built)."""
     global _lib
@@ -87,6 +103,9 @@ def lib() -> C.CDLL:
         L.starkv_check_device_error.argtypes = [st, C.c_void_p]
         L.starkv_set_wait_limit.argtypes = [st, C.c_uint64]
         L.starkv_selftest_wait.argtypes = [st, C.c_uint64, C.c_void_p]
+        L.starkv_slot_state_bytes.argtypes = [st, C.POINTER(C.c_size_t)]
+        L.starkv_export_slot.argtypes = [st, C.c_int32, C.c_void_p, C.c_size_t, C.c_void_p]
+        L.starkv_import_slot.argtypes = [st, C.c_int32, C.c_void_p, C.c_size_t, C.c_void_p]
         L.starkv_set_timing.argtypes = [st, C.c_int32]
         L.starkv_kernel_times.argtypes = [st, C.POINTER(C.c_int64), C.POINTER(C.c_float)]
         L.starkv_last_error.argtypes = []
@@ -271,6 +290,30 @@ def reset_seq(st: State, slot: int, stream=None) -> None:
 
 def set_wait_limit(st: State, limit_ns: int) -> None:
     _check(lib().starkv_set_wait_limit(st.handle, int(limit_ns)))
+
+
+def slot_state_bytes(st: State) -> int:
+    n = C.c_size_t(0)
+    _check(lib().starkv_slot_state_bytes(st.handle, C.byref(n)))
+    return int(n.value)
+
+
+def export_slot(st: State, slot: int, out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Slot ``slot``'s carried state (n, MI EMA, m_g of every layer) as a uint8
+    host tensor (page-locked unless ``out`` is given); valid once the stream
+    has been synchronised."""
+    n = slot_state_bytes(st)
+    if out is None:
+        out = torch.empty(n, dtype=torch.uint8, pin_memory=torch.cuda.is_available())
+    _check(lib().starkv_export_slot(st.handle, int(slot), out.data_ptr(), out.numel() * out.element_size(),
+                                    _stream(stream)))
+    return out
+
+
+def import_slot(st: State, slot: int, buf: torch.Tensor, stream=None) -> None:
+    """Replaces slot ``slot``'s carried state with one written by ``export_slot``."""
+    _check(lib().starkv_import_slot(st.handle, int(slot), buf.data_ptr(), buf.numel() * buf.element_size(),
+                                    _stream(stream)))
 
 
 def selftest_wait(st: State, limit_ns: int, stream=None) -> None:

@@ -88,3 +88,36 @@ def test_meta_packing_roundtrip():
 
 def test_wait_selftest_checks_its_arguments_on_the_host(library):
     assert library.starkv_selftest_wait(None, 1000000, None) == sk.ERR_INVALID_ARG
+
+
+def test_header_compiles_as_c_and_its_layouts_match_the_binding(tmp_path):
+    """The header alone, compiled by the host C compiler: struct sizes, the
+    slot-state size macro and the constants, against the ctypes mirror."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "probe.c"
+    src.write_text(
+        '#include <stdio.h>\n#include "starkv.h"\n'
+        "int main(void) {\n"
+        '  printf("%zu %zu %zu %zu %u %d\\n", sizeof(starkv_config), sizeof(starkv_seq),\n'
+        "         sizeof(starkv_slot_header), (size_t)STARKV_SLOT_STATE_BYTES(28, 4, 2704),\n"
+        "         (unsigned)STARKV_SLOT_MAGIC, (int)STARKV_STATS_STRIDE(4));\n"
+        "  return 0;\n}\n")
+    exe = tmp_path / "probe"
+    subprocess.run([cc, "-std=c99", "-Wall", "-Werror", f"-I{ROOT / 'include'}", str(src), "-o", str(exe)],
+                   check=True, capture_output=True)
+    got = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()
+    want = [ctypes.sizeof(sk.CConfig), ctypes.sizeof(sk.CSeq), ctypes.sizeof(sk.CSlotHeader),
+            sk.slot_state_bytes_for(28, 4, 2704), sk.SLOT_MAGIC, sk.stats_stride(4)]
+    assert [int(x) for x in got] == want
+
+
+def test_slot_calls_check_their_arguments_on_the_host(library):
+    n = ctypes.c_size_t(0)
+    assert library.starkv_slot_state_bytes(None, ctypes.byref(n)) == sk.ERR_INVALID_ARG
+    buf = (ctypes.c_uint8 * 64)()
+    assert library.starkv_export_slot(None, 0, buf, 64, None) == sk.ERR_INVALID_ARG
+    assert library.starkv_import_slot(None, 0, buf, 64, None) == sk.ERR_INVALID_ARG
