@@ -3,6 +3,7 @@
 // sequencing.  All arithmetic of the method runs in the kernels of score.cu,
 // select.cu and compact.cu.
 #include <cudaTypedefs.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <algorithm>
 #include <cmath>
@@ -112,8 +113,29 @@ cudaEvent_t take_event(starkv_state* st) {
 
 // Launches one kernel kind through `fn`, counting it and, when timing is on,
 // bracketing it with an event pair on `stream`.
+// NVTX ranges name each host-side enqueue for a profiler's timeline (no cost
+// unless a tool is attached; NVTX v3 is header-only).
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
+const char* kernel_range_name(int kind) {
+  switch (kind) {
+    case STARKV_KERNEL_SCORE_LSE: return "starkv: scoring pass 1 (row LSE)";
+    case STARKV_KERNEL_SCORE_ACCUM: return "starkv: scoring pass 2 (group sums)";
+    case STARKV_KERNEL_POOL: return "starkv: pooling";
+    case STARKV_KERNEL_CALIBRATE: return "starkv: calibration + top-B";
+    case STARKV_KERNEL_COMPACT: return "starkv: compaction";
+    default: return "starkv: kernel";
+  }
+}
+
 template <typename F>
 cudaError_t launch(starkv_state* st, int kind, cudaStream_t stream, F&& fn) {
+  NvtxRange range(kernel_range_name(kind));
   st->launches[kind] += 1;
   if (!st->timing) return fn();
   starkv_state::Rec r{kind, take_event(st), take_event(st)};
@@ -722,6 +744,7 @@ starkv_status starkv_compact(starkv_state* st, int32_t layer, const starkv_seq* 
 
 starkv_status starkv_step(starkv_state* st, const starkv_seq* seqs, int32_t nseq, void* workspace,
                           size_t workspace_bytes, void* stream) {
+  NvtxRange range("starkv_step");
   starkv_status s = validate_seqs(st, seqs, nseq, kNeedK | kNeedQ | kNeedV | kNeedMeta | kNeedIdx | kNeedOut);
   if (s != STARKV_OK) return s;
   if ((s = check_device(st)) != STARKV_OK) return s;
@@ -731,6 +754,7 @@ starkv_status starkv_step(starkv_state* st, const starkv_seq* seqs, int32_t nseq
 
 starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t nseq, void* workspace,
                                size_t workspace_bytes, void* stream) {
+  NvtxRange range("starkv_step_host");
   starkv_status s = validate_seqs(st, seqs, nseq, kNeedK | kNeedQ | kNeedV | kNeedMeta | kNeedIdx | kNeedOut);
   if (s != STARKV_OK) return s;
   if ((s = check_device(st)) != STARKV_OK) return s;
