@@ -153,7 +153,7 @@ starkv_status validate_config(const starkv_config& c) {
     return set_error(STARKV_ERR_INVALID_ARG, "config: n_layers, n_heads, n_kv_heads, window, max_seqs must be >= 1");
   if (c.head_dim != kHeadDim) return set_error(STARKV_ERR_UNSUPPORTED, "config: head_dim must be 128");
   if (c.n_heads % c.n_kv_heads) return set_error(STARKV_ERR_UNSUPPORTED, "config: n_heads %% n_kv_heads != 0");
-  if (c.n_kv_heads > kMaxGroups) return set_error(STARKV_ERR_UNSUPPORTED, "config: n_kv_heads > 8");
+  if (c.n_kv_heads > kMaxGroups) return set_error(STARKV_ERR_UNSUPPORTED, "config: n_kv_heads > 32");
   if ((c.n_heads / c.n_kv_heads) * c.window > kMaxRows)
     return set_error(STARKV_ERR_UNSUPPORTED, "config: (H/G)*w > 256");
   if (c.grid_rows < 1 || c.grid_cols < 1 || c.grid_rows > 1024 || c.grid_cols > 1024 ||
@@ -170,6 +170,8 @@ starkv_status validate_config(const starkv_config& c) {
     return set_error(STARKV_ERR_INVALID_ARG, "config: decay_mode in 0..2, aeb_mode and mi_span in 0..1");
   if (c.select_mode != STARKV_SELECT_GLOBAL && c.select_mode != STARKV_SELECT_PER_HEAD)
     return set_error(STARKV_ERR_INVALID_ARG, "config: select_mode must be 0 (global) or 1 (per KV head)");
+  if (c.select_mode == STARKV_SELECT_PER_HEAD && c.n_kv_heads > kMaxCluster)
+    return set_error(STARKV_ERR_UNSUPPORTED, "config: the per-KV-head mode takes n_kv_heads <= 8");
   if (!(c.rho_mi >= 0.f && c.rho_mi <= 1.f) || !(c.rho_t >= 0.f && c.rho_t <= 1.f) ||
       !(c.d_min >= 0.f && c.d_min <= 1.f) || !(c.eps >= 0.f) || !(c.eps_h >= 0.f) || !(c.delta >= 0.f))
     return set_error(STARKV_ERR_INVALID_ARG, "config: a rate or epsilon is out of range");

@@ -13,7 +13,8 @@ namespace starkv {
 constexpr int kHeadDim = 128;       // d
 constexpr int kTileKeys = 128;      // keys per MMA tile (M of pass 2, N of pass 1)
 constexpr int kMaxRows = 256;       // (H / G) * w window rows per group
-constexpr int kMaxGroups = 8;       // G
+constexpr int kMaxGroups = 32;      // G (KV heads; the global mode up to one per query head)
+constexpr int kMaxCluster = 8;      // CTAs of a calibration cluster (portable cluster size)
 constexpr int kMaxBatch = 32;       // sequences per launch (kernel-parameter arrays)
 constexpr int kMaxBins = 64;        // K rank bins
 constexpr int kMaxHist = 4096;      // K * M^2

@@ -137,18 +137,18 @@ struct CalShared {
   int nb[16];                     // rank-bin marginals
   int scan[33];
   float fred[32];
-  double mib_old[kMaxGroups];     // MI EMA before this step
+  double mib_old[kMaxGroups];     // MI EMA before this step, per group
   float w[kMaxGroups], ph[kMaxGroups];
   float lam;
   int n_old;
   int any_tie;
   float fredn[4][32];             // multi-value block reductions
   uint32_t uredn[3][32];
-  float pz[kMaxGroups], pzl[kMaxGroups], pv[kMaxGroups];   // every CTA's phase-2 partials
-  uint32_t pkmin[kMaxGroups], pkmax[kMaxGroups], psmax[kMaxGroups];
-  int pncand[kMaxGroups], pbelow[kMaxGroups];
+  float pz[kMaxCluster], pzl[kMaxCluster], pv[kMaxCluster];   // every CTA's phase-2 partials
+  uint32_t pkmin[kMaxCluster], pkmax[kMaxCluster], psmax[kMaxCluster];
+  int pncand[kMaxCluster], pbelow[kMaxCluster];
   // read by the other CTAs of the cluster
-  float mi, phi;                  // this CTA's group (phase 1)
+  float mi[kMaxGroups / kMaxCluster], phi[kMaxGroups / kMaxCluster];   // this CTA's groups (phase 1)
   float zpart, hpart, vpart;      // this CTA's token range (phase 2)
   uint32_t kminp, kmaxp, smaxp;
   int tcand, nbelow;              // top-B boundary-bucket candidates, tokens below it
@@ -188,13 +188,13 @@ __device__ void block_reduce(float (&v)[NF], uint32_t& mn, uint32_t& mx, CalShar
 // Sum of the int4 at `p` over the CTAs [r_lo, r_hi) of the cluster: every
 // remote load is issued before the first add.
 __device__ __forceinline__ int4 sum_peers_v4(const int* p, int r_lo, int r_hi) {
-  int4 q[kMaxGroups];
+  int4 q[kMaxCluster];
 #pragma unroll
-  for (int r = 0; r < kMaxGroups; ++r)
+  for (int r = 0; r < kMaxCluster; ++r)
     if (r < r_hi - r_lo) q[r] = dsmem_ld_v4(dsmem_map(p, r_lo + r));
   int4 h = make_int4(0, 0, 0, 0);
 #pragma unroll
-  for (int r = 0; r < kMaxGroups; ++r)
+  for (int r = 0; r < kMaxCluster; ++r)
     if (r < r_hi - r_lo) {
       h.x += q[r].x;
       h.y += q[r].y;
@@ -326,18 +326,20 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   uint16_t* scells = reinterpret_cast<uint16_t*>(scand + capl);
 
   const SeqView& sv = b.s[blockIdx.z];
-  const int g = blockIdx.x;              // == rank in the cluster (the cluster spans grid x)
+  // the cluster spans grid x: one CTA per group, or kMaxCluster CTAs when G is
+  // larger (global mode), CTA `rank` then taking groups rank, rank + ncta, ...
+  const int rank = blockIdx.x, ncta = gridDim.x;
   const int ll = blockIdx.y, layer = b.layer0 + ll;
   const int Lp = sv.Lp;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  // this group's metadata row (the one shared row when meta_group_stride is 0)
-  const uint32_t* meta = sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride + g * sv.meta_group_stride;
   const int sl = sv.slot * kp.n_layers + layer;
-  float* S = sv.S + (static_cast<int64_t>(layer) * G + g) * Lp;
   const bool in_smem = Lp <= capl;
-  uint32_t* keys = in_smem ? skeys : sv.vis + static_cast<int64_t>(ll * G + g) * Lp * 3;
-  uint32_t* cand = in_smem ? scand : keys + Lp;
-  uint16_t* cells = in_smem ? scells : reinterpret_cast<uint16_t*>(keys + 2 * static_cast<int64_t>(Lp));
+  // metadata row of group gi (the one shared row when meta_group_stride is 0)
+  auto meta_of = [&](int gi) {
+    return sv.meta + static_cast<int64_t>(layer) * sv.meta_layer_stride + gi * sv.meta_group_stride;
+  };
+  // the per-token arrays of row r: shared memory, or row r's workspace region
+  auto keys_of = [&](int r) { return in_smem ? skeys : sv.vis + static_cast<int64_t>(ll * G + r) * Lp * 3; };
   // phase 1 walks the row in one contiguous segment per warp, so that warp
   // order and lane order are position order
   const int seg = ceil_div(Lp, 32 * 32) * 32;
@@ -349,9 +351,10 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   for (int i = tid; i < RC; i += kCalThreads) cur[i] = 0.f;
   for (int r = tid; r < R; r += kCalThreads) rowc[r] = static_cast<uint8_t>(r * M / R);
   for (int c = tid; c < C; c += kCalThreads) colc[c] = static_cast<uint8_t>(c * M / C);
-  // this group's temporal EMA row (state of the previous step, read after
-  // phase 1) on its way into L2
-  if (tid * 32 < RC) prefetch_l2(st.m + static_cast<int64_t>(sl * G + g) * RC + tid * 32);
+  // this CTA's groups' temporal EMA rows (state of the previous step, read
+  // after phase 1) on their way into L2
+  for (int gi = rank; gi < G; gi += ncta)
+    if (tid * 32 < RC) prefetch_l2(st.m + static_cast<int64_t>(sl * G + gi) * RC + tid * 32);
   __syncthreads();
   // the set-up above overlaps the previous kernel's tail; its outputs are read below
   griddep_launch_dependents();
@@ -359,7 +362,13 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   if (tid < G) sh.mib_old[tid] = st.mi_bar[sl * G + tid];
   if (tid == 0) sh.n_old = st.n[sl];
 
-  // ================= phase 1: group g =================
+  // ================= phase 1: groups rank, rank + ncta, ... =================
+  for (int g = rank, gl = 0; g < G; g += ncta, ++gl) {
+  const uint32_t* meta = meta_of(g);
+  float* S = sv.S + (static_cast<int64_t>(layer) * G + g) * Lp;
+  uint32_t* keys = keys_of(g);
+  uint32_t* cand = in_smem ? scand : keys + Lp;
+  uint16_t* cells = in_smem ? scells : reinterpret_cast<uint16_t*>(keys + 2 * static_cast<int64_t>(Lp));
   // ---- the row, staged in shared memory by one pass of independent loads:
   // the unpooled sums (the four column-quarter copies added in order) or the
   // given S, into the candidate region; the metadata words into the key region
@@ -745,31 +754,46 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     }
   }
   if (tid == 0) {
-    sh.mi = mi;
-    sh.phi = phi;
+    sh.mi[gl] = mi;
+    sh.phi[gl] = phi;
     st.mi_cur[sl * G + g] = mi;
     st.phi_cur[sl * G + g] = phi;
   }
+  if (g + ncta < G) {   // the next group of this CTA starts from clean arrays
+    __syncthreads();
+    if (tid == 0) sh.any_tie = 0;
+    for (int i = tid; i < kBins0; i += kCalThreads) hist[i] = 0;
+    for (int i = tid; i < K * MM; i += kCalThreads) joint[i] = 0;
+    for (int i = tid; i < RC; i += kCalThreads) cur[i] = 0.f;
+    __syncthreads();
+  }
+  }   // phase-1 group loop
   for (int i = tid; i < kBins0; i += kCalThreads) hist[i] = 0;   // top-B digit 1 (below)
   cluster_sync();   // every group's S row, MI_g and phi_g are complete
 
   // ================= phase 2 =================
-  // global mode: CTA r scores and selects tokens [r Lp / G, (r + 1) Lp / G) of
-  // s_bar; per-KV-head mode: CTA g its own row S[g, .]
+  // global mode: CTA r scores and selects tokens [r Lp / ncta, (r + 1) Lp / ncta)
+  // of s_bar; per-KV-head mode (one CTA per group): CTA g its own row S[g, .]
   const bool per_head = kp.per_head != 0;
+  const int g = rank;   // per-KV-head mode: this CTA's group
+  const uint32_t* meta = meta_of(per_head ? g : 0);
+  uint32_t* keys = keys_of(rank);
+  uint32_t* cand = in_smem ? scand : keys + Lp;
   float* stats = sv.stats ? sv.stats + static_cast<int64_t>(layer) * (8 + 6 * G) : nullptr;
   // ---- Eqs. (6)-(7): MI EMA (double state), min-max, softmax prior; lambda
   // schedule.  The same arithmetic in every CTA; CTA 0 stores the new state.
-  // warp 0, lane gg < G: group gg's MI (from CTA gg), its EMA, then the
-  // min-max and the softmax over the groups by warp reductions
+  // warp 0, lane gg < G: group gg's MI (from CTA gg % ncta), its EMA, then
+  // the min-max and the softmax over the groups by warp reductions
+  static_assert(kMaxGroups <= 32, "one lane per group");
   if (warp == 0) {
     const int n = sh.n_old;
     const bool on = lane < G;
     double mib = 0.0;
     float mic = 0.f, mf = 0.f;
     if (on) {
-      mic = dsmem_ld_f32(dsmem_map(&sh.mi, lane));
-      sh.ph[lane] = dsmem_ld_f32(dsmem_map(&sh.phi, lane));
+      const int owner = lane % ncta, slot = lane / ncta;
+      mic = dsmem_ld_f32(dsmem_map(&sh.mi[slot], owner));
+      sh.ph[lane] = dsmem_ld_f32(dsmem_map(&sh.phi[slot], owner));
       mib = n == 0 ? static_cast<double>(mic)
                    : kp.rho_mi * sh.mib_old[lane] + (1.0 - kp.rho_mi) * static_cast<double>(mic);
       mf = static_cast<float>(mib);
@@ -794,7 +818,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       lam = kp.n_ramp <= 0 ? kp.lambda
                            : kp.lambda * fminf(1.f, static_cast<float>(n - kp.n_warmup) / kp.n_ramp);
     if (lane == 0) sh.lam = lam;
-    if (g == 0) {
+    if (rank == 0) {
       if (on) st.mi_bar[sl * G + lane] = mib;
       if (lane == 0) st.n[sl] = n + 1;
       if (stats) {
@@ -816,11 +840,11 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   __syncthreads();   // w and lambda are read by every thread below
   // (range boundaries on multiples of 4 tokens, so that the ranges can be read in 16 bytes)
   auto split = [&](int r) {
-    const int64_t t = (static_cast<int64_t>(r) * Lp / G + 3) & ~static_cast<int64_t>(3);
+    const int64_t t = (static_cast<int64_t>(r) * Lp / ncta + 3) & ~static_cast<int64_t>(3);
     return static_cast<int>(t < Lp ? t : Lp);
   };
-  const int ta = per_head ? 0 : split(g);
-  const int tb = per_head ? Lp : split(g + 1);
+  const int ta = per_head ? 0 : split(rank);
+  const int tb = per_head ? Lp : split(rank + 1);
   const int nr = tb - ta;
   const float* S0 = sv.S + static_cast<int64_t>(layer) * G * Lp;
   const float invG = 1.f / static_cast<float>(G);
@@ -886,9 +910,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       const uint4 m4 = *reinterpret_cast<const uint4*>(meta + t);
       float4 acc = *reinterpret_cast<const float4*>(S0 + t), best = acc;
       int gs[4] = {0, 0, 0, 0};
-#pragma unroll
-      for (int gg = 1; gg < kMaxGroups; ++gg) {
-        if (gg >= G) break;
+      auto take = [&](int gg) {
         const float4 q = *reinterpret_cast<const float4*>(S0 + static_cast<int64_t>(gg) * Lp + t);
         acc.x += q.x;
         acc.y += q.y;
@@ -898,6 +920,15 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         if (q.y > best.y) { best.y = q.y; gs[1] = gg; }
         if (q.z > best.z) { best.z = q.z; gs[2] = gg; }
         if (q.w > best.w) { best.w = q.w; gs[3] = gg; }
+      };
+      if (G <= kMaxCluster) {   // GQA: unrolled, every row's load issued up front
+#pragma unroll
+        for (int gg = 1; gg < kMaxCluster; ++gg) {
+          if (gg >= G) break;
+          take(gg);
+        }
+      } else {
+        for (int gg = 1; gg < G; ++gg) take(gg);
       }
       fuse(i0, acc.x * invG, gs[0], m4.x);
       fuse(i0 + 1, acc.y * invG, gs[1], m4.y);
@@ -905,41 +936,20 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       fuse(i0 + 3, acc.w * invG, gs[3], m4.w);
     }
   } else {
-    for (int i0 = 0; i0 < nr; i0 += 2 * kCalThreads) {
-      float v[2][kMaxGroups];
-      uint32_t mw[2];
-#pragma unroll
-      for (int k = 0; k < 2; ++k) {
-        const int i = i0 + k * kCalThreads + tid;
-        mw[k] = 0u;
-#pragma unroll
-        for (int gg = 0; gg < kMaxGroups; ++gg) v[k][gg] = 0.f;
-        if (i < nr) {
-          const int t = ta + i;
-          mw[k] = meta[t];
-#pragma unroll
-          for (int gg = 0; gg < kMaxGroups; ++gg)
-            if (gg < G) v[k][gg] = S0[static_cast<int64_t>(gg) * Lp + t];
+    for (int i = tid; i < nr; i += kCalThreads) {
+      const int t = ta + i;
+      // s_bar (Eq. 4) and its governing group g* (lowest on ties)
+      float best = S0[t], acc = best;
+      int gs = 0;
+      for (int gg = 1; gg < G; ++gg) {
+        const float v = S0[static_cast<int64_t>(gg) * Lp + t];
+        acc += v;
+        if (v > best) {
+          best = v;
+          gs = gg;
         }
       }
-#pragma unroll
-      for (int k = 0; k < 2; ++k) {
-        const int i = i0 + k * kCalThreads + tid;
-        if (i >= nr) continue;
-        // s_bar (Eq. 4) and its governing group g* (lowest on ties)
-        float best = v[k][0], acc = best;
-        int gs = 0;
-#pragma unroll
-        for (int gg = 1; gg < kMaxGroups; ++gg) {
-          if (gg >= G) break;
-          acc += v[k][gg];
-          if (v[k][gg] > best) {
-            best = v[k][gg];
-            gs = gg;
-          }
-        }
-        fuse(i, acc * invG, gs, mw[k]);
-      }
+      fuse(i, acc * invG, gs, meta[t]);
     }
   }
   {
@@ -958,7 +968,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     sh.smaxp = smx;
   }
   cluster_sync();
-  if (tid < G) {   // every CTA's partials, one peer per thread
+  if (tid < ncta) {   // every CTA's partials, one peer per thread
     sh.pz[tid] = dsmem_ld_f32(dsmem_map(&sh.zpart, tid));
     sh.pzl[tid] = dsmem_ld_f32(dsmem_map(&sh.hpart, tid));
     sh.pv[tid] = dsmem_ld_f32(dsmem_map(&sh.vpart, tid));
@@ -984,7 +994,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   if (per_head) {
     Hn = entropy(z, zl, smx);   // this CTA's own row
     T = temperature(Hn);
-    if (tid == 0 && g == 0 && stats) {
+    if (tid == 0 && rank == 0 && stats) {
       float hs = 0.f, ts = 0.f, zs = 0.f;
       for (int r = 0; r < G; ++r) {
         const float Hr = entropy(sh.pz[r], sh.pzl[r], sh.psmax[r]);
@@ -1005,7 +1015,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     uint32_t SM = 0u;
     kmin2 = 0xFFFFFFFFu;
     kmax2 = 0u;
-    for (int r = 0; r < G; ++r) {
+    for (int r = 0; r < ncta; ++r) {
       Z += sh.pz[r];
       ZL += sh.pzl[r];
       NV += sh.pv[r];
@@ -1015,7 +1025,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     }
     Hn = entropy(Z, ZL, SM);
     T = temperature(Hn);
-    if (tid == 0 && g == 0 && stats) {
+    if (tid == 0 && rank == 0 && stats) {
       stats[0] = Hn;
       stats[1] = T;
       stats[4] = Z;
@@ -1045,7 +1055,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   // cluster; per-KV-head mode: over this CTA's row, block barriers only)
   const int B = sv.budget;   // the same in every CTA of the cluster
   if (B > 0) {
-    const int r_lo = per_head ? g : 0, r_hi = per_head ? g + 1 : G;
+    const int r_lo = per_head ? g : 0, r_hi = per_head ? g + 1 : ncta;
     auto sel_sync = [&]() {
       if (per_head) __syncthreads();
       else cluster_sync();
@@ -1111,7 +1121,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         for (int j = tid; j < 2 * n; j += kCalThreads)
           all[2 * nall + j] = static_cast<uint32_t>(dsmem_ld_s32(dsmem_map(clist + j, r)));
         nall += n;
-        if (r < g) nlow += sh.pbelow[r];
+        if (r < rank) nlow += sh.pbelow[r];
       }
       __syncthreads();
       for (int i = tid; i < nall; i += kCalThreads) {
@@ -1191,12 +1201,12 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         sel_sync();
         int v = 0;
         {
-          int q[kMaxGroups];
+          int q[kMaxCluster];
 #pragma unroll
-          for (int r = 0; r < kMaxGroups; ++r)
+          for (int r = 0; r < kMaxCluster; ++r)
             if (r < r_hi - r_lo) q[r] = dsmem_ld_s32(dsmem_map(hp + tid, r_lo + r));
 #pragma unroll
-          for (int r = 0; r < kMaxGroups; ++r)
+          for (int r = 0; r < kMaxCluster; ++r)
             if (r < r_hi - r_lo) v += q[r];
         }
         const int excl = block_excl_scan(v, sh.scan, nullptr);
@@ -1224,7 +1234,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         sh.neq = tot_eq;
       }
       sel_sync();
-      for (int r = r_lo; r < g; ++r) {
+      for (int r = r_lo; r < rank; ++r) {
         lt_b += dsmem_ld_s32(dsmem_map(&sh.nlt, r));
         eq_b += dsmem_ld_s32(dsmem_map(&sh.neq, r));
       }
@@ -1265,13 +1275,14 @@ cudaError_t calibrate_launch(const SeqBatch& b, const KParams& kp, const DevStat
   const int capl = std::min(cap, (lp_max + 15) & ~15);
   const size_t smem = fixed_bytes(kp.K, kp.M, kp.R, kp.C) + static_cast<size_t>(capl) * kBytesPerToken;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(kp.G, b.nlayers, b.nseq);
+  const int ncta = std::min(kp.G, kMaxCluster);   // the per-KV-head mode has G <= kMaxCluster
+  cfg.gridDim = dim3(ncta, b.nlayers, b.nseq);
   cfg.blockDim = dim3(kCalThreads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kp.G;
+  attr[0].val.clusterDim.x = ncta;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // set-up under the previous kernel's tail

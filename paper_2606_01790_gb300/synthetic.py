@@ -69,6 +69,11 @@ class Workload:
     shots_range: Tuple[int, int] = (1, 12)
     text_range: Tuple[int, int] = (128, 1024)
     pct_choices: Tuple[int, ...] = (10, 20, 30)
+    # MHA-head granularity on a GQA model (the paper's ablation of MI
+    # granularity): keys and values are drawn for this many groups and each
+    # group's rows are replicated for its n_kv_heads / kv_source_groups query
+    # heads, so that every query head has its own KV head (0: no replication)
+    kv_source_groups: int = 0
 
     @property
     def visual_per_shot(self) -> int:
@@ -95,6 +100,14 @@ WORKLOADS: Dict[str, Workload] = {
     "ragged": Workload("ragged", 5, n_layers=28, n_seqs=16, ragged=True),
     # the timed per-step workload: 28 layers of the 5-screenshot UI-TARS shape
     "uitars_5shot_28l": Workload("uitars_5shot_28l", 6, n_layers=28),
+    # the same step at MHA-head granularity: the 4 groups' keys and values
+    # replicated for each of the 28 query heads (G = H = 28)
+    "uitars_5shot_28l_mha": Workload("uitars_5shot_28l_mha", 6, n_layers=28, n_kv_heads=28,
+                                     kv_source_groups=4),
+    # one layer of that shape, and the tiny case at MHA-head granularity
+    "uitars_layer_mha": Workload("uitars_layer_mha", 2, n_layers=1, n_kv_heads=28, kv_source_groups=4),
+    "tiny_mha": Workload("tiny_mha", 1, n_layers=1, window=8, grid_rows=16, grid_cols=16,
+                         n_shots=2, n_text=64, n_kv_heads=28, kv_source_groups=4),
 }
 
 
@@ -297,6 +310,14 @@ def make_sequence(wl: Workload, seq: int = 0, seed: int = 0,
     ``layers`` restricts generation to a subset (the result is then stacked in
     that order); by default all ``wl.n_layers`` layers are drawn.
     """
+    if wl.kv_source_groups:
+        # draw the GQA model's keys and values, then give every query head its own copy
+        src = dataclasses.replace(wl, n_kv_heads=wl.kv_source_groups, kv_source_groups=0)
+        si = make_sequence(src, seq=seq, seed=seed, layers=layers)
+        rep = wl.n_kv_heads // wl.kv_source_groups
+        si.k = si.k.repeat_interleave(rep, dim=1)
+        si.v = si.v.repeat_interleave(rep, dim=1)
+        return si
     sh = seq_shape(seed, wl, seq)
     lay = token_layout(sh.n_shots, sh.n_text, wl.grid_rows, wl.grid_cols, wl.window)
     layers = list(range(wl.n_layers)) if layers is None else list(layers)

@@ -65,7 +65,9 @@ def test_default_config_matches_paper_defaults(library):
 @pytest.mark.parametrize("bad", [dict(head_dim=64), dict(n_heads=30), dict(window=64),
                                  dict(pool_kernel=4), dict(mi_bins=1), dict(t_min=0.0),
                                  dict(n_kv_heads=0), dict(grid_rows=2000), dict(select_mode=2),
-                                 dict(decay_mode=3), dict(aeb_mode=2), dict(mi_span=-1)])
+                                 dict(decay_mode=3), dict(aeb_mode=2), dict(mi_span=-1),
+                                 dict(n_heads=40, n_kv_heads=40, window=4),
+                                 dict(n_kv_heads=28, select_mode=1)])
 def test_invalid_config_rejected_before_any_device_call(library, bad):
     cfg = sk.Config(**bad)
     with pytest.raises(sk.StarkvError) as e:

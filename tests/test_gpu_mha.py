@@ -1,0 +1,103 @@
+"""GPU parity at MHA-head granularity and other group counts above the
+portable cluster size (8): the paper's ablation replicates each GQA group's
+keys and values for every query head of the group (G = H = 28), so the MI
+prior is estimated per head.  The calibration then runs clusters of 8 CTAs,
+each taking several groups in its first phase.  Same bars as the other parity
+tests: S and the fused scores within 1e-3 relative of the oracle, index sets
+equal except ties inside that band, compacted K/V/metadata bit copies, and the
+per-group MI, prior weights and phi."""
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import starkv_oracle as O
+from paper_2606_01790_gb300 import starkv as sk
+from paper_2606_01790_gb300 import synthetic as syn
+
+import harness as H
+
+pytestmark = pytest.mark.gpu
+
+if not torch.cuda.is_available():
+    pytest.skip("needs a CUDA device", allow_module_level=True)
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def _check_layer(ds, si, layer, wl, p, ost):
+    ref = H.oracle_layer(si, layer, wl, ost, p)
+    S_gpu = ds.seq.S[layer].double().cpu().numpy()
+    assert (np.abs(S_gpu - ref["S"]) / np.abs(ref["S"])).max() < 1e-3
+    sc = H.check_scores(ds.seq.score[layer].double().cpu().numpy(), ref, ref["S"], si, layer, wl, p)
+    assert sc["ok"], (layer, sc)
+    ix = H.check_index_set(ds.seq.idx[layer].cpu().numpy(), ref, si.budget)
+    assert ix["ok"], (layer, ix)
+    H.check_compaction(ds.seq, si, layer, wl.window)
+    G = wl.n_kv_heads
+    stats = ds.seq.stats[layer].double().cpu().numpy()
+    assert abs(stats[0] - ref["H"]) < 1e-5 and abs(stats[1] - ref["T"]) < 1e-5
+    np.testing.assert_allclose(stats[8:8 + G], ref["mi"], rtol=2e-3, atol=2e-4)
+    np.testing.assert_allclose(stats[8 + 2 * G:8 + 3 * G], ref["w"], rtol=2e-3)
+    np.testing.assert_allclose(stats[8 + 3 * G:8 + 4 * G], ref["phi"], atol=1e-4)
+    return ref
+
+
+def _run(wl, si, h, calls=1):
+    st = sk.init_state(H.gpu_config(wl, h))
+    ds = H.device_seq(si, wl)
+    ws = sk.workspace(st, [ds.seq])
+    for _ in range(calls):
+        sk.step(st, [ds.seq], ws)
+    torch.cuda.synchronize()
+    sk.check_device_error(st)
+    return ds
+
+
+@pytest.mark.parametrize("name", ["tiny_mha", "uitars_layer_mha"])
+def test_mha_head_granularity_matches_oracle_over_two_calls(name):
+    wl = syn.WORKLOADS[name]
+    si = syn.make_sequence(wl)
+    assert torch.equal(si.k[:, 0], si.k[:, 6]) and not torch.equal(si.k[:, 6], si.k[:, 7])   # replicated per group
+    h = H.hyper(n_warmup=0, n_ramp=0, t_min=0.75, t_max=1.25)
+    p = H.oracle_params(h)
+    st = sk.init_state(H.gpu_config(wl, h))
+    ost = O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols)
+    for _ in range(2):   # the second call carries the MI and temporal state of 28 groups
+        ds = H.device_seq(si, wl)
+        sk.step(st, [ds.seq], sk.workspace(st, [ds.seq]))
+        torch.cuda.synchronize()
+        sk.check_device_error(st)
+        ref = _check_layer(ds, si, 0, wl, p, ost)
+    assert np.max(ref["phi"]) > 0.0
+
+
+# (query heads, KV heads, window): clusters of 8 CTAs with 1 to 4 groups each
+SHAPES = [(32, 16, 16), (32, 32, 8), (24, 12, 16), (20, 10, 8), (28, 28, 32)]
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=[f"H{a}_G{b}_w{c}" for a, b, c in SHAPES])
+def test_group_counts_above_the_cluster_size(shape):
+    Hq, G, w = shape
+    wl = dataclasses.replace(syn.WORKLOADS["tiny"], n_heads=Hq, n_kv_heads=G, window=w)
+    si = syn.make_sequence(wl)
+    h = H.hyper(n_warmup=0, n_ramp=0, t_min=0.75, t_max=1.25)
+    ds = _run(wl, si, h)
+    _check_layer(ds, si, 0, wl, H.oracle_params(h), O.LayerState.fresh(G, wl.grid_rows, wl.grid_cols))
+
+
+def test_mha_28_layer_step_at_the_benchmark_shape():
+    """The 28-layer 5-screenshot step at MHA-head granularity (28 KV heads, the
+    4 groups' keys replicated), sampled layers against the oracle."""
+    wl = syn.WORKLOADS["uitars_5shot_28l_mha"]
+    si = syn.make_sequence(wl)
+    h = H.hyper(n_warmup=0, n_ramp=0)
+    p = H.oracle_params(h)
+    ds = _run(wl, si, h)
+    for layer in (0, 27):
+        _check_layer(ds, si, layer, wl, p, O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols))

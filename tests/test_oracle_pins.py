@@ -597,3 +597,30 @@ def test_mi_over_the_newest_frame_vs_sklearn():
     full = O.select_layer(s, *meta, F_, 9, 4, 5, O.LayerState.fresh(2, 4, 5),
                           O.Params(n_warmup=0, n_ramp=0, pool_kernel=1, mi_bins=4, mi_grid=2))
     assert not np.allclose(full["mi"], o["mi"])   # the span matters
+
+
+def test_mha_granularity_by_replicated_kv_keeps_s_bar():
+    """The paper's MHA-head ablation on a GQA model: every group's keys
+    replicated for each of its query heads (G' = H).  Each head's row of S is
+    then that head's pooled attention, the mean of a group's head rows is the
+    GQA row S[g], so s_bar is unchanged; with lambda = 0, no temporal term and
+    T = 1 the fused score is s_bar and the selected set equals the GQA one.
+    The MI prior, now over H groups, is what the granularity changes."""
+    q, k, meta, F_ = _small_case(31, H=8, G=2)
+    w, H, G = q.shape[1], q.shape[0], k.shape[0]
+    k_mha = np.repeat(k, H // G, axis=0)
+    p = O.Params()
+    S = O.score_layer(q, k, w, p)
+    S_mha = O.score_layer(q, k_mha, w, p)
+    np.testing.assert_allclose(S_mha, O.avg_pool(O.window_attention(q, k_mha, w), p.pool_kernel), rtol=1e-13)
+    np.testing.assert_allclose(S_mha.reshape(G, H // G, -1).mean(axis=1), S, rtol=1e-12)
+    np.testing.assert_allclose(S_mha.mean(axis=0), S.mean(axis=0), rtol=1e-12)
+    base = O.Params(lam=0.0, delta=0.0, t_min=1.0, t_max=1.0)
+    outs = []
+    for S_, g in ((S, G), (S_mha, H)):
+        st = O.LayerState.fresh(g, 4, 5)
+        outs.append(O.select_layer(S_, *meta, F_, 17, 4, 5, st, base))
+    np.testing.assert_array_equal(outs[0]["idx"], outs[1]["idx"])
+    st = O.LayerState.fresh(H, 4, 5)
+    o = O.select_layer(S_mha, *meta, F_, 17, 4, 5, st, O.Params(n_warmup=0, n_ramp=0))
+    assert o["w"].shape == (H,) and abs(o["w"].sum() - 1.0) < 1e-12
