@@ -308,7 +308,9 @@ __device__ void calibrate_refine_radix(CalShared& sh, int* hist, int* joint, con
   }
 }
 
-template <bool FROM_RAW>
+// MULTI: more groups than CTAs in the cluster (G > kMaxCluster, global mode);
+// the GQA shapes (G <= kMaxCluster) compile without the group loop.
+template <bool FROM_RAW, bool MULTI>
 __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_constant__ SeqBatch b,
                                                               const __grid_constant__ KParams kp, DevState st,
                                                               int capl) {
@@ -328,7 +330,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   const SeqView& sv = b.s[blockIdx.z];
   // the cluster spans grid x: one CTA per group, or kMaxCluster CTAs when G is
   // larger (global mode), CTA `rank` then taking groups rank, rank + ncta, ...
-  const int rank = blockIdx.x, ncta = gridDim.x;
+  const int rank = blockIdx.x, ncta = MULTI ? static_cast<int>(gridDim.x) : G;
   const int ll = blockIdx.y, layer = b.layer0 + ll;
   const int Lp = sv.Lp;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -340,6 +342,9 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   };
   // the per-token arrays of row r: shared memory, or row r's workspace region
   auto keys_of = [&](int r) { return in_smem ? skeys : sv.vis + static_cast<int64_t>(ll * G + r) * Lp * 3; };
+  // row `rank`'s arrays (the only ones without MULTI)
+  const uint32_t* const meta0 = meta_of(rank);
+  uint32_t* const keys0 = keys_of(rank);
   // phase 1 walks the row in one contiguous segment per warp, so that warp
   // order and lane order are position order
   const int seg = ceil_div(Lp, 32 * 32) * 32;
@@ -353,8 +358,10 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   for (int c = tid; c < C; c += kCalThreads) colc[c] = static_cast<uint8_t>(c * M / C);
   // this CTA's groups' temporal EMA rows (state of the previous step, read
   // after phase 1) on their way into L2
-  for (int gi = rank; gi < G; gi += ncta)
+  for (int gi = rank; gi < G; gi += ncta) {
     if (tid * 32 < RC) prefetch_l2(st.m + static_cast<int64_t>(sl * G + gi) * RC + tid * 32);
+    if (!MULTI) break;
+  }
   __syncthreads();
   // the set-up above overlaps the previous kernel's tail; its outputs are read below
   griddep_launch_dependents();
@@ -363,10 +370,10 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   if (tid == 0) sh.n_old = st.n[sl];
 
   // ================= phase 1: groups rank, rank + ncta, ... =================
-  for (int g = rank, gl = 0; g < G; g += ncta, ++gl) {
-  const uint32_t* meta = meta_of(g);
+  for (int g = rank, gl = 0; MULTI ? g < G : gl == 0; g += ncta, ++gl) {
+  const uint32_t* meta = MULTI ? meta_of(g) : meta0;
   float* S = sv.S + (static_cast<int64_t>(layer) * G + g) * Lp;
-  uint32_t* keys = keys_of(g);
+  uint32_t* keys = MULTI ? keys_of(g) : keys0;
   uint32_t* cand = in_smem ? scand : keys + Lp;
   uint16_t* cells = in_smem ? scells : reinterpret_cast<uint16_t*>(keys + 2 * static_cast<int64_t>(Lp));
   // ---- the row, staged in shared memory by one pass of independent loads:
@@ -759,7 +766,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     st.mi_cur[sl * G + g] = mi;
     st.phi_cur[sl * G + g] = phi;
   }
-  if (g + ncta < G) {   // the next group of this CTA starts from clean arrays
+  if (MULTI && g + ncta < G) {   // the next group of this CTA starts from clean arrays
     __syncthreads();
     if (tid == 0) sh.any_tie = 0;
     for (int i = tid; i < kBins0; i += kCalThreads) hist[i] = 0;
@@ -776,8 +783,8 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   // of s_bar; per-KV-head mode (one CTA per group): CTA g its own row S[g, .]
   const bool per_head = kp.per_head != 0;
   const int g = rank;   // per-KV-head mode: this CTA's group
-  const uint32_t* meta = meta_of(per_head ? g : 0);
-  uint32_t* keys = keys_of(rank);
+  const uint32_t* meta = MULTI ? meta_of(0) : meta0;   // global mode: the shared row
+  uint32_t* keys = keys0;
   uint32_t* cand = in_smem ? scand : keys + Lp;
   float* stats = sv.stats ? sv.stats + static_cast<int64_t>(layer) * (8 + 6 * G) : nullptr;
   // ---- Eqs. (6)-(7): MI EMA (double state), min-max, softmax prior; lambda
@@ -791,7 +798,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     double mib = 0.0;
     float mic = 0.f, mf = 0.f;
     if (on) {
-      const int owner = lane % ncta, slot = lane / ncta;
+      const int owner = MULTI ? lane % ncta : lane, slot = MULTI ? lane / ncta : 0;
       mic = dsmem_ld_f32(dsmem_map(&sh.mi[slot], owner));
       sh.ph[lane] = dsmem_ld_f32(dsmem_map(&sh.phi[slot], owner));
       mib = n == 0 ? static_cast<double>(mic)
@@ -921,7 +928,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         if (q.z > best.z) { best.z = q.z; gs[2] = gg; }
         if (q.w > best.w) { best.w = q.w; gs[3] = gg; }
       };
-      if (G <= kMaxCluster) {   // GQA: unrolled, every row's load issued up front
+      if (!MULTI) {   // GQA: unrolled, every row's load issued up front
 #pragma unroll
         for (int gg = 1; gg < kMaxCluster; ++gg) {
           if (gg >= G) break;
@@ -1264,9 +1271,11 @@ int calibrate_capacity(int K, int M, int R, int C) {
 
 cudaError_t select_configure() {
   const int bytes = static_cast<int>(kSmemMax);
-  cudaError_t e = cudaFuncSetAttribute(k_calibrate<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  cudaError_t e = cudaFuncSetAttribute(k_calibrate<true, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_calibrate<true, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_calibrate<false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(k_calibrate<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  return cudaFuncSetAttribute(k_calibrate<false, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
 }
 
 cudaError_t calibrate_launch(const SeqBatch& b, const KParams& kp, const DevState& st, bool from_raw, int lp_max,
@@ -1289,8 +1298,11 @@ cudaError_t calibrate_launch(const SeqBatch& b, const KParams& kp, const DevStat
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (from_raw) return cudaLaunchKernelEx(&cfg, k_calibrate<true>, b, kp, st, capl);
-  return cudaLaunchKernelEx(&cfg, k_calibrate<false>, b, kp, st, capl);
+  const bool multi = kp.G > kMaxCluster;
+  if (from_raw) return multi ? cudaLaunchKernelEx(&cfg, k_calibrate<true, true>, b, kp, st, capl)
+                             : cudaLaunchKernelEx(&cfg, k_calibrate<true, false>, b, kp, st, capl);
+  return multi ? cudaLaunchKernelEx(&cfg, k_calibrate<false, true>, b, kp, st, capl)
+               : cudaLaunchKernelEx(&cfg, k_calibrate<false, false>, b, kp, st, capl);
 }
 
 }  // namespace starkv
