@@ -101,3 +101,47 @@ def test_mha_28_layer_step_at_the_benchmark_shape():
     ds = _run(wl, si, h)
     for layer in (0, 27):
         _check_layer(ds, si, layer, wl, p, O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols))
+
+
+def test_mha_through_the_per_layer_calls_and_the_host_buffer_call():
+    """MHA-head granularity through the other entry points: the three per-layer
+    calls against the oracle, and starkv_step_host from page-locked buffers
+    against the device step (S within fp32 rounding, sets equal except near
+    ties, compacted rows bit copies of the host run's own selection)."""
+    wl = syn.WORKLOADS["tiny_mha"]
+    si = syn.make_sequence(wl)
+    h = H.hyper(n_warmup=0, n_ramp=0, t_min=0.75, t_max=1.25)
+    p = H.oracle_params(h)
+    st = sk.init_state(H.gpu_config(wl, h))
+    ds = H.device_seq(si, wl)
+    ws = sk.workspace(st, [ds.seq])
+    sk.score_layer(st, 0, [ds.seq], ws)
+    sk.select(st, 0, [ds.seq], ws)
+    sk.compact(st, 0, [ds.seq], ws)
+    torch.cuda.synchronize()
+    sk.check_device_error(st)
+    _check_layer(ds, si, 0, wl, p, O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols))
+
+    def host(t):
+        o = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        o.copy_(t.cpu())
+        return o
+
+    d = ds.seq
+    hs = sk.Seq(k=host(d.k), v=host(d.v), q=host(d.q), meta=host(d.meta), meta_layer_stride=d.meta_layer_stride,
+                L=d.L, cur_frame=d.cur_frame, budget=d.budget, slot=0,
+                k_out=torch.empty(d.k_out.shape, dtype=d.k_out.dtype, pin_memory=True),
+                v_out=torch.empty(d.v_out.shape, dtype=d.v_out.dtype, pin_memory=True),
+                meta_out=torch.empty(d.meta_out.shape, dtype=d.meta_out.dtype, pin_memory=True),
+                idx=torch.empty(d.idx.shape, dtype=d.idx.dtype, pin_memory=True),
+                S=torch.empty(d.S.shape, dtype=d.S.dtype, pin_memory=True))
+    st_h = sk.init_state(H.gpu_config(wl, h))
+    sk.step_host(st_h, [hs], sk.workspace(st_h, [hs], host=True))
+    torch.cuda.synchronize()
+    sk.check_device_error(st_h)
+    np.testing.assert_allclose(hs.S.numpy(), d.S.cpu().numpy(), rtol=1e-5, atol=0)
+    ref = H.oracle_layer(si, 0, wl, O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols), p)
+    assert H.check_index_set(hs.idx[0].numpy(), ref, si.budget)["ok"]
+    rows = torch.from_numpy(np.concatenate([hs.idx[0].numpy(), np.arange(si.L - wl.window, si.L)]).astype(np.int64))
+    assert torch.equal(hs.k_out[0], si.k[0].index_select(1, rows))
+    assert torch.equal(hs.v_out[0], si.v[0].index_select(1, rows))
