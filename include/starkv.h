@@ -56,7 +56,7 @@
  *   returns a thread-local message for the last non-OK status.
  * - Supported shapes: d = 128; w >= 1; H % G == 0; (H / G) * w <= 256;
  *   G <= 32 in the global selection mode (G = H is the MHA-head granularity of
- *   the paper's ablation: each group's key/value replicated for each of its
+ *   the ablation in Sec. 4.2: each group's key/value replicated for each of its
  *   query heads), G <= 8 in the per-KV-head mode; L >= w (L_p = L - w >= 0;
  *   L_p = 0 keeps only the window);
  *   0 <= B <= L_p; L < 2^24; 1 <= R, C <= 1024; R * C <= 16384;

@@ -69,8 +69,8 @@ class Workload:
     shots_range: Tuple[int, int] = (1, 12)
     text_range: Tuple[int, int] = (128, 1024)
     pct_choices: Tuple[int, ...] = (10, 20, 30)
-    # MHA-head granularity on a GQA model (the paper's ablation of MI
-    # granularity): keys and values are drawn for this many groups and each
+    # MHA-head granularity on a GQA model (the ablation of the MI prior's
+    # granularity in Sec. 4.2): keys and values are drawn for this many groups and each
     # group's rows are replicated for its n_kv_heads / kv_source_groups query
     # heads, so that every query head has its own KV head (0: no replication)
     kv_source_groups: int = 0

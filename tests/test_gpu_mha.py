@@ -1,5 +1,5 @@
 """GPU parity at MHA-head granularity and other group counts above the
-portable cluster size (8): the paper's ablation replicates each GQA group's
+portable cluster size (8): the ablation in Sec. 4.2 replicates each GQA group's
 keys and values for every query head of the group (G = H = 28), so the MI
 prior is estimated per head.  The calibration then runs clusters of 8 CTAs,
 each taking several groups in its first phase.  Same bars as the other parity
