@@ -78,3 +78,29 @@ def test_recorded_traffic_follows_the_kernel_code_not_its_comments():
     h = bench.kernel_src_hash("score_lse", tree.__getitem__)
     assert bench.kernel_src_hash("score_lse", edited.__getitem__) == h
     assert bench.kernel_src_hash("score_lse", changed.__getitem__) != h
+
+
+def test_algorithmic_bytes_match_the_tensors_of_the_step():
+    """The roofline's algorithmic bytes for the 28-layer 5-screenshot step,
+    rebuilt from the byte sizes of the tensors the step must touch once (torch
+    meta tensors with the ABI's layouts): the past keys and the window queries
+    read, the group score map written and read, and every kept K/V row and
+    metadata word read and written."""
+    from paper_2606_01790_gb300 import synthetic as syn
+    wl = syn.WORKLOADS["uitars_5shot_28l"]
+    lay = syn.token_layout(wl.n_shots, wl.n_text, wl.grid_rows, wl.grid_cols, wl.window)
+    L, nl, G, H, w, d = lay.L, wl.n_layers, wl.n_kv_heads, wl.n_heads, wl.window, wl.head_dim
+    B = syn.budget(wl.budget_pct, wl.n_shots * wl.visual_per_shot, L - w)
+    meta = dict(device="meta")
+    nbytes = lambda t: t.numel() * t.element_size()
+    k_past = torch.empty((nl, G, L - w, d), dtype=torch.bfloat16, **meta)
+    q = torch.empty((nl, H, w, d), dtype=torch.bfloat16, **meta)
+    S = torch.empty((nl, G, L - w), dtype=torch.float32, **meta)
+    kv_out = torch.empty((2, nl, G, B + w, d), dtype=torch.bfloat16, **meta)
+    meta_out = torch.empty((nl, B + w), dtype=torch.int32, **meta)
+    want = nbytes(k_past) + nbytes(q) + 2 * nbytes(S) + 2 * nbytes(kv_out) + 2 * nbytes(meta_out)
+    work = bench.work_per_step(wl, [dict(L=L, B=B)])
+    assert work["step_bytes"] == want
+    assert work["qk_flops"] == 2 * H * w * d * nl * (L - w)
+    peaks = dict(hbm=6698.5, tc=1903.3, tc_sus=1721.9)
+    assert bench.kernel_work("score_lse", work, peaks)[0] == "hbm"   # 224 flop/B, below the ridge
