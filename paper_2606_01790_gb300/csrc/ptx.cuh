@@ -308,6 +308,16 @@ __device__ __forceinline__ void cluster_sync() {
       "barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
+// The two halves of cluster_sync, for work that needs no peer in between:
+// every thread arrives after its writes that the peers read, and waits before
+// its first read of a peer's.
+__device__ __forceinline__ void cluster_arrive() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 // Address of `p` (this CTA's shared memory) in the shared window of cluster CTA `rank`.
 __device__ __forceinline__ uint32_t dsmem_map(const void* p, uint32_t rank) {
   uint32_t a;

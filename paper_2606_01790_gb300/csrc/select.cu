@@ -370,6 +370,8 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   if (tid == 0) sh.n_old = st.n[sl];
 
   // ================= phase 1: groups rank, rank + ncta, ... =================
+  float* mrow_last = nullptr;   // the last group's m_g row and its update (0 none, 1 EMA, 2 first row),
+  int mupd_last = 0;            // done while the phase-1 cluster barrier settles
   for (int g = rank, gl = 0; MULTI ? g < G : gl == 0; g += ncta, ++gl) {
   const uint32_t* meta = MULTI ? meta_of(g) : meta0;
   float* S = sv.S + (static_cast<int64_t>(layer) * G + g) * Lp;
@@ -751,14 +753,20 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     nm = r3[2];
   }
   float phi = 0.f;
+  int mupd = 0;
   if (ncur > 0.f) {
-    if (nm > 0.f) {
-      phi = dot / (sqrtf(ncur) * sqrtf(nm));
-      const float rt = kp.rho_t;
+    mupd = nm > 0.f ? 1 : 2;
+    if (nm > 0.f) phi = dot / (sqrtf(ncur) * sqrtf(nm));
+  }
+  if (MULTI && g + ncta < G) {   // an earlier group of this CTA: its current row is cleared next
+    const float rt = kp.rho_t;
+    if (mupd == 1)
       for (int i = tid; i < RC; i += kCalThreads) mrow[i] = rt * mrow[i] + (1.f - rt) * cur[i];
-    } else {
+    else if (mupd == 2)
       for (int i = tid; i < RC; i += kCalThreads) mrow[i] = cur[i];
-    }
+  } else {
+    mrow_last = mrow;
+    mupd_last = mupd;
   }
   if (tid == 0) {
     sh.mi[gl] = mi;
@@ -775,8 +783,19 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
     __syncthreads();
   }
   }   // phase-1 group loop
+  // every group's S row, MI_g and phi_g are written: the peers may read them
+  // once the barrier completes; the last group's m_g (read by no peer) and the
+  // top-B histogram's zeroing go in between
+  cluster_arrive();
+  {
+    const float rt = kp.rho_t;
+    if (mupd_last == 1)
+      for (int i = tid; i < RC; i += kCalThreads) mrow_last[i] = rt * mrow_last[i] + (1.f - rt) * cur[i];
+    else if (mupd_last == 2)
+      for (int i = tid; i < RC; i += kCalThreads) mrow_last[i] = cur[i];
+  }
   for (int i = tid; i < kBins0; i += kCalThreads) hist[i] = 0;   // top-B digit 1 (below)
-  cluster_sync();   // every group's S row, MI_g and phi_g are complete
+  cluster_wait();
 
   // ================= phase 2 =================
   // global mode: CTA r scores and selects tokens [r Lp / ncta, (r + 1) Lp / ncta)
@@ -1053,21 +1072,25 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   auto sbucket = [&](uint32_t u) {
     return min(kBins0 - 1, static_cast<int>(static_cast<float>(u - kmin2) * sbinv));
   };
-  for (int i = tid; i < nr; i += kCalThreads) {
-    score[i] = ex2_approx(invT * lg2_approx(xs[i]));
-    atomicAdd(&hist[sbucket(keys[i])], 1);
-  }
+  const int B = sv.budget;   // the same in every CTA of the cluster
+  for (int i = tid; i < nr; i += kCalThreads) atomicAdd(&hist[sbucket(keys[i])], 1);
+  // global mode: the peers read this CTA's histogram next; the tempered
+  // scores, which no peer reads, are written while the cluster barrier settles
+  const bool early_arrive = B > 0 && !per_head;
+  if (early_arrive) cluster_arrive();
+  for (int i = tid; i < nr; i += kCalThreads) score[i] = ex2_approx(invT * lg2_approx(xs[i]));
 
   // ---- Sec. 3.7: top-B, ties to the lower index (global mode: over the
   // cluster; per-KV-head mode: over this CTA's row, block barriers only)
-  const int B = sv.budget;   // the same in every CTA of the cluster
+  bool done_remote = false;   // arrived at the final cluster barrier after the last remote read
   if (B > 0) {
     const int r_lo = per_head ? g : 0, r_hi = per_head ? g + 1 : ncta;
     auto sel_sync = [&]() {
       if (per_head) __syncthreads();
       else cluster_sync();
     };
-    sel_sync();   // every bucket histogram of the selection is complete
+    if (early_arrive) cluster_wait();   // every bucket histogram of the selection is complete
+    else __syncthreads();
     {
       int4 h = sum_peers_v4(hist + 4 * tid, r_lo, r_hi);
       const int sum = (h.x + h.y) + (h.z + h.w);
@@ -1131,6 +1154,10 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
         if (r < rank) nlow += sh.pbelow[r];
       }
       __syncthreads();
+      if (!per_head) {   // no peer's shared memory is read after this point
+        cluster_arrive();
+        done_remote = true;
+      }
       for (int i = tid; i < nall; i += kCalThreads) {
         const uint32_t ki = all[2 * i], ti = all[2 * i + 1];
         int rank = 0;
@@ -1260,7 +1287,9 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       }
     }
   }
-  cluster_sync();   // the peers' shared memory stays valid until every remote read is done
+  // the peers' shared memory stays valid until every remote read is done
+  if (done_remote) cluster_wait();
+  else cluster_sync();
 }
 
 int calibrate_capacity(int K, int M, int R, int C) {
