@@ -152,6 +152,7 @@ struct CalShared {
   float zpart, hpart, vpart;      // this CTA's token range (phase 2)
   uint32_t kminp, kmaxp, smaxp;
   int tcand, nbelow;              // top-B boundary-bucket candidates, tokens below it
+  int lowcnt;                     // kept candidates of the lower-ranked CTAs
   int nlt, neq;
   // top-B select
   int tb, tcnt;                   // boundary bucket and its token count
@@ -1146,6 +1147,7 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
       // peer reads it any more), then rank each by (key, position)
       uint32_t* all = reinterpret_cast<uint32_t*>(hist);
       int nall = 0, nlow = 0;
+      if (tid == 0) sh.lowcnt = 0;
       for (int r = r_lo; r < r_hi; ++r) {
         const int n = sh.pncand[r];
         for (int j = tid; j < 2 * n; j += kCalThreads)
@@ -1169,27 +1171,19 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
           sh.tkey = ki;
           sh.tpos = static_cast<int>(ti);
         }
+        // kept (rank <= the B-th's: the order is by key, then position) and
+        // before this CTA's range: a kept candidate of a lower-ranked CTA
+        if (rank <= rkb && static_cast<int>(ti) < ta) atomicAdd(&sh.lowcnt, 1);
       }
       __syncthreads();
       const uint32_t kT = sh.tkey;
       const uint32_t tT = static_cast<uint32_t>(sh.tpos);
       auto kept = [&](uint32_t u, uint32_t t) { return u < kT || (u == kT && t <= tT); };
-      // kept tokens of the lower-ranked CTAs: all of their tokens below the
-      // boundary bucket and their kept candidates
-      float lowc = 0.f;
-      for (int i = tid; i < nall; i += kCalThreads) {
-        const uint32_t ti = all[2 * i + 1];
-        if (static_cast<int>(ti) < ta && kept(all[2 * i], ti)) lowc += 1.f;
-      }
       int nk = 0;
       for (int i = i0; i < i1; ++i) nk += kept(keys[i], static_cast<uint32_t>(ta + i));
-      {
-        float l1[1] = {lowc};
-        uint32_t u0 = 0u, u1 = 0u;
-        block_reduce<1>(l1, u0, u1, sh);
-        lowc = l1[0];
-      }
-      int pos = nlow + static_cast<int>(lowc) + block_excl_scan(nk, sh.scan, nullptr);
+      // kept tokens of the lower-ranked CTAs: all of their tokens below the
+      // boundary bucket and their kept candidates
+      int pos = nlow + sh.lowcnt + block_excl_scan(nk, sh.scan, nullptr);
       for (int i = i0; i < i1; ++i) {
         if (!kept(keys[i], static_cast<uint32_t>(ta + i))) continue;
         if (pos >= B) atomicOr(st.err, kErrIndex);   // cannot happen for a correct select
