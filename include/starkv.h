@@ -335,7 +335,8 @@ enum {
   STARKV_KERNEL_SCORE_ACCUM = 1,  /* scoring pass 2: normalised group sums (Eqs. 2-4)      */
   STARKV_KERNEL_POOL = 2,         /* AvgPool1D + group mean (Eqs. 3-4), per-layer calls    */
   STARKV_KERNEL_CALIBRATE = 3,    /* MI, phi, prior, temperature, fused score, top-B
-                                     (Sec. 3.4-3.7): one cluster of G CTAs per layer       */
+                                     (Sec. 3.4-3.7): one cluster of min(G, 8) CTAs per
+                                     layer                                                 */
   STARKV_KERNEL_COMPACT = 4,      /* KV gather (Eq. 11)                                    */
   STARKV_NUM_KERNELS = 5
 };

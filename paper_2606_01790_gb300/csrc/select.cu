@@ -1,14 +1,15 @@
 // Calibration and selection of Sec. 3.4 - 3.7 (Algorithm 1 from s_bar to I):
-// one thread-block cluster of G CTAs per (sequence, layer).
+// one thread-block cluster of n = min(G, 8) CTAs per (sequence, layer).
 //
-// Phase 1, CTA g of the cluster works on group g:
+// Phase 1, CTA r of the cluster works on groups g = r, r + n, ... (group r
+// alone when G <= 8), one after the other:
 //   (step path) AvgPool1D + group mean of the unpooled sums -> S[g, :] (Eqs. 3-4);
 //   RankBin: the K - 1 equal-frequency boundaries of S[g, visual tokens] by an
 //     exact multi-target radix select (12 + 10 + 10-bit digits) on
 //     order-preserving keys, equal keys ordered by position;
 //   SpatialBin + joint histogram -> plug-in MI_g                        (Eq. 5);
 //   phi_g = cos(current-frame row on the patch grid, m_g); m_g update    (Eq. 8).
-// Phase 2, CTA r of the cluster works on tokens [r Lp / G, (r + 1) Lp / G):
+// Phase 2, CTA r of the cluster works on tokens [r Lp / n, (r + 1) Lp / n):
 //   MI EMA, min-max and softmax prior, lambda schedule                  (Eqs. 6-7);
 //   s_bar, g*, Z = sum s_bar and the entropy H (Sec. 3.6), the per-CTA
 //     partial sums exchanged through distributed shared memory;
