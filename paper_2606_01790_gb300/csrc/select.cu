@@ -503,36 +503,59 @@ __global__ void __launch_bounds__(kCalThreads, 1) k_calibrate(const __grid_const
   if (vec) {
     const float4* st4 = reinterpret_cast<const float4*>(stage);
     const bool s16 = (reinterpret_cast<uintptr_t>(S) & 15) == 0;   // S row on a 16-byte boundary
-    for (int t0 = 4 * tid; t0 < Lp; t0 += 4 * kCalThreads) {
-      float sv4[4];
-      if (half == 2 && t0 >= 4 && t0 + 8 <= Lp) {   // x[t0 - 4 .. t0 + 7] in three 16-byte loads
-        const float4 a = st4[(t0 >> 2) - 1], b = st4[t0 >> 2], c = st4[(t0 >> 2) + 1];
-        const float x[12] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w, c.x, c.y, c.z, c.w};
+    // two vectors of four tokens per thread and pass: both vectors' loads are
+    // issued before either's arithmetic and stores
+    for (int t00 = 4 * tid; t00 < Lp; t00 += 8 * kCalThreads) {
+      float4 a[2], b[2], c[2];
+      uint4 m4[2];
+      bool in[2], fast[2];
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          sv4[k] = ((((x[k + 2] + x[k + 3]) + x[k + 4]) + x[k + 5]) + x[k + 6]) * pscale;
-      } else {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) sv4[k] = t0 + k < Lp ? pooled(t0 + k) : 0.f;
-      }
-      const uint4 m4 = reinterpret_cast<const uint4*>(keys)[t0 >> 2];
-      const uint32_t mts[4] = {m4.x, m4.y, m4.z, m4.w};
-      uint32_t ks[4];
-      uint16_t cs[4];
-      if (s16 && t0 + 3 < Lp) *reinterpret_cast<float4*>(S + t0) = make_float4(sv4[0], sv4[1], sv4[2], sv4[3]);
-#pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        ks[k] = 0u;
-        cs[k] = kNoCell;
-        if (t0 + k < Lp) {
-          if (!s16 || t0 + 3 >= Lp) S[t0 + k] = sv4[k];
-          classify(sv4[k], mts[k], ks[k], cs[k]);
+      for (int v = 0; v < 2; ++v) {
+        const int t0 = t00 + 4 * v * kCalThreads;
+        in[v] = t0 < Lp;
+        fast[v] = in[v] && half == 2 && t0 >= 4 && t0 + 8 <= Lp;   // x[t0 - 4 .. t0 + 7] in three 16-byte loads
+        a[v] = b[v] = c[v] = make_float4(0.f, 0.f, 0.f, 0.f);
+        m4[v] = make_uint4(0u, 0u, 0u, 0u);
+        if (fast[v]) {
+          a[v] = st4[(t0 >> 2) - 1];
+          b[v] = st4[t0 >> 2];
+          c[v] = st4[(t0 >> 2) + 1];
         }
+        if (in[v]) m4[v] = reinterpret_cast<const uint4*>(keys)[t0 >> 2];
       }
-      reinterpret_cast<uint4*>(keys)[t0 >> 2] = make_uint4(ks[0], ks[1], ks[2], ks[3]);
-      reinterpret_cast<uint2*>(cells)[t0 >> 2] =
-          make_uint2(static_cast<uint32_t>(cs[0]) | (static_cast<uint32_t>(cs[1]) << 16),
-                     static_cast<uint32_t>(cs[2]) | (static_cast<uint32_t>(cs[3]) << 16));
+#pragma unroll
+      for (int v = 0; v < 2; ++v) {
+        const int t0 = t00 + 4 * v * kCalThreads;
+        if (!in[v]) continue;
+        float sv4[4];
+        if (fast[v]) {
+          const float x[12] = {a[v].x, a[v].y, a[v].z, a[v].w, b[v].x, b[v].y, b[v].z, b[v].w,
+                               c[v].x, c[v].y, c[v].z, c[v].w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            sv4[k] = ((((x[k + 2] + x[k + 3]) + x[k + 4]) + x[k + 5]) + x[k + 6]) * pscale;
+        } else {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) sv4[k] = t0 + k < Lp ? pooled(t0 + k) : 0.f;
+        }
+        const uint32_t mts[4] = {m4[v].x, m4[v].y, m4[v].z, m4[v].w};
+        uint32_t ks[4];
+        uint16_t cs[4];
+        if (s16 && t0 + 3 < Lp) *reinterpret_cast<float4*>(S + t0) = make_float4(sv4[0], sv4[1], sv4[2], sv4[3]);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          ks[k] = 0u;
+          cs[k] = kNoCell;
+          if (t0 + k < Lp) {
+            if (!s16 || t0 + 3 >= Lp) S[t0 + k] = sv4[k];
+            classify(sv4[k], mts[k], ks[k], cs[k]);
+          }
+        }
+        reinterpret_cast<uint4*>(keys)[t0 >> 2] = make_uint4(ks[0], ks[1], ks[2], ks[3]);
+        reinterpret_cast<uint2*>(cells)[t0 >> 2] =
+            make_uint2(static_cast<uint32_t>(cs[0]) | (static_cast<uint32_t>(cs[1]) << 16),
+                       static_cast<uint32_t>(cs[2]) | (static_cast<uint32_t>(cs[3]) << 16));
+      }
     }
   } else {
     for (int t = tid; t < Lp; t += kCalThreads) {
