@@ -247,7 +247,7 @@ starkv_status starkv_get_config(const starkv_state* st, starkv_config* out);
 starkv_status starkv_workspace_bytes(const starkv_state* st, const starkv_seq* seqs, int32_t nseq,
                                      int32_t host, size_t* bytes);
 
-/* Sec. 3.3, Eqs. (2)-(4) (Algorithm 1, first two steps): for layer `layer` of
+/* Sec. 3.3, Eqs. (2)-(4): for layer `layer` of
  * every sequence, writes S[g][t] = (G/H) * sum_{h in g} AvgPool1D(
  * sum_{i<w} softmax_t(Q_{-i,h} K_past[g]^T / sqrt(d)))[t]  for t < L_p,
  * softmax over K_past only.  Reads k, q; writes S.  Uses tcgen05 tensor cores
@@ -263,21 +263,25 @@ starkv_status starkv_score_layer(starkv_state* st, int32_t layer, const starkv_s
  * runtime that owns every device allocation.  The paper has no counterpart;
  * this is a deployment aid.  Same arguments and results as starkv_score_layer,
  * minus the workspace: the scratch (pass-1 partials and unpooled sums) is one
- * static device array of 16 MiB per device, which every GPU that loads this
- * library holds until the process exits.  The call allocates no device memory
- * (no cudaMalloc / cudaFree).  Its first call on a device looks up the array's
- * device address (cudaGetSymbolAddress) with that device current, so make that
- * first call before any stream capture.  Every call on a device shares the one
- * array and leaves its last contents there (nothing in it has to start at
- * zero): calls that may overlap on the GPU (different streams, or threads
- * without ordering) race on it and must not be issued.  A batch whose scratch
- * would exceed 16 MiB is rejected with STARKV_ERR_UNSUPPORTED before any
- * launch (about 1.8 MB per sequence at the 5-screenshot UI-TARS shape); kernel
- * timing must be off (it creates CUDA events). */
+ * static device array of 16 MiB per device.  The array is reserved on a device
+ * when this library's device code is loaded there: at context creation under
+ * eager module loading, else (CUDA's default lazy loading) in
+ * starkv_init_state, which looks up the array's device address
+ * (cudaGetSymbolAddress) with the state's device current; it stays reserved
+ * until the process exits.  The call itself allocates no device memory (no
+ * cudaMalloc / cudaFree, no allocating library routine).  Every call on a
+ * device shares the one array and leaves its last contents there (nothing in
+ * it has to start at zero): calls that may overlap on the GPU (different
+ * streams, or threads without ordering) race on it and must not be issued.  A
+ * batch whose scratch would exceed 16 MiB is rejected with
+ * STARKV_ERR_UNSUPPORTED before any launch (about 1.8 MB per sequence at the
+ * 5-screenshot UI-TARS shape); kernel timing must be off (it creates CUDA
+ * events).  STARKV_ERR_CUDA if the array could not be reserved when the state
+ * was created. */
 starkv_status starkv_score_layer_noalloc(starkv_state* st, int32_t layer, const starkv_seq* seqs,
                                          int32_t nseq, void* stream);
 
-/* Sec. 3.3 - 3.7 after the group score map (Algorithm 1 from s_bar to I): from
+/* Sec. 3.3 - 3.7 after the group score map (Eq. 4 to Eq. 10): from
  * S of layer `layer`: s_bar, g*, online MI per group (Eq. 5) -> EMA (Eq. 6) ->
  * prior w (Eq. 7) -> beta; phi_g and the m_g update (Eq. 8) -> D_t (Eq. 9);
  * H_hat and T (Sec. 3.6); s_t = max(s_bar beta D, 0)^(1/T); global top-B with

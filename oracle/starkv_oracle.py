@@ -4,8 +4,12 @@ TEST INFRASTRUCTURE.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
 ``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import this
 module.  It shares no code with the CUDA library and imports nothing from it.
 
-It follows Algorithm 1 (App. A.2) step by step, with the equations of
-Sec. 3.3 - 3.7, in float64 from bf16-rounded inputs (upcast exactly).  Library
+It is organised by the equations it restates: Sec. 3.3 Eqs. 2-4 (window
+attention, pooling, group scores), Sec. 3.4 Eqs. 5-7 (spatial MI, its EMA and
+the group prior), Sec. 3.5 Eqs. 8-9 (temporal stability and decay), Sec. 3.6
+(entropy temperature), Sec. 3.7 Eqs. 10-11 (top-B and compaction); the layer
+functions at the end compose them as the paper's Algorithm 1 does as a whole.
+Everything runs in float64 from bf16-rounded inputs (upcast exactly).  Library
 primitives used as single steps: numpy matmul, exp/log, lexsort, bincount.
 
 Readings of points the paper leaves open (each is a keyword argument or a
@@ -29,8 +33,8 @@ parameter with the stated default):
   s_g^(c) is S[g, .] over the visual tokens of the current frame F, summed per
   cell.  Fresh (||m_g|| = 0): phi_g = 0 and m_g <- s_g^(c).  A current frame
   with no visual tokens: phi_g = 0 and m_g unchanged.
-* Top-B (Sec. 3.7, Algorithm 1 "Sort(TopK)"): one global token-level set per
-  layer, ties to the lower index, returned ascending.
+* Top-B (Sec. 3.7, Eq. 10): one global token-level set per layer, ties to
+  the lower index, returned ascending (the paper sorts the kept indices).
 * Method variants of the ablations (Table 3 and the AEB ablation), off by
   default; the paper names them but prints no formula, so each is a reading:
   decay_mode 1 "linear": D = D_min + (1 - D_min) max(0, 1 - delta Df phi);
@@ -137,7 +141,7 @@ def window_attention_given_lse(q: np.ndarray, k: np.ndarray, window: int, lse: n
 
 
 def window_attention(q: np.ndarray, k: np.ndarray, window: int) -> np.ndarray:
-    """Sec. 3.3, Eq. (2) / Algorithm 1 first step: A_raw[h, t] = sum over the w
+    """Sec. 3.3, Eq. (2): A_raw[h, t] = sum over the w
     window queries of softmax_t(Q_{-i,h} . K_past[g(h), t] / sqrt(d)).
 
     q: [H][w][d] window queries; k: [G][L][d] keys of the whole cache.
@@ -174,7 +178,7 @@ def avg_pool(a_raw: np.ndarray, kernel: int) -> np.ndarray:
 
 
 def group_scores(a: np.ndarray, n_kv_heads: int) -> np.ndarray:
-    """Sec. 3.3, Eq. (4) / Algorithm 1 second step: S[g, t] = (G/H) sum of
+    """Sec. 3.3, Eq. (4): S[g, t] = (G/H) sum of
     A[h, t] over the H/G heads of group g."""
     H, lp = a.shape
     G = n_kv_heads
@@ -198,8 +202,9 @@ def governing_group(s: np.ndarray) -> np.ndarray:
 
 def entropy_temperature(sbar: np.ndarray, t_min: float, t_max: float,
                         eps_h: float) -> tuple:
-    """Sec. 3.6, Eq. (9) in Algorithm 1's form: p_t = s_bar_t / (sum s_bar + eps),
-    H = -sum p_t log(p_t + eps) / log L, T = T_min + (T_max - T_min) H."""
+    """Sec. 3.6, with the epsilons placed as the paper's Algorithm 1 places
+    them: p_t = s_bar_t / (sum s_bar + eps), H = -sum p_t log(p_t + eps) / log L,
+    T = T_min + (T_max - T_min) H."""
     lp = sbar.shape[0]
     if lp <= 1:
         h = 0.0
@@ -343,7 +348,7 @@ def final_score(sbar: np.ndarray, beta: np.ndarray, d: np.ndarray, temp: float) 
 
 
 def top_b(score: np.ndarray, b: int) -> np.ndarray:
-    """Sec. 3.7, Eq. (10) / Algorithm 1 "Sort(TopK)": the b largest scores,
+    """Sec. 3.7, Eq. (10): the b largest scores,
     ties to the lower index, returned in ascending index order."""
     n = score.shape[0]
     order = np.lexsort((np.arange(n), -score))
@@ -381,7 +386,8 @@ class LayerState:
 
 def score_layer(q: np.ndarray, k: np.ndarray, window: int, p: Params,
                 lse: Optional[np.ndarray] = None) -> np.ndarray:
-    """Algorithm 1, first two steps: S = group-mean of Pool(sum_i softmax(Q_{-i} K^T / sqrt d)).
+    """Sec. 3.3, Eqs. (2)-(4) composed:
+    S = group-mean of Pool(sum_i softmax(Q_{-i} K^T / sqrt d)).
     ``lse`` [H][w], when given, is the softmax normaliser of each window row."""
     a_raw = window_attention(q, k, window) if lse is None else window_attention_given_lse(q, k, window, lse)
     a = avg_pool(a_raw, p.pool_kernel)
@@ -397,7 +403,8 @@ def _group_meta(a: np.ndarray, g: int) -> np.ndarray:
 def calibrate_layer(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarray, row: np.ndarray,
                     col: np.ndarray, cur_frame: int, R: int, C: int, st: LayerState,
                     p: Params) -> Dict:
-    """Algorithm 1's per-group calibration, shared by both selection modes:
+    """The per-group calibration of Sec. 3.4-3.5 (Eqs. 5-8), shared by both
+    selection modes:
     MI_g (Eq. 5) -> MI EMA (Eq. 6) -> prior w (Eq. 7) and lambda_n (Sec. 3.4);
     phi_g and the m_g update (Eq. 8).  The metadata arrays are [L] (shared) or
     [G][L] (one row per group).  Does not modify ``st``; returns the new EMAs
@@ -429,7 +436,8 @@ def _advance(st: LayerState, cal: Dict) -> None:
 def select_layer(s: np.ndarray, is_visual: np.ndarray, frame: np.ndarray, row: np.ndarray,
                  col: np.ndarray, cur_frame: int, budget: int, R: int, C: int,
                  st: LayerState, p: Params, gstar_override: Optional[np.ndarray] = None) -> Dict:
-    """Algorithm 1 from the base score to the index set, for one layer.
+    """Sec. 3.3 Eq. 4 to Sec. 3.7 Eq. 10 for one layer: from the group score
+    map to the index set.
 
     ``s`` is the group score map S [G][L_past]; the metadata arrays cover the
     L_past historical tokens.  ``st`` is updated in place (MI EMA, m_g, n).
@@ -492,8 +500,8 @@ def step_layer(q: np.ndarray, k: np.ndarray, v: np.ndarray, is_visual: np.ndarra
                frame: np.ndarray, row: np.ndarray, col: np.ndarray, cur_frame: int,
                budget: int, window: int, R: int, C: int, st: LayerState, p: Params,
                per_head: bool = False) -> Dict:
-    """Algorithm 1 for one layer: scores, calibration, selection and the
-    compressed cache (K', V', metadata'); ``per_head`` picks the per-KV-head
+    """The whole method for one layer (the paper's Algorithm 1 as a whole):
+    scores, calibration, selection and the compressed cache (K', V', metadata'); ``per_head`` picks the per-KV-head
     selection mode (idx [G][B], metadata' [G][B + w])."""
     s = score_layer(q, k, window, p)
     meta = (is_visual, frame, row, col)

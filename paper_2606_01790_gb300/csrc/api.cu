@@ -41,6 +41,10 @@ struct starkv_state {
   // starkv_step_host: copy-in / copy-out streams and their ordering events
   cudaStream_t pipe_in = nullptr, pipe_out = nullptr;
   std::vector<cudaEvent_t> pipe_ev;
+  // starkv_score_layer_noalloc: device address of the static scratch on this
+  // state's device (looked up at init), or NULL with the reason kept
+  void* noalloc_scratch = nullptr;
+  std::string noalloc_error;
 };
 
 namespace {
@@ -147,6 +151,14 @@ cudaError_t launch(starkv_state* st, int kind, cudaStream_t stream, F&& fn) {
   st->recs.push_back(r);
   return e;
 }
+
+// Scratch of starkv_score_layer_noalloc, the scoring call for callers that
+// cannot allocate device memory: one static device array that every call on a
+// device shares.  Host code may not hand the symbol itself to a kernel (on the
+// host it names a stand-in, not device memory): starkv_init_state looks up its
+// device address with the state's device current.
+constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;   // 16 MiB per device
+__device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 starkv_status validate_config(const starkv_config& c) {
   if (c.n_layers < 1 || c.n_heads < 1 || c.n_kv_heads < 1 || c.window < 1 || c.max_seqs < 1)
@@ -523,6 +535,16 @@ starkv_status starkv_init_state(const starkv_config* cfg, starkv_state** out, vo
     delete st;
     return set_error(STARKV_ERR_CUDA, "device setup failed: %s", cudaGetErrorString(e));
   }
+  // The no-allocation scoring call's scratch on this device.  Under lazy module
+  // loading this lookup loads the module that holds the array, so its 16 MiB
+  // are reserved here, where the library allocates anyway, and not inside a
+  // call that promises to allocate nothing.  A failure only disables that call.
+  e = cudaGetSymbolAddress(&st->noalloc_scratch, g_noalloc_scratch);
+  if (e != cudaSuccess || !st->noalloc_scratch) {
+    st->noalloc_scratch = nullptr;
+    st->noalloc_error = cudaGetErrorString(e);
+    cudaGetLastError();   // the failure is recorded, not left for the next call
+  }
   const size_t SL = static_cast<size_t>(cfg->max_seqs) * cfg->n_layers;
   const size_t G = cfg->n_kv_heads, RC = static_cast<size_t>(cfg->grid_rows) * cfg->grid_cols;
   const size_t o_n = 0;
@@ -889,7 +911,7 @@ starkv_status starkv_check_device_error(starkv_state* st, void* stream) {
   CUDA_TRY(cudaMemsetAsync(st->dev.err, 0, sizeof(uint32_t), s));
   if (h & kErrTimeout) return set_error(STARKV_ERR_TIMEOUT, "a bounded device wait ran out");
   if (h & kErrMeta) return set_error(STARKV_ERR_DEVICE, "token metadata outside the patch grid");
-  if (h & kErrIndex) return set_error(STARKV_ERR_DEVICE, "an index outside the cache reached the gather");
+  if (h & kErrIndex) return set_error(STARKV_ERR_DEVICE, "a kept index outside the past tokens reached the gather");
   return STARKV_OK;
 }
 
@@ -938,19 +960,8 @@ const char* starkv_last_error(void) { return g_last_error.c_str(); }
 
 // ---------------------------------------------------------------------------
 // starkv_score_layer_noalloc: the scoring call for callers that cannot
-// allocate device memory (see include/starkv.h).  Its scratch is one static
-// device array shared by every call on a device; the array's device address is
-// looked up once per device with that device current.
-
-namespace {
-
-constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;   // 16 MiB per device
-__device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
-constexpr int kNoAllocMaxDevices = 64;
-std::mutex g_noalloc_mu;
-void* g_noalloc_ptr[kNoAllocMaxDevices] = {};
-
-}  // namespace
+// allocate device memory (see include/starkv.h).  Its scratch is the static
+// device array above, whose address starkv_init_state looked up.
 
 extern "C" starkv_status starkv_score_layer_noalloc(starkv_state* st, int32_t layer, const starkv_seq* seqs,
                                                     int32_t nseq, void* stream) {
@@ -960,9 +971,9 @@ extern "C" starkv_status starkv_score_layer_noalloc(starkv_state* st, int32_t la
   if (st->timing)
     return set_error(STARKV_ERR_INVALID_ARG, "kernel timing creates CUDA events: turn it off for this call");
   if ((s = check_device(st)) != STARKV_OK) return s;
-  if (st->device < 0 || st->device >= kNoAllocMaxDevices)
-    return set_error(STARKV_ERR_UNSUPPORTED, "device index %d is beyond the %d this call tracks", st->device,
-                     kNoAllocMaxDevices);
+  if (!st->noalloc_scratch)
+    return set_error(STARKV_ERR_CUDA, "the static scratch is unavailable on device %d: %s", st->device,
+                     st->noalloc_error.c_str());
   WsPlan plan;
   plan_ws(st, seqs, nseq, 1, false, false, &plan);
   if (plan.total > kNoAllocScratchBytes)
@@ -970,19 +981,6 @@ extern "C" starkv_status starkv_score_layer_noalloc(starkv_state* st, int32_t la
                      "this call needs %zu bytes of scratch; the static scratch holds %zu bytes: "
                      "split the batch or use starkv_score_layer with a workspace",
                      plan.total, kNoAllocScratchBytes);
-  void* scratch = nullptr;
-  {
-    std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    if (!g_noalloc_ptr[st->device]) {
-      void* p = nullptr;
-      const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-      if (e != cudaSuccess || !p)
-        return set_error(STARKV_ERR_CUDA, "cudaGetSymbolAddress of the static scratch failed: %s",
-                         cudaGetErrorString(e));
-      g_noalloc_ptr[st->device] = p;
-    }
-    scratch = g_noalloc_ptr[st->device];
-  }
-  return run_stages(st, seqs, nseq, layer, 1, kScore | kPool, scratch, kNoAllocScratchBytes,
+  return run_stages(st, seqs, nseq, layer, 1, kScore | kPool, st->noalloc_scratch, kNoAllocScratchBytes,
                     static_cast<cudaStream_t>(stream));
 }

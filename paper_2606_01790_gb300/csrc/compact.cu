@@ -1,4 +1,4 @@
-// Compressed cache of Sec. 3.7, Eq. (11) (Algorithm 1 last step):
+// Compressed cache of Sec. 3.7, Eq. (11):
 //   K' = [K_past[I]; K_rec],  V' = [V_past[I]; V_rec],  meta' likewise.
 // A bit copy bound by HBM bandwidth.  A warp task is 32 consecutive output
 // rows of one (tensor, group): lane i resolves the source row of output row
@@ -62,7 +62,8 @@ __global__ void __launch_bounds__(kCompactThreads) k_compact(const __grid_consta
     int src = 0;
     if (r < rows_out) {
       src = r < B ? idx_l[static_cast<int64_t>(p) * B + r] : Lp + (r - B);
-      if (src < 0 || src >= L) {   // an index outside the cache: report, copy row 0
+      // a kept index must name a past token (< L_p): the window rows follow it
+      if (src < 0 || src >= (r < B ? Lp : L)) {   // report, copy row 0
         atomicOr(err, kErrIndex);
         src = 0;
       }

@@ -1,5 +1,4 @@
-// Window-query x key scoring of Sec. 3.3 (Eqs. 2-4, Algorithm 1 first two
-// steps) on tcgen05 tensor cores.
+// Window-query x key scoring of Sec. 3.3 (Eqs. 2-4) on tcgen05 tensor cores.
 //
 //   A_raw[h, t] = sum_{i<w} softmax_t(Q_{-i,h} . K_past[g(h), t] / sqrt(d))
 //   S_raw[g, t] = sum_{h in g} A_raw[h, t]          (pooling + 1/(H/G) later)

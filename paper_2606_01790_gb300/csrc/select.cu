@@ -1,12 +1,17 @@
-// Calibration and selection of Sec. 3.4 - 3.7 (Algorithm 1 from s_bar to I):
+// Calibration and selection of Sec. 3.4 - 3.7 (from s_bar to the index set I):
 // one thread-block cluster of n = min(G, 8) CTAs per (sequence, layer).
 //
 // Phase 1, CTA r of the cluster works on groups g = r, r + n, ... (group r
 // alone when G <= 8), one after the other:
 //   (step path) AvgPool1D + group mean of the unpooled sums -> S[g, :] (Eqs. 3-4);
-//   RankBin: the K - 1 equal-frequency boundaries of S[g, visual tokens] by an
-//     exact multi-target radix select (12 + 10 + 10-bit digits) on
-//     order-preserving keys, equal keys ordered by position;
+//   RankBin: the K - 1 equal-frequency boundaries of S[g, visual tokens] on
+//     order-preserving keys, equal keys ordered by position: a 4096-bucket
+//     histogram spread linearly over the row's key range locates each
+//     boundary's bucket; tokens of a boundary-free bucket go straight to their
+//     bin, and the few tokens of the boundary buckets are ranked pairwise by
+//     (key, position).  Only when a boundary bucket holds more than 2048
+//     tokens (many equal scores) does an exact radix select over four 8-bit
+//     digits take over;
 //   SpatialBin + joint histogram -> plug-in MI_g                        (Eq. 5);
 //   phi_g = cos(current-frame row on the patch grid, m_g); m_g update    (Eq. 8).
 // Phase 2, CTA r of the cluster works on tokens [r Lp / n, (r + 1) Lp / n):
@@ -14,12 +19,17 @@
 //   s_bar, g*, Z = sum s_bar and the entropy H (Sec. 3.6), the per-CTA
 //     partial sums exchanged through distributed shared memory;
 //   s_t = max(s_bar beta D, 0)^(1/T)                     (Eq. final_score, Eq. 9);
-//   global top-B with ties to the lower index (Sec. 3.7): one radix select
-//     whose digit histograms are summed over the cluster, then an ordered
-//     compaction whose offsets come from the lower-ranked CTAs.
+//   global top-B with ties to the lower index (Sec. 3.7): a 4096-bucket
+//     histogram over the cluster's key range, summed over the cluster, finds
+//     the boundary bucket; its tokens (at most 2048) are gathered from every
+//     CTA and ranked pairwise by (key, position); an ordered compaction with
+//     offsets from the lower-ranked CTAs writes I.  A boundary bucket with
+//     more tokens (many equal scores) falls back to an exact radix select
+//     (12 + 10 + 10-bit digits) whose digit histograms are summed over the
+//     cluster.
 // Per-KV-head selection mode: in phase 2 CTA g works on its own row instead,
 //   s_{g,t} = max(S[g,t] beta_g D_{g,t}, 0)^(1/T_g) with phi_g and the entropy of
-//   S[g, .], and the same radix select over that row alone.
+//   S[g, .], and the same bucket / pairwise select over that row alone.
 #include <algorithm>
 
 #include "common.cuh"

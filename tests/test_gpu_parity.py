@@ -101,6 +101,21 @@ def test_step_matches_oracle(name, sched):
     assert np.all(stats[8 + 4 * G:8 + 5 * G] == stats[0]) and np.all(stats[8 + 5 * G:8 + 6 * G] == stats[1])
     np.testing.assert_allclose(stats[8:8 + G], ref["mi"], rtol=2e-3, atol=2e-4)
     np.testing.assert_allclose(stats[8 + 2 * G:8 + 3 * G], ref["w"], rtol=2e-3)
+    # No visual token in the rank-bin tie band (the GPU's S puts every visual
+    # token in the same equal-frequency bin as the oracle's S): MI and the prior
+    # then differ by arithmetic alone, and w is held to 1e-4.
+    if _same_rank_bins(S_gpu, ref["S"], si.layout[0], p):
+        np.testing.assert_allclose(stats[8:8 + G], ref["mi"], rtol=1e-5, atol=1e-7)
+        np.testing.assert_allclose(stats[8 + 2 * G:8 + 3 * G], ref["w"], rtol=1e-4)
+
+
+def _same_rank_bins(S_gpu, S_ref, lay, p):
+    """Every group's visual tokens fall in the same rank bins (Sec. 3.4) under
+    the GPU's and the oracle's group score maps."""
+    lp = S_ref.shape[1]
+    vis = lay.is_visual[:lp] != 0
+    return all(np.array_equal(O.rank_bins(S_gpu[g][vis], p.mi_bins), O.rank_bins(S_ref[g][vis], p.mi_bins))
+               for g in range(S_ref.shape[0]))
 
 
 def test_select_stage_isolated_on_oracle_scores():
@@ -281,3 +296,29 @@ def test_invalid_arguments_rejected():
     with pytest.raises(sk.StarkvError) as e:
         sk.step(st, [mis], ws)
     assert e.value.status == sk.ERR_INVALID_ARG
+
+
+def test_gather_reports_a_kept_index_past_the_history():
+    """A kept index must name a past token (< L_p): the gather reports one that
+    names a window row (in bounds of the cache, so nothing faults) through the
+    device error word instead of copying the window row into the kept part."""
+    wl = syn.WORKLOADS["tiny"]
+    si = syn.make_sequence(wl)
+    st = sk.init_state(H.gpu_config(wl, H.hyper()))
+    ds = H.device_seq(si, wl)
+    ws = sk.workspace(st, [ds.seq])
+    lp = si.L - wl.window
+    good = torch.arange(si.budget, dtype=torch.int32, device="cuda")[None]
+    ds.seq.idx.copy_(good)
+    sk.compact(st, 0, [ds.seq], ws)
+    torch.cuda.synchronize()
+    sk.check_device_error(st)             # indices below L_p: no report
+    H.check_compaction(ds.seq, si, 0, wl.window)
+    bad = good.clone()
+    bad[0, -1] = lp                       # the first window row
+    ds.seq.idx.copy_(bad)
+    sk.compact(st, 0, [ds.seq], ws)
+    torch.cuda.synchronize()
+    assert sk.device_error_status(st) == sk.ERR_DEVICE
+    sk.check_device_error(st)             # the read cleared the word
+    st.close()
