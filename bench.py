@@ -188,24 +188,26 @@ class ClockSampler:
 def oracle_worker(args):
     """Times the fp64 oracle on the workload; prints one JSON line.
 
-    Budget mode (``--repeat 0``): layers 0, 1, ... of sequence 0, cycled,
-    until ``--budget-s`` seconds of oracle work have run.  Repeat mode: layer
-    0, ``--repeat`` times (the reference arm's steps)."""
+    Layers 0, 1, ... of sequence 0 (step 0 of the workload), cycled: either
+    ``--repeat`` layer compressions (the reference arm's steps) or, with
+    ``--repeat 0``, until ``--budget-s`` seconds of oracle work have run.
+    ``--budget-pct`` overrides the workload's budget as in the GPU arm."""
     from oracle import starkv_oracle as O
     from paper_2606_01790_gb300 import synthetic as syn
     wl = syn.WORKLOADS[args.workload]
     p = O.Params()
     per_head = args.select_mode == "per_head"
     spent, tokens = 0.0, 0
-    per_call = []
+    per_call, layers_done = [], []
     nl = min(wl.n_layers, args.max_layers)
-    # repeat mode: layer 0, --repeat times; budget mode: layers 0, 1, ... cycled
-    # until --budget-s seconds of oracle work have run
-    layers = [0] * args.repeat if args.repeat > 0 else (i % nl for i in range(1 << 30))
+    layers = (i % nl for i in range(args.repeat if args.repeat > 0 else 1 << 30))
     cache = {}
     for layer in layers:
         if layer not in cache:
-            cache[layer] = syn.make_sequence(wl, seq=0, layers=[layer])
+            si = syn.make_sequence(wl, seq=0, layers=[layer])
+            if args.budget_pct:
+                si.budget = syn.budget(args.budget_pct, si.n_visual_history, si.L - wl.window)
+            cache = {layer: si}   # one layer's inputs held at a time
         si = cache[layer]
         lay = si.layout[0]
         st = O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols)
@@ -215,21 +217,26 @@ def oracle_worker(args):
                      wl.window, wl.grid_rows, wl.grid_cols, st, p, per_head=per_head)
         dt = time.perf_counter() - t
         per_call.append(dt)
+        layers_done.append(layer)
         spent += dt
         tokens += si.L - wl.window
         if args.repeat == 0 and spent >= args.budget_s:
             break
     print(json.dumps(dict(tokens=tokens, seconds=spent, calls=len(per_call), per_call=per_call,
-                          l_past=syn.make_sequence(wl, seq=0, layers=[0]).L - wl.window)))
+                          layers=layers_done, l_past=si.L - wl.window, n_layers=wl.n_layers)))
 
 
-def run_oracle_subprocess(workload, budget_s=15.0, max_layers=28, repeat=0, select_mode="global"):
-    threads = str(os.cpu_count() or 1)
+def run_oracle_subprocess(workload, budget_s=15.0, max_layers=28, repeat=0, select_mode="global",
+                          threads=None, budget_pct=0):
+    """The oracle worker in a child process with ``threads`` BLAS threads
+    (default: all host cores)."""
+    threads = str(threads or os.cpu_count() or 1)
     env = dict(os.environ, OPENBLAS_NUM_THREADS=threads, OMP_NUM_THREADS=threads,
                MKL_NUM_THREADS=threads, CUDA_VISIBLE_DEVICES="")
     r = subprocess.run([sys.executable, str(ROOT / "bench.py"), "--oracle-worker", "--workload", workload,
                         "--budget-s", str(budget_s), "--max-layers", str(max_layers),
-                        "--repeat", str(repeat), "--select-mode", select_mode],
+                        "--repeat", str(repeat), "--select-mode", select_mode,
+                        "--budget-pct", str(budget_pct)],
                        capture_output=True, text=True, env=env, timeout=3600)
     if r.returncode != 0:
         raise RuntimeError(f"oracle worker failed:\n{r.stderr[-2000:]}")
@@ -238,25 +245,55 @@ def run_oracle_subprocess(workload, budget_s=15.0, max_layers=28, repeat=0, sele
     return d
 
 
+def oracle_sample(d, what):
+    """Words for a timed oracle sample, with the whole-step extrapolation."""
+    per_layer = d["seconds"] / max(1, d["calls"])
+    return (f"{what}: {d['calls']} layer compressions of sequence 0 (layers "
+            f"{min(d['layers'])}..{max(d['layers'])} cycled, step 0 of the workload), {d['tokens']} "
+            f"tokens scored in {d['seconds']:.1f} s, numpy BLAS on {d['cores']} thread(s); a whole "
+            f"{d['n_layers']}-layer step extrapolates to {d['n_layers'] * per_layer:.1f} s at this rate")
+
+
+def cpu_baselines(args):
+    """The oracle timed on the host cores: all cores (the reported
+    cpu_baseline) and one thread, each on a bounded sample."""
+    sel = args.select_mode
+    o = run_oracle_subprocess(args.workload, budget_s=args.cpu_budget_s, select_mode=sel,
+                              budget_pct=args.budget_pct)
+    one = run_oracle_subprocess(args.workload, budget_s=args.cpu_budget_s / 2, select_mode=sel, threads=1,
+                                budget_pct=args.budget_pct)
+    cpu = {"value": o["tokens"] / o["seconds"], "unit": UNIT, "cores": o["cores"], "kind": "oracle",
+           "sample": oracle_sample(o, "all host cores")}
+    cpu1 = {"value": one["tokens"] / one["seconds"], "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": oracle_sample(one, "one thread")}
+    return cpu, cpu1
+
+
 def reference_arm(args):
     """--impl reference: the fp64 oracle as it stands, one layer of the
-    workload per step, on the host cores (rank 0 only)."""
+    workload per step (layer = step mod n_layers), on the host cores (rank 0
+    only)."""
     if rank_env()[1] != 0:
         return
     from paper_2606_01790_gb300 import synthetic as syn
     wl = syn.WORKLOADS[args.workload]
-    d = run_oracle_subprocess(args.workload, repeat=args.warmup + args.steps, select_mode=args.select_mode)
+    d = run_oracle_subprocess(args.workload, repeat=args.warmup + args.steps, select_mode=args.select_mode,
+                              budget_pct=args.budget_pct)
     times = d["per_call"][args.warmup:]
+    toks = d["tokens"] * len(times) / max(1, d["calls"])   # the same L_past in every layer
     total = sum(times)
-    value = d["l_past"] * len(times) / total
-    sample = (f"layer 0 of {wl.n_layers} per step (L_past = {d['l_past']} tokens scored per step), "
-              f"numpy BLAS on {d['cores']} threads")
+    value = toks / total
+    sample = (f"one layer compression per step (layer = step mod {wl.n_layers}, sequence 0, step 0 of the "
+              f"workload; L_past = {d['l_past']} tokens scored per step), numpy BLAS on {d['cores']} "
+              f"threads; a whole {wl.n_layers}-layer step extrapolates to "
+              f"{wl.n_layers * total / len(times):.1f} s at this rate")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1e3 * total / len(times), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": args.workload, "select_mode": args.select_mode},
+        "config": {"workload": args.workload, "select_mode": args.select_mode,
+                   "budget_pct": args.budget_pct or None},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": d["cores"], "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -310,132 +347,117 @@ def window_lse_torch(si, wl, dev):
     return out
 
 
-def gpu_arm(args):
-    import numpy as np
-    import torch
-    import __graft_entry__
-    from paper_2606_01790_gb300 import starkv as sk
-    from paper_2606_01790_gb300 import synthetic as syn
+class GpuBench:
+    """Device set-up, inputs and the timed loops of the GPU arm."""
 
-    world, rank, local = rank_env()
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
-    torch.cuda.set_device(local)
-    dev = torch.device("cuda", local)
-    __graft_entry__.build()
+    def __init__(self, args):
+        import torch
+        import __graft_entry__
+        from paper_2606_01790_gb300 import starkv as sk
+        from paper_2606_01790_gb300 import synthetic as syn
+        self.torch, self.sk, self.syn, self.args = torch, sk, syn, args
+        self.world, self.rank, local = rank_env()
+        self.dist = None
+        if self.world > 1:
+            import torch.distributed as dist
+            dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+            self.dist = dist
+        torch.cuda.set_device(local)
+        self.local = local
+        self.dev = torch.device("cuda", local)
+        __graft_entry__.build()
+        self.wl = syn.WORKLOADS[args.workload]
+        self.peaks = _peaks()
 
-    wl = syn.WORKLOADS[args.workload]
-    seeds = rank_seeds(rank, wl.n_seqs)
-    sis = [syn.make_sequence(wl, seq=i, seed=s) for i, s in enumerate(seeds)]
-    cfg = sk.Config(n_layers=wl.n_layers, n_heads=wl.n_heads, n_kv_heads=wl.n_kv_heads,
-                    head_dim=wl.head_dim, window=wl.window, grid_rows=wl.grid_rows,
-                    grid_cols=wl.grid_cols, max_seqs=len(sis),
-                    select_mode=sk.SELECT_PER_HEAD if args.select_mode == "per_head" else sk.SELECT_GLOBAL)
-    st = sk.init_state(cfg)
-    G, w, d, nl = wl.n_kv_heads, wl.window, wl.head_dim, wl.n_layers
-    P = sk.sel_rows(cfg)   # rows of idx / meta_out per layer
+    def config(self, n_seqs):
+        sk, wl = self.sk, self.wl
+        return sk.Config(n_layers=wl.n_layers, n_heads=wl.n_heads, n_kv_heads=wl.n_kv_heads,
+                         head_dim=wl.head_dim, window=wl.window, grid_rows=wl.grid_rows,
+                         grid_cols=wl.grid_cols, max_seqs=n_seqs,
+                         select_mode=sk.SELECT_PER_HEAD if self.args.select_mode == "per_head"
+                         else sk.SELECT_GLOBAL)
 
-    def make_seq(si, slot, device, pin=False):
+    def with_budget(self, si):
+        if self.args.budget_pct:
+            si.budget = self.syn.budget(self.args.budget_pct, si.n_visual_history, si.L - self.wl.window)
+        return si
+
+    def make_seq(self, si, slot, P, pin=False):
+        """Device (or page-locked host) buffers of one sequence."""
+        torch, sk, wl = self.torch, self.sk, self.wl
+        G, w, d, nl = wl.n_kv_heads, wl.window, wl.head_dim, wl.n_layers
         L, B = si.L, si.budget
         words = sk.pack_meta(si.layout[0].is_visual, si.layout[0].frame, si.layout[0].row, si.layout[0].col)
         alloc = (lambda shape, dt: torch.empty(shape, dtype=dt, pin_memory=True)) if pin else \
-            (lambda shape, dt: torch.empty(shape, dtype=dt, device=device))
+            (lambda shape, dt: torch.empty(shape, dtype=dt, device=self.dev))
+
         def put(t):
             if pin:
                 o = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
                 o.copy_(t)
                 return o
-            return t.to(device)
+            return t.to(self.dev)
         return sk.Seq(k=put(si.k), v=put(si.v), q=put(si.q), meta=put(sk.meta_tensor(words)),
                       meta_layer_stride=0, L=L, cur_frame=si.cur_frame, budget=B, slot=slot,
                       k_out=alloc((nl, G, B + w, d), torch.bfloat16),
                       v_out=alloc((nl, G, B + w, d), torch.bfloat16),
                       meta_out=alloc((nl, P, B + w), torch.int32), idx=alloc((nl, P, B), torch.int32))
 
-    seqs = [make_seq(si, i, dev) for i, si in enumerate(sis)]
-    if args.lse == "given":
-        # the softmax normaliser of each window row over the past keys, as the
-        # layer's prefill attention pass supplies it (input preparation, torch)
-        for s_, si in zip(seqs, sis):
-            s_.lse = window_lse_torch(si, wl, dev)
-    ws = sk.workspace(st, seqs, device=dev)
-    stream = torch.cuda.current_stream(dev)
-    work = work_per_step(wl, [dict(L=si.L, B=si.budget) for si in sis], per_head=P > 1)
+    def barrier(self):
+        if self.dist is not None:
+            self.dist.barrier()
+        self.torch.cuda.synchronize(self.dev)
 
-    def barrier():
-        if dist is not None:
-            dist.barrier()
-        torch.cuda.synchronize(dev)
-
-    clocks = ClockSampler(local)
-    for _ in range(args.warmup):
-        sk.step(st, seqs, ws)
-    torch.cuda.synchronize(dev)
-    sk.check_device_error(st)
-    # soak: untimed steps so that clocks settle and are sampled under load
-    t_soak = time.time()
-    while time.time() - t_soak < args.soak_s:
-        for _ in range(10):
+    def time_steps(self, st, seqs, ws, steps, warmup, soak_s=0.0):
+        """Device ms of ``steps`` back-to-back starkv_step calls (CUDA events on
+        the launch stream), after ``warmup`` untimed steps and a soak; the
+        launches made in the timed region."""
+        torch, sk = self.torch, self.sk
+        for _ in range(warmup):
             sk.step(st, seqs, ws)
-        torch.cuda.synchronize(dev)
-    sk.kernel_times(st)  # reset counters
-    barrier()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        sk.step(st, seqs, ws)
-    e1.record(stream)
-    barrier()
-    t_end = time.time()
-    ms = e0.elapsed_time(e1)
-    launches = sum(v[0] for v in sk.kernel_times(st).values())   # launch counts are kept with timing off
-    sk.check_device_error(st)
-    clocks.stop()
-    ms_max = max_over_ranks(ms, dist, dev)
-    ms_step = ms_max / args.steps
-    value = job_throughput(work["tokens"], world, args.steps, ms_max)
-    # per-kernel device times in a separate pass: the event pair around every
-    # launch keeps the next kernel from starting under the previous one's tail
-    n_kt = max(1, min(args.steps, 20))
-    sk.set_timing(st, True)
-    for _ in range(n_kt):
-        sk.step(st, seqs, ws)
-    torch.cuda.synchronize(dev)
-    sk.set_timing(st, False)
-    kt = sk.kernel_times(st)
+        torch.cuda.synchronize(self.dev)
+        sk.check_device_error(st)
+        t_soak = time.time()
+        while time.time() - t_soak < soak_s:
+            for _ in range(10):
+                sk.step(st, seqs, ws)
+            torch.cuda.synchronize(self.dev)
+        sk.kernel_times(st)   # reset counters
+        self.barrier()
+        stream = torch.cuda.current_stream(self.dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            sk.step(st, seqs, ws)
+        e1.record(stream)
+        self.barrier()
+        ms = e0.elapsed_time(e1)
+        launches = sum(v[0] for v in sk.kernel_times(st).values())   # kept with timing off
+        sk.check_device_error(st)
+        return ms, launches
 
-    # roofline of the dominant kernel
-    peaks = _peaks()
-    kernels = {}
-    for kind, (n, tms) in kt.items():
-        if n == 0:
-            continue
-        kernels[kind] = {"launches": n, "avg_us": 1e3 * tms / n, "share": tms / max(1e-9, sum(v[1] for v in kt.values()))}
-    dom = max(kernels, key=lambda k: kernels[k]["avg_us"] * kernels[k]["launches"])
-    bound, units_per_step, unit = kernel_work(dom, work, peaks)
-    per_launch = units_per_step * n_kt / kernels[dom]["launches"]
-    achieved = per_launch / (kernels[dom]["avg_us"] * 1e-6)
-    peak = peaks["tc_sus"] if bound == "tensor" else peaks["hbm"]
-    traffic = recorded_traffic(dom, args.workload)
-    roofline = {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
-                "traffic": traffic, "kernel": dom,
-                "peak_src": f"{peaks['src']} ({'bf16 sustained' if bound == 'tensor' else 'HBM copy'})"}
-    step_roof_us = max(work["step_bytes"] / (peaks["hbm"] * 1e9), work["qk_flops"] / (peaks["tc"] * 1e12)) * 1e6
-    step_roofline = {"roofline_us": step_roof_us, "measured_us": 1e3 * ms_step,
-                     "frac": step_roof_us / (1e3 * ms_step), "alg_bytes": work["step_bytes"],
-                     "alg_flops": work["qk_flops"], "peak_src": peaks["src"]}
+    def kernel_pass(self, st, seqs, ws, n):
+        """Per-kernel device times in a separate pass: the event pair around
+        every launch keeps the next kernel from starting under the previous
+        one's tail.  {kind: (launches, total_ms)}."""
+        torch, sk = self.torch, self.sk
+        sk.set_timing(st, True)
+        for _ in range(n):
+            sk.step(st, seqs, ws)
+        torch.cuda.synchronize(self.dev)
+        sk.set_timing(st, False)
+        return sk.kernel_times(st)
 
-    # e2e through the public host-buffer call
-    e2e = None
-    if not args.no_e2e:
-        hseqs = [make_seq(si, i, None, pin=True) for i, si in enumerate(sis)]
-        if args.lse == "given":
-            for hs_, s_ in zip(hseqs, seqs):
+    def e2e(self, st, sis, P, n, devseqs):
+        """The same metric through starkv_step_host (page-locked host buffers,
+        copies in the timed region): (ms per step, h2d bytes, d2h bytes)."""
+        torch, sk = self.torch, self.sk
+        hseqs = [self.make_seq(si, i, P, pin=True) for i, si in enumerate(sis)]
+        for hs_, s_ in zip(hseqs, devseqs):
+            if s_.lse is not None:
                 hs_.lse = torch.empty(s_.lse.shape, dtype=torch.float32, pin_memory=True)
                 hs_.lse.copy_(s_.lse)
-        hws = sk.workspace(st, hseqs, host=True, device=dev)
+        hws = sk.workspace(st, hseqs, host=True, device=self.dev)
         # K, Q and metadata are uploaded; V is page-locked, so the gather reads
         # only its kept rows in place (the same bytes as V')
         h2d = sum(s.k.numel() * 2 + s.v_out.numel() * 2 + s.q.numel() * 2 + s.meta.numel() * 4 +
@@ -444,48 +466,201 @@ def gpu_arm(args):
                   for s in hseqs)
         for _ in range(2):
             sk.step_host(st, hseqs, hws)
-        barrier()
-        n_e2e = max(1, min(args.steps, 20))
+        self.barrier()
+        stream = torch.cuda.current_stream(self.dev)
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
-        for _ in range(n_e2e):
+        for _ in range(n):
             sk.step_host(st, hseqs, hws)
         b.record(stream)
-        barrier()
-        e_ms = max_over_ranks(a.elapsed_time(b), dist, dev)
-        e2e = {"value": job_throughput(work["tokens"], world, n_e2e, e_ms), "unit": UNIT,
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n_e2e,
-               "ms_per_step": e_ms / n_e2e}
+        self.barrier()
+        e_ms = max_over_ranks(a.elapsed_time(b), self.dist, self.dev)
         sk.check_device_error(st)
+        return e_ms / n, h2d, d2h
 
-    cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        o = run_oracle_subprocess(args.workload, budget_s=args.cpu_budget_s, max_layers=wl.n_layers,
-                                  select_mode=args.select_mode)
-        cpu = {"value": o["tokens"] / o["seconds"], "unit": UNIT, "cores": o["cores"], "kind": "oracle",
-               "sample": f"{o['calls']} layer compressions of sequence 0 (layers 0..{wl.n_layers - 1} "
-                         f"cycled; {o['tokens']} tokens scored in {o['seconds']:.1f} s, "
-                         f"numpy BLAS on {o['cores']} threads)"}
+    def roofline(self, kt, work, n_kt, workload):
+        """The dominant kernel's achieved rate against its binding peak, and its
+        share of the per-kernel pass."""
+        kernels = {}
+        total = max(1e-9, sum(v[1] for v in kt.values()))
+        for kind, (n, tms) in kt.items():
+            if n:
+                kernels[kind] = {"launches": n, "avg_us": 1e3 * tms / n, "share": tms / total}
+        dom = max(kernels, key=lambda k: kernels[k]["avg_us"] * kernels[k]["launches"])
+        bound, units_per_step, unit = kernel_work(dom, work, self.peaks)
+        per_launch = units_per_step * n_kt / kernels[dom]["launches"]
+        achieved = per_launch / (kernels[dom]["avg_us"] * 1e-6)
+        peak = self.peaks["tc_sus"] if bound == "tensor" else self.peaks["hbm"]
+        roof = {"bound": bound, "achieved": achieved, "peak": peak, "unit": unit, "frac": achieved / peak,
+                "traffic": recorded_traffic(dom, workload), "kernel": dom,
+                "scope": "the dominant kernel alone; the whole step's fraction is step_roofline.frac",
+                "peak_src": f"{self.peaks['src']} ({'bf16 sustained' if bound == 'tensor' else 'HBM copy'})"}
+        return roof, kernels
 
-    if rank == 0:
+    def step_roofline(self, work, ms_step):
+        us = max(work["step_bytes"] / (self.peaks["hbm"] * 1e9),
+                 work["qk_flops"] / (self.peaks["tc"] * 1e12)) * 1e6
+        return {"roofline_us": us, "measured_us": 1e3 * ms_step, "frac": us / (1e3 * ms_step),
+                "alg_bytes": work["step_bytes"], "alg_flops": work["qk_flops"], "peak_src": self.peaks["src"]}
+
+
+def gpu_arm(args):
+    gb = GpuBench(args)
+    if args.trajectory:
+        return trajectory_arm(gb)
+    torch, sk, syn, wl = gb.torch, gb.sk, gb.syn, gb.wl
+    seeds = rank_seeds(gb.rank, wl.n_seqs)
+    sis = [gb.with_budget(syn.make_sequence(wl, seq=i, seed=s)) for i, s in enumerate(seeds)]
+    st = sk.init_state(gb.config(len(sis)))
+    P = sk.sel_rows(st.cfg)   # rows of idx / meta_out per layer
+    seqs = [gb.make_seq(si, i, P) for i, si in enumerate(sis)]
+    if args.lse == "given":
+        # the softmax normaliser of each window row over the past keys, as the
+        # layer's prefill attention pass supplies it (input preparation, torch)
+        for s_, si in zip(seqs, sis):
+            s_.lse = window_lse_torch(si, wl, gb.dev)
+    ws = sk.workspace(st, seqs, device=gb.dev)
+    work = work_per_step(wl, [dict(L=si.L, B=si.budget) for si in sis], per_head=P > 1)
+
+    clocks = ClockSampler(gb.local)
+    t0 = time.time()
+    ms, launches = gb.time_steps(st, seqs, ws, args.steps, args.warmup, args.soak_s)
+    t_end = time.time()
+    clocks.stop()
+    ms_max = max_over_ranks(ms, gb.dist, gb.dev)
+    ms_step = ms_max / args.steps
+    value = job_throughput(work["tokens"], gb.world, args.steps, ms_max)
+    n_kt = max(1, min(args.steps, 20))
+    roofline, kernels = gb.roofline(gb.kernel_pass(st, seqs, ws, n_kt), work, n_kt, args.workload)
+    step_roofline = gb.step_roofline(work, ms_step)
+
+    e2e = None
+    if not args.no_e2e:
+        n_e2e = max(1, min(args.steps, 20))
+        e_ms, h2d, d2h = gb.e2e(st, sis, P, n_e2e, seqs)
+        e2e = {"value": job_throughput(work["tokens"], gb.world, 1, e_ms), "unit": UNIT,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n_e2e, "ms_per_step": e_ms}
+
+    cpu = cpu1 = None
+    if gb.rank == 0 and gb.world == 1 and not args.no_cpu_baseline:
+        cpu, cpu1 = cpu_baselines(args)
+
+    if gb.rank == 0:
         print(json.dumps({
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": gb.world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": args.workload, "select_mode": args.select_mode,
                        "lse": "supplied (prefill attention); first scoring pass skipped" if args.lse == "given"
-                       else "computed (both scoring passes)", "layers": nl, "seqs_per_gpu": len(sis),
-                       "L": [si.L for si in sis], "w": w, "B": [si.budget for si in sis],
-                       "H": wl.n_heads, "G": G, "d": d,
+                       else "computed (both scoring passes)", "layers": wl.n_layers, "seqs_per_gpu": len(sis),
+                       "L": [si.L for si in sis], "w": wl.window, "B": [si.budget for si in sis],
+                       "budget_pct": args.budget_pct or None, "H": wl.n_heads, "G": wl.n_kv_heads,
+                       "d": wl.head_dim,
                        "l2": f"inputs {2 * sum(s.k.numel() for s in seqs) * 2 / 1e9:.2f} GB per step "
                              "> 129 MB L2 (no flush)",
-                       "parallelism": f"replicas x{world}"},
-            "roofline": roofline, "step_roofline": step_roofline, "kernels": kernels,
-            "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
-            "clocks": clocks.summary(t_soak, t_end),
+                       "parallelism": f"replicas x{gb.world}"},
+            "step_roofline": step_roofline, "roofline": roofline, "kernels": kernels,
+            "cpu_baseline": cpu, "cpu_baseline_1thread": cpu1, "e2e": e2e, "gpu_launches": launches,
+            "clocks": clocks.summary(t0, t_end),
         }))
-    if dist is not None:
-        dist.destroy_process_group()
+    if gb.dist is not None:
+        gb.dist.destroy_process_group()
+    st.close()
+
+
+def trajectory_arm(gb):
+    """Config 3 as a trajectory: step s compresses the cache that step s - 1's
+    own compaction produced plus one new screenshot and its text, with the
+    temporal and MI state carried.  Each step is timed on its own input: the
+    slot's state is saved before the timed repeats and restored after them,
+    then the step runs once more to produce the next step's cache."""
+    import numpy as np
+    args, torch, sk, syn, wl = gb.args, gb.torch, gb.sk, gb.syn, gb.wl
+    if wl.steps <= 1 or args.select_mode != "global":
+        raise SystemExit("--trajectory needs a workload with several steps and the global selection")
+    seed = rank_seeds(gb.rank, 1)[0]
+    si = gb.with_budget(syn.make_sequence(wl, seq=0, seed=seed))
+    st = sk.init_state(gb.config(1))
+    P = sk.sel_rows(st.cfg)
+    clocks = ClockSampler(gb.local)
+    t0 = time.time()
+    rows, tok_sum, ms_sum, e2e_ms_sum, launches = [], 0, 0.0, 0.0, 0
+    kt_sum, work_sum = {}, None
+    n_kt = max(1, min(args.steps, 20))
+    h2d_sum = d2h_sum = 0
+    for step in range(wl.steps):
+        seq = gb.make_seq(si, 0, P)
+        ws = sk.workspace(st, [seq], device=gb.dev)
+        work = work_per_step(wl, [dict(L=si.L, B=si.budget)], per_head=P > 1)
+        snap = sk.export_slot(st, 0)
+        torch.cuda.synchronize(gb.dev)
+        ms, nl = gb.time_steps(st, [seq], ws, args.steps, args.warmup)
+        launches += nl
+        ms = max_over_ranks(ms, gb.dist, gb.dev)
+        kt = gb.kernel_pass(st, [seq], ws, n_kt)
+        e_ms = None
+        if not args.no_e2e:
+            sk.import_slot(st, 0, snap)
+            e_ms, h2d, d2h = gb.e2e(st, [si], P, 3, [seq])
+            e2e_ms_sum += e_ms
+            h2d_sum += h2d
+            d2h_sum += d2h
+        sk.import_slot(st, 0, snap)
+        sk.step(st, [seq], ws)   # the step itself, from the restored state
+        torch.cuda.synchronize(gb.dev)
+        sk.check_device_error(st)
+        ms_step = ms / args.steps
+        roof, kernels = gb.roofline(kt, work, n_kt, args.workload)
+        rows.append({"step": step, "L": si.L, "B": si.budget, "tokens": work["tokens"], "ms": ms_step,
+                     "tokens_per_s": work["tokens"] / (ms_step / 1e3),
+                     "step_roofline_frac": gb.step_roofline(work, ms_step)["frac"],
+                     "roofline_us": gb.step_roofline(work, ms_step)["roofline_us"],
+                     "kernels_us": {k: v["avg_us"] for k, v in kernels.items()},
+                     "e2e_ms": e_ms})
+        tok_sum += work["tokens"]
+        ms_sum += ms_step
+        for k, v in kt.items():
+            a = kt_sum.get(k, (0, 0.0))
+            kt_sum[k] = (a[0] + v[0], a[1] + v[1])
+        work_sum = work if work_sum is None else {k: work_sum[k] + work[k] for k in work}
+        if step + 1 == wl.steps:
+            break
+        lp = si.L - wl.window
+        layouts = [si.layout[l].take(np.concatenate([seq.idx[l, 0].cpu().numpy(), np.arange(lp, si.L)]))
+                   for l in range(wl.n_layers)]
+        si = gb.with_budget(syn.append_step(wl, seq.k_out.cpu(), seq.v_out.cpu(), layouts, step + 1,
+                                            si.n_visual_history, seed=seed))
+    t_end = time.time()
+    clocks.stop()
+    roofline, kernels = gb.roofline(kt_sum, work_sum, n_kt, args.workload)
+    step_roofline = gb.step_roofline(work_sum, ms_sum)
+    value = job_throughput(tok_sum, gb.world, 1, ms_sum)
+    e2e = None
+    if not args.no_e2e:
+        e2e = {"value": job_throughput(tok_sum, gb.world, 1, e2e_ms_sum), "unit": UNIT,
+               "h2d_bytes_per_step": h2d_sum / wl.steps, "d2h_bytes_per_step": d2h_sum / wl.steps,
+               "steps": 3, "ms_per_step": e2e_ms_sum / wl.steps}
+    cpu = cpu1 = None
+    if gb.rank == 0 and gb.world == 1 and not args.no_cpu_baseline:
+        cpu, cpu1 = cpu_baselines(args)
+    if gb.rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": gb.world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_sum / wl.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": args.workload, "mode": f"trajectory of {wl.steps} steps, each timed on "
+                       "its own input (the previous step's GPU compaction plus one screenshot and "
+                       f"{wl.step_text} text tokens), state carried",
+                       "select_mode": args.select_mode, "layers": wl.n_layers, "w": wl.window,
+                       "budget_pct": args.budget_pct or wl.budget_pct,
+                       "l2": "inputs 0.5-1.2 GB per step > 129 MB L2 (no flush)",
+                       "parallelism": f"replicas x{gb.world}"},
+            "trajectory_steps": rows, "step_roofline": step_roofline, "roofline": roofline,
+            "kernels": kernels, "cpu_baseline": cpu, "cpu_baseline_1thread": cpu1, "e2e": e2e,
+            "gpu_launches": launches, "clocks": clocks.summary(t0, t_end),
+        }))
+    if gb.dist is not None:
+        gb.dist.destroy_process_group()
     st.close()
 
 
@@ -501,6 +676,10 @@ def main():
     ap.add_argument("--lse", choices=["computed", "given"], default="computed",
                     help="given: the window rows' softmax normalisers are inputs (from the prefill "
                          "attention pass), so the first scoring pass is skipped")
+    ap.add_argument("--budget-pct", type=int, default=0,
+                    help="budget as this percentage of the visual tokens (0: the workload's own)")
+    ap.add_argument("--trajectory", action="store_true",
+                    help="run the workload's steps as a trajectory (config 3), timing each step")
     ap.add_argument("--soak-s", type=float, default=2.0)
     ap.add_argument("--cpu-budget-s", type=float, default=15.0)
     ap.add_argument("--no-e2e", action="store_true")

@@ -1,10 +1,13 @@
 """GPU parity at the full sizes of the five workload configs, through the C ABI
 in the launch configuration the benchmark times: one starkv_step over every
-layer of every sequence.  The layers and sequences of a step are independent
-(Algorithm 1 runs per layer), so the fp64 oracle checks sampled layers /
-sequences exactly as the single-layer tests do: fused scores within 1e-3
-relative, index sets equal except ties inside that band, compacted K/V/meta
-bit copies of the GPU's own selection."""
+layer of every sequence.  The fp64 oracle (run on a pool of spawned worker
+processes, one layer per job) checks every layer of the 28-layer benchmark
+step, every layer of the first and last steps of the 10-step trajectory (the
+oracle carries every layer's state through all ten), one layer of each of the
+16 ragged sequences (the layer rotating over the stack) and a deep layer of
+the long cache at each budget, with the single-layer rules: fused scores
+within 1e-3 relative, index sets equal except ties inside that band,
+compacted K/V/meta bit copies of the GPU's own selection."""
 import numpy as np
 import pytest
 import torch
@@ -14,6 +17,7 @@ from paper_2606_01790_gb300 import starkv as sk
 from paper_2606_01790_gb300 import synthetic as syn
 
 import harness as H
+import oracle_pool as OP
 
 pytestmark = pytest.mark.gpu
 
@@ -34,8 +38,16 @@ def _step(st, dss):
     sk.check_device_error(st)
 
 
-def _check(ds, si, layer, wl, ost, p, S=None):
-    ref = H.oracle_layer(si, layer, wl, ost, p, S_override=S)
+@pytest.fixture(scope="module")
+def pool():
+    pl = OP.OraclePool()
+    yield pl
+    pl.close()
+
+
+def _check(ds, si, layer, wl, ost, p, S=None, ref=None):
+    if ref is None:
+        ref = H.oracle_layer(si, layer, wl, ost, p, S_override=S)
     sc = H.check_scores(ds.seq.score[layer].double().cpu().numpy(), ref, ref["S"], si, layer, wl, p)
     assert sc["ok"], (layer, sc)
     ix = H.check_index_set(ds.seq.idx[layer].cpu().numpy(), ref, si.budget)
@@ -45,8 +57,8 @@ def _check(ds, si, layer, wl, ost, p, S=None):
 
 
 @pytest.mark.parametrize("sched", ["paper", "prior_on"])
-def test_28_layer_step_at_the_benchmark_shape(sched):
-    """Config 2 over the 28-layer stack (the benchmark's workload)."""
+def test_28_layer_step_at_the_benchmark_shape(sched, pool):
+    """Config 2 over the 28-layer stack (the benchmark's workload): every layer."""
     wl = syn.WORKLOADS["uitars_5shot_28l"]
     si = syn.make_sequence(wl)
     h = H.hyper() if sched == "paper" else H.hyper(n_warmup=0, n_ramp=0)
@@ -54,29 +66,35 @@ def test_28_layer_step_at_the_benchmark_shape(sched):
     st = sk.init_state(H.gpu_config(wl, h))
     ds = H.device_seq(si, wl)
     _step(st, [ds])
-    for layer in (0, 13, 27):
-        _check(ds, si, layer, wl, O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols), p)
+    fresh = lambda: O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols)
+    refs = pool.map([OP.layer_job(si, l, wl, fresh(), p) for l in range(wl.n_layers)])
+    for layer, (ref, _) in enumerate(refs):
+        _check(ds, si, layer, wl, None, p, ref=ref)
 
 
-def test_ten_step_trajectory_carries_the_state():
+def test_ten_step_trajectory_carries_the_state(pool):
     """Config 3: 28 layers, 10 steps; each step appends a screenshot and 64 text
     tokens to the compressed cache and re-compresses, with the MI and temporal
     EMAs carried.  Both sides see the same cache each step (the GPU's
-    compaction, which is checked bit-exact)."""
+    compaction, which is checked bit-exact); the oracle carries every layer's
+    state and every layer is checked on the first and the last step."""
     wl = syn.WORKLOADS["trajectory"]
     h = H.hyper(n_warmup=2, n_ramp=3)
     p = H.oracle_params(h)
     st = sk.init_state(H.gpu_config(wl, h))
-    sampled = (4, 21)
-    ost = {l: O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols) for l in sampled}
+    ost = [O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols) for _ in range(wl.n_layers)]
     si = syn.make_sequence(wl)
-    phis = []
+    phis, checked = [], 0
     for step in range(wl.steps):
         ds = H.device_seq(si, wl)
         _step(st, [ds])
-        for l in sampled:
-            ref = _check(ds, si, l, wl, ost[l], p)
+        res = pool.map([OP.layer_job(si, l, wl, ost[l], p) for l in range(wl.n_layers)])
+        for l, (ref, st_l) in enumerate(res):
+            ost[l] = st_l
             phis.append(float(np.max(ref["phi"])))
+            if step in (0, wl.steps - 1):
+                _check(ds, si, l, wl, None, p, ref=ref)
+                checked += 1
         if step + 1 == wl.steps:
             break
         lp = si.L - wl.window
@@ -86,6 +104,7 @@ def test_ten_step_trajectory_carries_the_state():
             layouts.append(si.layout[l].take(rows))
         si = syn.append_step(wl, ds.seq.k_out.cpu(), ds.seq.v_out.cpu(), layouts, step + 1,
                              si.n_visual_history)
+    assert checked == 2 * wl.n_layers
     assert max(phis) > 0.0   # the temporal discount took part
 
 
@@ -112,9 +131,10 @@ def long_input():
     return wl, si, S7
 
 
-def test_sixteen_ragged_trajectories():
+def test_sixteen_ragged_trajectories(pool):
     """Config 5: 16 independent sequences (1-12 screenshots, 128-1,024 text
-    tokens, budgets 10/20/30 %) in one batched step over 28 layers."""
+    tokens, budgets 10/20/30 %) in one batched step over 28 layers; one layer
+    of every sequence is checked, the layer rotating over the stack."""
     wl = syn.WORKLOADS["ragged"]
     h = H.hyper(n_warmup=0, n_ramp=0)
     p = H.oracle_params(h)
@@ -122,6 +142,8 @@ def test_sixteen_ragged_trajectories():
     st = sk.init_state(H.gpu_config(wl, h, max_seqs=wl.n_seqs))
     dss = [H.device_seq(si, wl, slot=i) for i, si in enumerate(sis)]
     _step(st, dss)
-    lens = [si.L for si in sis]
-    for i, layer in ((int(np.argmin(lens)), 3), (int(np.argmax(lens)), 26), (5, 14)):
-        _check(dss[i], sis[i], layer, wl, O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols), p)
+    fresh = lambda: O.LayerState.fresh(wl.n_kv_heads, wl.grid_rows, wl.grid_cols)
+    layers = [(11 * i) % wl.n_layers for i in range(wl.n_seqs)]
+    refs = pool.map([OP.layer_job(si, l, wl, fresh(), p) for si, l in zip(sis, layers)])
+    for i, (l, (ref, _)) in enumerate(zip(layers, refs)):
+        _check(dss[i], sis[i], l, wl, None, p, ref=ref)
