@@ -140,6 +140,30 @@ def window_attention_given_lse(q: np.ndarray, k: np.ndarray, window: int, lse: n
     return a_raw
 
 
+def window_attention_output(q: np.ndarray, k: np.ndarray, v: np.ndarray, window: int) -> np.ndarray:
+    """The attention output of the w window rows over the past keys, the part of
+    the layer's own attention pass that computes the logits Eq. (2) scores
+    (App. A.3 counts that Q K^T as shared with the attention):
+    O[h, i] = sum_t softmax_t(Q_{-i,h} . K_past[g(h), t] / sqrt(d)) V_past[g(h), t]
+    over t < L_past, the window keys excluded as in Eq. (2).  [H][w][d]; zeros
+    when L_past = 0.  Its softmax normaliser is ``window_lse``."""
+    H, w, d = q.shape
+    G, L, _ = k.shape
+    assert w == window and v.shape == k.shape
+    lp = L - w
+    out = np.zeros((H, w, d), np.float64)
+    if lp == 0:
+        return out
+    for h in range(H):
+        g = head_group(h, H, G)
+        z = (q[h].astype(np.float64) @ k[g, :lp].astype(np.float64).T) / math.sqrt(d)   # [w][lp]
+        z = z - z.max(axis=1, keepdims=True)
+        p = np.exp(z)
+        p = p / p.sum(axis=1, keepdims=True)
+        out[h] = p @ v[g, :lp].astype(np.float64)
+    return out
+
+
 def window_attention(q: np.ndarray, k: np.ndarray, window: int) -> np.ndarray:
     """Sec. 3.3, Eq. (2): A_raw[h, t] = sum over the w
     window queries of softmax_t(Q_{-i,h} . K_past[g(h), t] / sqrt(d)).

@@ -537,6 +537,53 @@ def test_attention_with_the_exact_normaliser_is_the_softmax_sum():
     np.testing.assert_allclose(shifted, O.window_attention(q, k, 5) * math.exp(-0.5), rtol=1e-12)
 
 
+def test_window_attention_output_vs_torch_sdpa():
+    """The attention output of the window rows over the past keys against
+    torch's scaled_dot_product_attention in float64 (GQA by repeating each
+    group's keys and values for its heads)."""
+    r = _rng(62)
+    H, G, w, L, d = 8, 2, 4, 70, 16
+    q, k, v = r.standard_normal((H, w, d)) * 2, r.standard_normal((G, L, d)), r.standard_normal((G, L, d))
+    got = O.window_attention_output(q, k, v, w)
+    kk = torch.from_numpy(k[:, :L - w]).repeat_interleave(H // G, dim=0)
+    vv = torch.from_numpy(v[:, :L - w]).repeat_interleave(H // G, dim=0)
+    ref = F.scaled_dot_product_attention(torch.from_numpy(q), kk, vv)
+    np.testing.assert_allclose(got, ref.numpy(), rtol=1e-12, atol=1e-13)
+    # the window's own keys and values take no part
+    k2, v2 = k.copy(), v.copy()
+    k2[:, L - w:] = 100.0
+    v2[:, L - w:] = -7.0
+    np.testing.assert_allclose(O.window_attention_output(q, k2, v2, w), got, rtol=1e-13)
+    assert np.all(O.window_attention_output(q, k[:, :w], v[:, :w], w) == 0.0)   # no past keys
+
+
+def test_window_attention_output_limits_and_normaliser():
+    """Zero queries give the mean of the past values; a query aligned with one
+    key far above the rest gives that key's value; exp(lse) O is the
+    unnormalised sum of exp(z) V."""
+    r = _rng(63)
+    H, G, w, L, d = 4, 2, 3, 40, 8
+    k, v = r.standard_normal((G, L, d)), r.standard_normal((G, L, d))
+    lp = L - w
+    out = O.window_attention_output(np.zeros((H, w, d)), k, v, w)
+    for h in range(H):
+        np.testing.assert_allclose(out[h], np.broadcast_to(v[h * G // H, :lp].mean(axis=0), (w, d)), rtol=1e-12)
+    kb = k.copy()
+    kb[:, 11] *= 10.0 / np.linalg.norm(kb[:, 11], axis=1, keepdims=True)   # key 11: length 10
+    q = np.zeros((H, w, d))
+    for h in range(H):
+        q[h] = 2.0 * kb[h * G // H, 11]    # logit 200 / sqrt(d) at key 11, far below elsewhere
+    out = O.window_attention_output(q, kb, v, w)
+    for h in range(H):
+        np.testing.assert_allclose(out[h], np.broadcast_to(v[h * G // H, 11], (w, d)), atol=1e-6)
+    q = r.standard_normal((H, w, d))
+    out, lse = O.window_attention_output(q, k, v, w), O.window_lse(q, k, w)
+    for h in range(H):
+        g = h * G // H
+        z = q[h] @ k[g, :lp].T / math.sqrt(d)
+        np.testing.assert_allclose(np.exp(lse[h])[:, None] * out[h], np.exp(z) @ v[g, :lp], rtol=1e-12)
+
+
 # ------------------------------------------------------------------ ablation variants (readings)
 
 def test_decay_variants_limits_and_ordering():
