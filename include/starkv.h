@@ -167,6 +167,14 @@ typedef struct {
                                    every sequence of a call gives it, the first
                                    scoring pass (a whole read of K) is skipped.
                                    NULL = computed.                                 */
+  float* attn_o;                /* f32 [n_layers][H][w][d], optional: written by
+                                   starkv_window_attention (the window rows'
+                                   attention output over the past keys); 16-byte
+                                   aligned                                          */
+  float* attn_lse;              /* f32 [n_layers][H][w]: written by
+                                   starkv_window_attention, each window row's
+                                   natural-log normaliser over the past keys, the
+                                   value `lse` takes                                */
 } starkv_seq;
 
 /* Per-layer diagnostics written to starkv_seq.stats (floats):
@@ -242,7 +250,8 @@ starkv_status starkv_import_slot(starkv_state* st, int32_t slot, const void* hos
 starkv_status starkv_get_config(const starkv_state* st, starkv_config* out);
 
 /* Bytes of device workspace that starkv_score_layer, starkv_select,
- * starkv_compact and starkv_step need for this batch (the maximum of the four).
+ * starkv_compact, starkv_step and starkv_window_attention need for this batch
+ * (the maximum of the five).
  * With host != 0: the bytes starkv_step_host needs (adds staging copies). */
 starkv_status starkv_workspace_bytes(const starkv_state* st, const starkv_seq* seqs, int32_t nseq,
                                      int32_t host, size_t* bytes);
@@ -280,6 +289,25 @@ starkv_status starkv_score_layer(starkv_state* st, int32_t layer, const starkv_s
  * was created. */
 starkv_status starkv_score_layer_noalloc(starkv_state* st, int32_t layer, const starkv_seq* seqs,
                                          int32_t nseq, void* stream);
+
+/* The attention pass whose logits Eq. (2) scores (Sec. 3.3; App. A.3 counts the
+ * compression's Q K^T as shared with the model's attention): for every layer of
+ * every sequence and every window row r = (h, i),
+ *   attn_o[r]   = sum_{t < L_p} softmax_t(Q_{-i,h} . K[g(h), t] / sqrt(d)) V[g(h), t]
+ *   attn_lse[r] = log sum_{t < L_p} exp(Q_{-i,h} . K[g(h), t] / sqrt(d))
+ * over the past keys only (the window keys excluded, as in Eq. 2; a model's
+ * causal attention for these rows merges in the window keys' part by the
+ * usual log-sum-exp rule).  attn_lse is exactly what `lse` takes, so a caller
+ * that runs this pass (or its own attention kernel with the same output)
+ * lets starkv_step skip its first scoring pass.  Reads k, v, q; writes attn_o
+ * (skipped when NULL) and attn_lse (required; -inf and a zero output when
+ * L_p = 0).  Tensor cores: Q K^T in bf16, P V with P rounded to fp16 and V
+ * converted to fp16 (|v| must stay below 65504), fp32 accumulation, so
+ * |attn_o - O| <= 2^-11 sum_t p_t |V_t| + fp32 rounding, and attn_lse carries
+ * the fp32 accuracy of the scoring passes.  Workspace from
+ * starkv_workspace_bytes. */
+starkv_status starkv_window_attention(starkv_state* st, const starkv_seq* seqs, int32_t nseq,
+                                      void* workspace, size_t workspace_bytes, void* stream);
 
 /* Sec. 3.3 - 3.7 after the group score map (Eq. 4 to Eq. 10): from
  * S of layer `layer`: s_bar, g*, online MI per group (Eq. 5) -> EMA (Eq. 6) ->
@@ -342,7 +370,9 @@ enum {
                                      (Sec. 3.4-3.7): one cluster of min(G, 8) CTAs per
                                      layer                                                 */
   STARKV_KERNEL_COMPACT = 4,      /* KV gather (Eq. 11)                                    */
-  STARKV_NUM_KERNELS = 5
+  STARKV_KERNEL_ATTENTION = 5,    /* window-row attention over the past keys (pieces)      */
+  STARKV_KERNEL_ATTN_COMBINE = 6, /* merge of its pieces into attn_o / attn_lse            */
+  STARKV_NUM_KERNELS = 7
 };
 
 /* Kernel timing, a profiling aid.  While `on` is non-zero every kernel launch

@@ -18,7 +18,7 @@ CSRC = PKG / "csrc"
 BUILD = PKG / "_build"
 LIB = PKG / "libstarkv.so"
 INCLUDE = PKG.parent / "include"
-SOURCES = ["api.cu", "score.cu", "select.cu", "compact.cu"]
+SOURCES = ["api.cu", "score.cu", "select.cu", "compact.cu", "attn.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", f"-I{INCLUDE}"]
 

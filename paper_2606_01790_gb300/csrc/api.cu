@@ -14,6 +14,7 @@
 #include <string>
 #include <vector>
 
+#include "attn.cuh"
 #include "common.cuh"
 #include "compact.cuh"
 #include "score.cuh"
@@ -133,6 +134,8 @@ const char* kernel_range_name(int kind) {
     case STARKV_KERNEL_POOL: return "starkv: pooling";
     case STARKV_KERNEL_CALIBRATE: return "starkv: calibration + top-B";
     case STARKV_KERNEL_COMPACT: return "starkv: compaction";
+    case STARKV_KERNEL_ATTENTION: return "starkv: window attention (pieces)";
+    case STARKV_KERNEL_ATTN_COMBINE: return "starkv: window attention (combine)";
     default: return "starkv: kernel";
   }
 }
@@ -228,9 +231,10 @@ starkv_status validate_seqs(const starkv_state* st, const starkv_seq* seqs, int 
         return set_error(STARKV_ERR_INVALID_ARG, "seq %d: meta_layer_stride must be 0 or >= (G-1)*meta_group_stride + L", i);
     }
     // 4-byte words: a misaligned pointer is an argument error, not a device fault
-    const void* words[] = {s.meta, s.meta_out, s.idx, s.S, s.score, s.stats, s.lse};
+    const void* words[] = {s.meta, s.meta_out, s.idx, s.S, s.score, s.stats, s.lse, s.attn_lse};
     for (const void* w : words)
       if (w && !aligned4(w)) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: a 4-byte array is not 4-byte aligned", i);
+    if (s.attn_o && !aligned16(s.attn_o)) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: attn_o not 16-byte aligned", i);
     if ((need & kNeedS) && !s.S && lp > 0) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: S is NULL", i);
     if ((need & kNeedIdx) && !s.idx && s.budget > 0) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: idx is NULL", i);
     if (need & kNeedOut) {
@@ -486,6 +490,90 @@ size_t seq_bytes_out(const starkv_config& c, const starkv_seq& s) {
   return b;
 }
 
+// ---- window attention (attn.cu): workspace and launches
+
+int64_t attn_units(const starkv_config& c, const starkv_seq* seqs, int i0, int i1) {
+  int64_t u = 0;
+  for (int i = i0; i < i1; ++i)
+    u += static_cast<int64_t>(c.n_layers) * c.n_kv_heads * ((seqs[i].L - c.window + kAttnUnitKeys - 1) / kAttnUnitKeys);
+  return u;
+}
+
+// Piece partials of one launch batch: (m, l) and the unnormalised output per slot.
+void attn_regions(const starkv_state* st, int nrows, int64_t units, int* grid, size_t* ml_bytes, size_t* o_bytes) {
+  *grid = units > 0 ? static_cast<int>(std::min<int64_t>(units, st->num_sms)) : 0;
+  const size_t slots = static_cast<size_t>(attn_slots(nrows, *grid));
+  *ml_bytes = align256(slots * kMaxRows * sizeof(float2));
+  *o_bytes = align256(slots * kMaxRows * kHeadDim * sizeof(float));
+}
+
+size_t attn_ws_bytes(const starkv_state* st, const starkv_seq* seqs, int nseq) {
+  const starkv_config& c = st->cfg;
+  size_t best = 0;
+  for (int i0 = 0; i0 < nseq; i0 += kMaxBatch) {
+    const int i1 = std::min(nseq, i0 + kMaxBatch);
+    int grid;
+    size_t ml, o;
+    attn_regions(st, (i1 - i0) * c.n_layers * c.n_kv_heads, attn_units(c, seqs, i0, i1), &grid, &ml, &o);
+    best = std::max(best, ml + o);
+  }
+  return best;
+}
+
+starkv_status run_attention(starkv_state* st, const starkv_seq* seqs, int nseq, void* workspace, size_t ws_bytes,
+                            cudaStream_t stream) {
+  const starkv_config& c = st->cfg;
+  const int G = c.n_kv_heads, H = c.n_heads, w = c.window;
+  starkv_status s = check_ws(st, workspace, ws_bytes, attn_ws_bytes(st, seqs, nseq));
+  if (s != STARKV_OK) return s;
+  if ((s = get_encoder()) != STARKV_OK) return s;
+  static thread_local AttnParams p;   // ~17 KB: kept off the stack
+  char* ws = static_cast<char*>(workspace);
+  for (int i0 = 0; i0 < nseq; i0 += kMaxBatch) {
+    const int i1 = std::min(nseq, i0 + kMaxBatch);
+    memset(&p, 0, sizeof(p));
+    p.nseq = i1 - i0;
+    p.layer0 = 0;
+    p.nlayers = c.n_layers;
+    p.G = G;
+    p.rows = (H / G) * w;
+    p.n_mtiles = (p.rows + 127) / 128;
+    p.q_rows = (p.rows + 15) & ~15;
+    p.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(kHeadDim)));
+    int64_t units = 0;
+    for (int i = i0; i < i1; ++i) {
+      const starkv_seq& q = seqs[i];
+      AttnSeq& a = p.seq[i - i0];
+      a.Lp = q.L - w;
+      a.nu = (a.Lp + kAttnUnitKeys - 1) / kAttnUnitKeys;
+      a.unit_base = units;
+      a.o = q.attn_o;
+      a.lse = q.attn_lse;
+      units += static_cast<int64_t>(c.n_layers) * G * a.nu;
+      if (a.nu == 0) continue;
+      const uint64_t zkv = static_cast<uint64_t>(c.n_layers) * G, qrows = static_cast<uint64_t>(H) * w;
+      if ((s = encode_3d(&p.tmk[i - i0], q.k, kHeadDim, q.L, zkv, kAttnUnitKeys)) != STARKV_OK) return s;
+      if ((s = encode_3d(&p.tmv[i - i0], q.v, kHeadDim, q.L, zkv, kAttnUnitKeys)) != STARKV_OK) return s;
+      if ((s = encode_3d(&p.tmqa[i - i0], q.q, kHeadDim, qrows, c.n_layers, std::min(p.rows, 128))) != STARKV_OK)
+        return s;
+      if (p.rows > 128 &&
+          (s = encode_3d(&p.tmqb[i - i0], q.q, kHeadDim, qrows, c.n_layers, p.rows - 128)) != STARKV_OK)
+        return s;
+    }
+    size_t ml_bytes, o_bytes;
+    attn_regions(st, p.nseq * c.n_layers * G, units, &p.grid, &ml_bytes, &o_bytes);
+    p.total_units = units;
+    p.part_ml = reinterpret_cast<float2*>(ws);
+    p.part_o = reinterpret_cast<float*>(ws + ml_bytes);
+    p.err = st->dev.err;
+    p.wait_ns = st->wait_ns;
+    if (units > 0)
+      CUDA_TRY(launch(st, STARKV_KERNEL_ATTENTION, stream, [&] { return attn_main_launch(p, stream); }));
+    CUDA_TRY(launch(st, STARKV_KERNEL_ATTN_COMBINE, stream, [&] { return attn_combine_launch(p, stream); }));
+  }
+  return STARKV_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -531,6 +619,7 @@ starkv_status starkv_init_state(const starkv_config* cfg, starkv_state** out, vo
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&st->num_sms, cudaDevAttrMultiProcessorCount, st->device);
   if (e == cudaSuccess) e = score_configure();
   if (e == cudaSuccess) e = select_configure();
+  if (e == cudaSuccess) e = attn_configure();
   if (e != cudaSuccess) {
     delete st;
     return set_error(STARKV_ERR_CUDA, "device setup failed: %s", cudaGetErrorString(e));
@@ -720,7 +809,7 @@ starkv_status starkv_workspace_bytes(const starkv_state* st, const starkv_seq* s
   plan_ws(st, seqs, nseq, st->cfg.n_layers, true, true, &a);   // starkv_step
   plan_ws(st, seqs, nseq, 1, false, false, &b);                 // starkv_score_layer, starkv_compact
   plan_ws(st, seqs, nseq, 1, false, true, &c1);                 // starkv_select
-  size_t total = std::max(a.total, std::max(b.total, c1.total));
+  size_t total = std::max(std::max(a.total, attn_ws_bytes(st, seqs, nseq)), std::max(b.total, c1.total));
   if (host) {
     std::vector<starkv_seq> dev(seqs, seqs + nseq);
     size_t staged = 0;
@@ -774,6 +863,17 @@ starkv_status starkv_step(starkv_state* st, const starkv_seq* seqs, int32_t nseq
   if ((s = check_device(st)) != STARKV_OK) return s;
   return run_stages(st, seqs, nseq, 0, st->cfg.n_layers, kScore | kStatsRaw | kSelect | kCompact, workspace,
                     workspace_bytes, static_cast<cudaStream_t>(stream));
+}
+
+starkv_status starkv_window_attention(starkv_state* st, const starkv_seq* seqs, int32_t nseq, void* workspace,
+                                      size_t workspace_bytes, void* stream) {
+  NvtxRange range("starkv_window_attention");
+  starkv_status s = validate_seqs(st, seqs, nseq, kNeedK | kNeedQ | kNeedV);
+  if (s != STARKV_OK) return s;
+  for (int i = 0; i < nseq; ++i)
+    if (!seqs[i].attn_lse) return set_error(STARKV_ERR_INVALID_ARG, "seq %d: attn_lse is NULL", i);
+  if ((s = check_device(st)) != STARKV_OK) return s;
+  return run_attention(st, seqs, nseq, workspace, workspace_bytes, static_cast<cudaStream_t>(stream));
 }
 
 starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t nseq, void* workspace,

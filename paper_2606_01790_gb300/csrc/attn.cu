@@ -1,0 +1,599 @@
+// Attention output and softmax normaliser of the window rows over the past
+// keys: the part of a layer's own attention pass that computes the logits the
+// compression scores (Sec. 3.3, Eq. 2; App. A.3 counts that Q K^T as shared
+// with the attention).  For every (layer, group) row block of (H/G) w window
+// rows r against the L_p past keys t (the window keys excluded, as in Eq. 2):
+//   O[r]   = sum_t softmax_t(Q_r . K_t / sqrt(d)) V_t
+//   lse[r] = log sum_t exp(Q_r . K_t / sqrt(d))       (natural log)
+// lse is what starkv_seq.lse takes, so the compression can skip its first
+// scoring pass (a whole read of K).  A model's causal attention for these
+// rows adds the window keys' part by the usual log-sum-exp merge.
+//
+// Work split: the flat (seq, layer, group, 64-key unit) space in one
+// contiguous range per CTA (persistent grid <= #SMs).  A run of units of one
+// row inside a range is a piece; its partial (reference m, sum l, unnormalised
+// O) goes to slot row + CTA (distinct for every piece: ranges and rows are
+// both in flat order) and k_attn_combine merges the pieces of each row.
+//
+// Per unit on tcgen05, with two 128-row M tiles for up to 256 window rows:
+//   S = Q K^T           M = 128 rows, N = 64 keys, K = d, bf16 -> fp32 in TMEM
+//                       (two S stages, so the MMA of unit u+1 runs under the
+//                       softmax of unit u);
+//   softmax             rows on TMEM lanes, one thread per row: p = exp2(S c - m),
+//                       l += p in fp32, P rounded to fp16 into shared memory
+//                       (128-byte swizzled K-major rows, two buffers);
+//   O += P V            M = 128, N = d = 128, K = 64 keys, fp16 -> fp32 in TMEM;
+//                       V arrives as bf16 and four warps convert it to fp16 in
+//                       place (exact for |v| < 65504), read as the transposed
+//                       (MN-major) operand.
+// The row reference m is the first unit's maximum and moves only when a
+// unit's maximum exceeds it by more than 15 (fp16 holds P < 2^16); the move
+// rescales that row's O in TMEM after the previous unit's P V is done (rare).
+// Warp roles: warp 0 TMA producer (K and V through a three-stage ring, Q per
+// piece), warp 1 MMA issuer and TMEM owner, warps 4..11 softmax (warpgroup =
+// M tile), warps 12..15 V conversion.
+#include <algorithm>
+#include <utility>
+
+#include <cuda_fp16.h>
+
+#include "attn.cuh"
+#include "common.cuh"
+#include "ptx.cuh"
+
+namespace starkv {
+
+namespace {
+
+constexpr int kStages = 3;                        // K/V ring depth
+constexpr int kUnitBytes = kAttnUnitKeys * 256;   // 64 keys x 128 bf16: 16 KB (K or V)
+constexpr int kHalfBytes = kAttnUnitKeys * 128;   // one 64-column half of a unit: 8 KB
+constexpr int kStageBytes = 2 * kUnitBytes;       // K then V
+constexpr int kPTileBytes = 128 * 128;            // one M tile of P: 128 rows x 64 fp16
+constexpr int kTmemCols = 512;                    // O [0, 256), S stage t at 256 + 128 t
+constexpr int kSoftWarp0 = 4, kSoftWarps = 8;
+constexpr int kConvWarp0 = 12, kConvWarps = 4;
+constexpr uint32_t kFull = 0xffffffffu;
+constexpr float kMoveThreshold = 15.f;            // log2 units: P stays below 2^16
+constexpr uint64_t kDrainWaitNs = 2000000000ull;
+constexpr size_t kSmemLimit = 227 * 1024;
+
+__device__ __forceinline__ uint64_t drain_limit(uint64_t wait_ns) {
+  return wait_ns > kDrainWaitNs ? wait_ns : kDrainWaitNs;
+}
+
+struct AttnCtl {
+  uint64_t kv_full[kStages], kv_empty[kStages], v_ready[kStages];
+  uint64_t s_full[2], s_empty[2];
+  uint64_t p_full[2], p_empty[2];
+  uint64_t q_full, q_empty, drain;
+  uint32_t tmem_base;
+  volatile int abort;
+};
+
+static_assert(sizeof(AttnCtl) <= 256, "the control block has 256 bytes");
+
+__device__ __forceinline__ void fail(AttnCtl* ctl, uint32_t* err) {
+  ctl->abort = 1;
+  atomicOr(err, kErrTimeout);
+}
+
+// Shared-memory descriptor of an MN-major operand in 128-byte swizzled rows
+// (TMA SWIZZLE_128B of a [K][MN] tile, MN contiguous): 64-element MN groups
+// `lbo` bytes apart, 8-row K groups `sbo` bytes apart.
+__device__ __forceinline__ uint64_t sdesc_mn_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+  d |= static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16;
+  d |= static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32;
+  d |= static_cast<uint64_t>(1) << 46;   // descriptor version (tcgen05)
+  d |= static_cast<uint64_t>(2) << 61;   // swizzle mode: 128 B
+  return d;
+}
+
+// Instruction descriptor of tcgen05.mma kind::f16 with fp16 A (K-major) and
+// fp16 B (MN-major), fp32 accumulator, shape M x N.
+__host__ __device__ constexpr uint32_t idesc_f16_bmn(int M, int N) {
+  return (1u << 4)                                   // D format: f32
+         | (1u << 16)                                // B major: MN
+         | (static_cast<uint32_t>(N >> 3) << 17)
+         | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                        uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// 16 consecutive fp32 columns of this warp's 32 TMEM lanes, stored.
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+      "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};\n" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+      "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+      : "memory");
+}
+
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+__device__ __forceinline__ uint32_t pack_half2(float a, float b) {
+  const __half2 h = __floats2half2_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// bf16 pair (one 32-bit word) -> fp16 pair, exact for |x| < 65504
+__device__ __forceinline__ uint32_t bf16x2_to_f16x2(uint32_t w) {
+  return pack_half2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+}
+
+// Coordinates of consecutive flat units [f0, f1), advanced without divisions.
+struct UnitIter {
+  int s, l, g, j, nu;
+  int64_t f, fe;
+  __device__ void init(const AttnParams& p, int64_t f0, int64_t f1) {
+    f = f0;
+    fe = f1;
+    s = l = g = j = nu = 0;
+    if (f >= fe) return;
+    while (s + 1 < p.nseq && p.seq[s + 1].unit_base <= f0) ++s;
+    nu = p.seq[s].nu;
+    const int64_t u = f0 - p.seq[s].unit_base;
+    const int per_layer = p.G * nu;
+    l = static_cast<int>(u / per_layer);
+    const int rem = static_cast<int>(u - static_cast<int64_t>(l) * per_layer);
+    g = rem / nu;
+    j = rem - g * nu;
+  }
+  __device__ bool valid() const { return f < fe; }
+  __device__ bool first(int64_t fb) const { return f == fb || j == 0; }
+  __device__ bool last() const { return f + 1 == fe || j + 1 == nu; }
+  __device__ int row(const AttnParams& p) const { return (s * p.nlayers + l) * p.G + g; }
+  __device__ void next(const AttnParams& p) {
+    ++f;
+    if (f >= fe) return;
+    if (++j < nu) return;
+    j = 0;
+    if (++g < p.G) return;
+    g = 0;
+    if (++l < p.nlayers) return;
+    l = 0;
+    do {
+      ++s;
+    } while (s + 1 < p.nseq && p.seq[s].nu == 0);
+    nu = p.seq[s].nu;
+  }
+};
+
+__device__ __forceinline__ int64_t range_begin(int64_t T, int c, int P) { return T * c / P; }
+
+// CTA whose range holds flat unit f
+__host__ __device__ __forceinline__ int cta_of(int64_t f, int64_t T, int P) {
+  return static_cast<int>(((f + 1) * P - 1) / T);
+}
+
+__device__ void producer_loop(const AttnParams& p, AttnCtl* ctl, uint8_t* sQ, uint8_t* sKV, int64_t fb,
+                              int64_t fe) {
+  const uint64_t pol = policy_evict_first();   // K and V stream through L2 once
+  const int qhalf = p.q_rows * 128;
+  int stage = 0, phase = 0, pc = 0, last_q_pc = -1;
+  int last_ph[kStages];
+  for (int i = 0; i < kStages; ++i) last_ph[i] = -1;
+  UnitIter c;
+  for (c.init(p, fb, fe); c.valid(); c.next(p)) {
+    if (ctl->abort) break;
+    if (c.first(fb)) {
+      if (!mbar_wait(&ctl->q_empty, (pc & 1) ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
+      const int zq = p.layer0 + c.l, y = c.g * p.rows;
+      mbar_arrive_expect_tx(&ctl->q_full, p.rows * 256);
+      for (int h = 0; h < 2; ++h) {
+        tma_load_3d(sQ + h * qhalf, &p.tmqa[c.s], &ctl->q_full, h * 64, y, zq);
+        if (p.rows > 128) tma_load_3d(sQ + h * qhalf + 128 * 128, &p.tmqb[c.s], &ctl->q_full, h * 64, y + 128, zq);
+      }
+      last_q_pc = pc;
+      ++pc;
+    }
+    if (!mbar_wait(&ctl->kv_empty[stage], phase ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
+    mbar_arrive_expect_tx(&ctl->kv_full[stage], kStageBytes);
+    const int zk = (p.layer0 + c.l) * p.G + c.g, y = c.j * kAttnUnitKeys;
+    uint8_t* st = sKV + stage * kStageBytes;
+    for (int h = 0; h < 2; ++h) {
+      tma_load_3d_hint(st + h * kHalfBytes, &p.tmk[c.s], &ctl->kv_full[stage], h * 64, y, zk, pol);
+      tma_load_3d_hint(st + kUnitBytes + h * kHalfBytes, &p.tmv[c.s], &ctl->kv_full[stage], h * 64, y, zk, pol);
+    }
+    last_ph[stage] = phase;
+    if (++stage == kStages) {
+      stage = 0;
+      phase ^= 1;
+    }
+  }
+  if (ctl->abort) {   // every issued copy completes before the CTA can exit
+    for (int i = 0; i < kStages; ++i)
+      if (last_ph[i] >= 0) mbar_wait(&ctl->kv_full[i], last_ph[i], drain_limit(p.wait_ns));
+    if (last_q_pc >= 0) mbar_wait(&ctl->q_full, last_q_pc & 1, drain_limit(p.wait_ns));
+  }
+}
+
+// Single MMA issuer: S(u) into S stage u & 1, then O += P(u - 1) V(u - 1)
+// once the softmax has written P(u - 1), so that the product of one unit runs
+// while the softmax of the next is computed.
+__device__ void mma_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sQ, const uint8_t* sKV,
+                         const uint8_t* sP, uint32_t tmem, int64_t fb, int64_t fe) {
+  const uint32_t idesc_s = idesc_bf16(128, kAttnUnitKeys);
+  const uint32_t idesc_o = idesc_f16_bmn(128, kHeadDim);
+  const uint64_t dq0 = sdesc_k_sw128(smem_u32(sQ));
+  const uint32_t qhalf16 = (p.q_rows * 128) >> 4;
+  int stage = 0, kphase = 0, pc = 0;
+  bool pend = false, pend_first = false;
+  int pend_stage = 0, pend_vph = 0;
+  int64_t ui = 0;
+  auto issue_pv = [&](int st, int vph, int64_t u, bool first_of_piece) -> bool {
+    const int b = static_cast<int>(u & 1);
+    if (!mbar_wait(&ctl->v_ready[st], vph, p.wait_ns)) return false;
+    if (!mbar_wait(&ctl->p_full[b], static_cast<uint32_t>((u >> 1) & 1), p.wait_ns)) return false;
+    tc_fence_after();
+    const uint64_t dv = sdesc_mn_sw128(smem_u32(sKV + st * kStageBytes + kUnitBytes), kHalfBytes, 1024);
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt) {
+      if (mt >= p.n_mtiles) break;
+      const uint64_t dp = sdesc_k_sw128(smem_u32(sP + (b * 2 + mt) * kPTileBytes));
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)   // 16 keys per step: +32 B along the P row, +16 rows of V
+        mma_f16(tmem + mt * kHeadDim, dp + static_cast<uint64_t>(kk * 2), dv + static_cast<uint64_t>(kk * 128),
+                idesc_o, (!first_of_piece || kk > 0) ? 1u : 0u);
+    }
+    mma_commit(&ctl->kv_empty[st]);
+    mma_commit(&ctl->p_empty[b]);
+    return true;
+  };
+  UnitIter c;
+  for (c.init(p, fb, fe); c.valid(); c.next(p), ++ui) {
+    if (ctl->abort) break;
+    const bool first = c.first(fb);
+    if (first) {
+      if (!mbar_wait(&ctl->q_full, pc & 1, p.wait_ns)) { fail(ctl, p.err); break; }
+      ++pc;
+    }
+    const int t = static_cast<int>(ui & 1);
+    if (!mbar_wait(&ctl->kv_full[stage], kphase, p.wait_ns)) { fail(ctl, p.err); break; }
+    if (!mbar_wait(&ctl->s_empty[t], static_cast<uint32_t>(((ui >> 1) & 1) ^ 1), p.wait_ns)) { fail(ctl, p.err); break; }
+    tc_fence_after();
+    const uint64_t dk = sdesc_k_sw128(smem_u32(sKV + stage * kStageBytes));
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt) {
+      if (mt >= p.n_mtiles) break;
+      // M tile 1 reads rows 128..255 of each Q half; rows past q_rows feed
+      // accumulator rows that no thread reads
+      const uint64_t dq = dq0 + static_cast<uint64_t>(mt * ((128 * 128) >> 4));
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint32_t koff16 = (kk >> 2) * (kHalfBytes >> 4) + (kk & 3) * 2;
+        const uint32_t qoff16 = (kk >> 2) * qhalf16 + (kk & 3) * 2;
+        mma_bf16(tmem + 256 + t * 128 + mt * kAttnUnitKeys, dq + qoff16, dk + koff16, idesc_s, kk > 0);
+      }
+    }
+    mma_commit(&ctl->s_full[t]);
+    if (c.last()) mma_commit(&ctl->q_empty);
+    if (pend && !issue_pv(pend_stage, pend_vph, ui - 1, pend_first)) { fail(ctl, p.err); pend = false; break; }
+    pend = true;
+    pend_first = first;
+    pend_stage = stage;
+    pend_vph = kphase;
+    if (++stage == kStages) {
+      stage = 0;
+      kphase ^= 1;
+    }
+  }
+  if (pend && !ctl->abort && !issue_pv(pend_stage, pend_vph, ui - 1, pend_first)) fail(ctl, p.err);
+  // every MMA issued above must be complete before TMEM is released
+  mma_commit(&ctl->drain);
+  mbar_wait(&ctl->drain, 0, drain_limit(p.wait_ns));
+}
+
+}  // namespace
+
+__global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_constant__ AttnParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem;                              // [2 halves][q_rows][128 B]
+  uint8_t* sKV = sQ + 2 * p.q_rows * 128;          // [kStages][K 16 KB | V 16 KB]
+  uint8_t* sP = sKV + kStages * kStageBytes;       // [2 buffers][2 M tiles][128 rows][128 B]
+  AttnCtl* ctl = reinterpret_cast<AttnCtl*>(sP + 4 * kPTileBytes);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kStages; ++i) {
+      mbar_init(&ctl->kv_full[i], 1);
+      mbar_init(&ctl->kv_empty[i], 1);
+      mbar_init(&ctl->v_ready[i], kConvWarps);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&ctl->s_full[i], 1);
+      mbar_init(&ctl->s_empty[i], kSoftWarps);
+      mbar_init(&ctl->p_full[i], kSoftWarps);
+      mbar_init(&ctl->p_empty[i], 1);
+    }
+    mbar_init(&ctl->q_full, 1);
+    mbar_init(&ctl->q_empty, 1);
+    mbar_init(&ctl->drain, 1);
+    ctl->abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&ctl->tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  griddep_launch_dependents();
+  griddep_wait();
+  const uint32_t tmem = ctl->tmem_base;
+  const int64_t T = p.total_units;
+  const int64_t fb = range_begin(T, blockIdx.x, gridDim.x);
+  const int64_t fe = range_begin(T, blockIdx.x + 1, gridDim.x);
+
+  if (warp == 0) {
+    if (lane == 0) producer_loop(p, ctl, sQ, sKV, fb, fe);
+  } else if (warp == 1) {
+    if (lane == 0) mma_loop(p, ctl, sQ, sKV, sP, tmem, fb, fe);
+  } else if (warp >= kSoftWarp0 && warp < kSoftWarp0 + kSoftWarps) {
+    const int mt = (warp - kSoftWarp0) >> 2, quad = warp & 3;
+    const int rho = quad * 32 + lane;                  // row within the M tile (TMEM lane)
+    const int r = mt * 128 + rho;                      // window row within the group
+    const bool wactive = mt < p.n_mtiles && mt * 128 + quad * 32 < p.rows;
+    const bool live = r < p.rows;
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    const uint32_t s_col0 = 256 + mt * kAttnUnitKeys, o_col = mt * kHeadDim;
+    const float c2 = p.scale2;
+    float m = -INFINITY, l = 0.f;
+    int fills0 = 0, fills1 = 0;   // fills of P buffers 0 and 1 so far
+    int64_t ui = 0;
+    UnitIter c;
+    for (c.init(p, fb, fe); c.valid(); c.next(p), ++ui) {
+      if (ctl->abort) break;
+      const bool first = c.first(fb), last = c.last();
+      const int t = static_cast<int>(ui & 1), b = t;
+      if (!__all_sync(kFull, mbar_wait(&ctl->s_full[t], static_cast<uint32_t>((ui >> 1) & 1), p.wait_ns))) {
+        fail(ctl, p.err);
+        break;
+      }
+      tc_fence_after();
+      uint32_t z[4][16];
+      if (wactive) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) tmem_ld16_async(lane_base + s_col0 + t * 128 + q * 16, z[q]);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) tmem_wait16(z[q]);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl->s_empty[t]);
+      const int lim = p.seq[c.s].Lp - c.j * kAttnUnitKeys;   // valid keys of the unit (>= 1)
+      float mx = 0.f;   // a warp without rows keeps a finite reference
+      if (wactive) {
+        mx = -INFINITY;
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+#pragma unroll
+          for (int i = 0; i < 16; ++i)
+            if (q * 16 + i < lim) mx = fmaxf(mx, __uint_as_float(z[q][i]));
+        mx *= c2;
+      }
+      float alpha = 1.f;
+      bool move = false;
+      if (first) {
+        m = mx;
+        l = 0.f;
+      } else if (mx > m + kMoveThreshold) {
+        move = true;
+        alpha = ex2_approx(m - mx);
+        m = mx;
+      }
+      if (wactive && __any_sync(kFull, move && live)) {
+        // the previous unit's P V must be done before this warp's O rows move
+        const int bp = b ^ 1;
+        if (!mbar_wait(&ctl->p_empty[bp], static_cast<uint32_t>(((bp ? fills1 : fills0) - 1) & 1), p.wait_ns)) {
+          fail(ctl, p.err);
+          break;
+        }
+        tc_fence_after();
+#pragma unroll 1
+        for (int ch = 0; ch < kHeadDim / 16; ++ch) {
+          uint32_t o[16];
+          tmem_ld16_async(lane_base + o_col + ch * 16, o);
+          tmem_wait16(o);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+          tmem_st16(lane_base + o_col + ch * 16, o);
+        }
+        tmem_wait_st();
+        tc_fence_before();
+      }
+      l *= alpha;
+      // P into buffer b once the product of its previous fill is done
+      const int nfill = b ? fills1 : fills0;   // earlier fills of buffer b
+      if (nfill > 0 &&
+          !__all_sync(kFull, mbar_wait(&ctl->p_empty[b], static_cast<uint32_t>((nfill - 1) & 1), p.wait_ns))) {
+        fail(ctl, p.err);
+        break;
+      }
+      if (wactive) {
+        const float2 sc2 = make_float2(c2, c2), nm2 = make_float2(-m, -m);
+        float2 acc = make_float2(0.f, 0.f);
+        uint8_t* prow = sP + (b * 2 + mt) * kPTileBytes + rho * 128;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          uint32_t h[8];
+#pragma unroll
+          for (int i = 0; i < 16; i += 2) {
+            const float2 e = ffma2(make_float2(__uint_as_float(z[q][i]), __uint_as_float(z[q][i + 1])), sc2, nm2);
+            const int k = q * 16 + i;
+            const float p0 = (live && k < lim) ? ex2_approx(e.x) : 0.f;
+            const float p1 = (live && k + 1 < lim) ? ex2_approx(e.y) : 0.f;
+            acc = fadd2(acc, make_float2(p0, p1));
+            h[i >> 1] = pack_half2(p0, p1);
+          }
+          // keys 16q .. 16q + 15 are 16-byte chunks 2q and 2q + 1 of the row
+          *reinterpret_cast<uint4*>(prow + (((2 * q) ^ (rho & 7)) * 16)) = make_uint4(h[0], h[1], h[2], h[3]);
+          *reinterpret_cast<uint4*>(prow + (((2 * q + 1) ^ (rho & 7)) * 16)) = make_uint4(h[4], h[5], h[6], h[7]);
+        }
+        l += acc.x + acc.y;
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl->p_full[b]);
+      if (b) ++fills1; else ++fills0;
+      if (last) {
+        // the piece's partial: (m, l) and the unnormalised O rows, once the
+        // product of this last unit (fill nfill of buffer b) is done
+        if (!__all_sync(kFull, mbar_wait(&ctl->p_empty[b], static_cast<uint32_t>(nfill & 1), p.wait_ns))) {
+          fail(ctl, p.err);
+          break;
+        }
+        tc_fence_after();
+        const int64_t slot = static_cast<int64_t>(c.row(p)) + blockIdx.x;
+        if (wactive) {
+          float* dst = p.part_o + (slot * kMaxRows + r) * kHeadDim;
+#pragma unroll 1
+          for (int ch = 0; ch < kHeadDim / 16; ++ch) {
+            uint32_t o[16];
+            tmem_ld16_async(lane_base + o_col + ch * 16, o);
+            tmem_wait16(o);
+            if (live)
+#pragma unroll
+              for (int i = 0; i < 16; i += 4)
+                *reinterpret_cast<float4*>(dst + ch * 16 + i) =
+                    make_float4(__uint_as_float(o[i]), __uint_as_float(o[i + 1]), __uint_as_float(o[i + 2]),
+                                __uint_as_float(o[i + 3]));
+          }
+          if (live) p.part_ml[slot * kMaxRows + r] = make_float2(m, l);
+        }
+        tc_fence_before();
+      }
+    }
+  } else if (warp >= kConvWarp0) {
+    // V of every unit to fp16 in place, then released to the P V product
+    const int ct = threadIdx.x - 32 * kConvWarp0;
+    int stage = 0, phase = 0;
+    for (int64_t f = fb; f < fe; ++f) {
+      if (ctl->abort) break;
+      if (!__all_sync(kFull, mbar_wait(&ctl->kv_full[stage], phase, p.wait_ns))) {
+        fail(ctl, p.err);
+        break;
+      }
+      uint4* v4 = reinterpret_cast<uint4*>(sKV + stage * kStageBytes + kUnitBytes);
+#pragma unroll
+      for (int i = 0; i < kUnitBytes / 16 / (32 * kConvWarps); ++i) {
+        uint4 x = v4[ct + i * 32 * kConvWarps];
+        x.x = bf16x2_to_f16x2(x.x);
+        x.y = bf16x2_to_f16x2(x.y);
+        x.z = bf16x2_to_f16x2(x.z);
+        x.w = bf16x2_to_f16x2(x.w);
+        v4[ct + i * 32 * kConvWarps] = x;
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&ctl->v_ready[stage]);
+      if (++stage == kStages) {
+        stage = 0;
+        phase ^= 1;
+      }
+    }
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// Merges the pieces of each (seq, layer, group) row: M = max m, L = sum
+// 2^(m - M) l, O = sum 2^(m - M) O_piece / L, lse = (M + log2 L) ln 2.
+// grid: (rows of the launch, ceil(window rows / 32)); one warp per window row
+// at a time, four output columns per lane.
+__global__ void __launch_bounds__(256) k_attn_combine(const __grid_constant__ AttnParams p) {
+  griddep_launch_dependents();
+  griddep_wait();
+  const int R = blockIdx.x;
+  const int per_seq = p.nlayers * p.G;
+  const int s = R / per_seq, rem = R - s * per_seq, l = rem / p.G, g = rem - l * p.G;
+  const AttnSeq& sq = p.seq[s];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t row0 = (static_cast<int64_t>(p.layer0 + l) * p.G + g) * p.rows;   // flat (h, i) row of r = 0
+  int c0 = 0, c1 = -1;
+  if (sq.nu > 0) {
+    const int64_t f0 = sq.unit_base + static_cast<int64_t>(l * p.G + g) * sq.nu;
+    c0 = cta_of(f0, p.total_units, p.grid);
+    c1 = cta_of(f0 + sq.nu - 1, p.total_units, p.grid);
+  }
+  for (int r = blockIdx.y * 32 + warp; r < min(p.rows, blockIdx.y * 32 + 32); r += 8) {
+    float M = -INFINITY;
+    for (int c = c0; c <= c1; ++c) M = fmaxf(M, p.part_ml[(static_cast<int64_t>(R) + c) * kMaxRows + r].x);
+    float L = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c = c0; c <= c1; ++c) {
+      const int64_t slot = static_cast<int64_t>(R) + c;
+      const float2 ml = p.part_ml[slot * kMaxRows + r];
+      const float wgt = exp2f(ml.x - M);
+      const float4 o = reinterpret_cast<const float4*>(p.part_o + (slot * kMaxRows + r) * kHeadDim)[lane];
+      L += wgt * ml.y;
+      acc.x += wgt * o.x;
+      acc.y += wgt * o.y;
+      acc.z += wgt * o.z;
+      acc.w += wgt * o.w;
+    }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    if (sq.o)
+      reinterpret_cast<float4*>(sq.o + (row0 + r) * kHeadDim)[lane] =
+          make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+    if (lane == 0) sq.lse[row0 + r] = L > 0.f ? (M + log2f(L)) * 0.6931471805599453f : -INFINITY;
+  }
+}
+
+size_t attn_smem_bytes(int q_rows) {
+  return 1024 + static_cast<size_t>(2 * q_rows * 128) + static_cast<size_t>(kStages) * kStageBytes +
+         4 * static_cast<size_t>(kPTileBytes) + 256;
+}
+
+cudaError_t attn_configure() {
+  return cudaFuncSetAttribute(k_window_attn, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              static_cast<int>(kSmemLimit));
+}
+
+namespace {
+
+cudaLaunchConfig_t pdl_config(cudaLaunchAttribute* attr, dim3 grid, dim3 block, size_t smem, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;   // set-up under the previous kernel's tail
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  cfg.stream = stream;
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  return cfg;
+}
+
+}  // namespace
+
+cudaError_t attn_main_launch(const AttnParams& p, cudaStream_t stream) {
+  if (p.total_units <= 0) return cudaSuccess;
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = pdl_config(attr, dim3(p.grid), dim3(kAttnThreads), attn_smem_bytes(p.q_rows), stream);
+  return cudaLaunchKernelEx(&cfg, k_window_attn, p);
+}
+
+cudaError_t attn_combine_launch(const AttnParams& p, cudaStream_t stream) {
+  cudaLaunchAttribute attr[1];
+  cudaLaunchConfig_t cfg = pdl_config(attr, dim3(p.nseq * p.nlayers * p.G, (p.rows + 31) / 32), dim3(256), 0, stream);
+  return cudaLaunchKernelEx(&cfg, k_attn_combine, p);
+}
+
+}  // namespace starkv

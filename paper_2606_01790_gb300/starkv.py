@@ -26,10 +26,10 @@ ABI_FUNCTIONS = [
     "starkv_compact", "starkv_step", "starkv_step_host", "starkv_check_device_error",
     "starkv_set_wait_limit", "starkv_set_timing", "starkv_kernel_times", "starkv_last_error",
     "starkv_score_layer_noalloc", "starkv_selftest_wait", "starkv_slot_state_bytes", "starkv_export_slot",
-    "starkv_import_slot",
+    "starkv_import_slot", "starkv_window_attention",
 ]
 
-KERNELS = ["score_lse", "score_accum", "pool", "calibrate", "compact"]
+KERNELS = ["score_lse", "score_accum", "pool", "calibrate", "compact", "attention", "attn_combine"]
 
 
 SELECT_GLOBAL, SELECT_PER_HEAD = 0, 1   # starkv_config.select_mode
@@ -56,7 +56,8 @@ class CSeq(C.Structure):
                 ("budget", C.c_int32), ("slot", C.c_int32), ("k_out", C.c_void_p),
                 ("v_out", C.c_void_p), ("meta_out", C.c_void_p), ("idx", C.c_void_p),
                 ("S", C.c_void_p), ("score", C.c_void_p), ("stats", C.c_void_p),
-                ("meta_group_stride", C.c_int64), ("lse", C.c_void_p)]
+                ("meta_group_stride", C.c_int64), ("lse", C.c_void_p), ("attn_o", C.c_void_p),
+                ("attn_lse", C.c_void_p)]
 
 
 _lib: Optional[C.CDLL] = None
@@ -88,7 +89,7 @@ def lib() -> C.CDLL:
         for name in ("starkv_score_layer", "starkv_select", "starkv_compact"):
             getattr(L, name).argtypes = [st, C.c_int32, C.POINTER(CSeq), C.c_int32, C.c_void_p,
                                          C.c_size_t, C.c_void_p]
-        for name in ("starkv_step", "starkv_step_host"):
+        for name in ("starkv_step", "starkv_step_host", "starkv_window_attention"):
             getattr(L, name).argtypes = [st, C.POINTER(CSeq), C.c_int32, C.c_void_p, C.c_size_t,
                                          C.c_void_p]
         L.starkv_score_layer_noalloc.argtypes = [st, C.c_int32, C.POINTER(CSeq), C.c_int32, C.c_void_p]
@@ -230,10 +231,13 @@ class Seq:
     stats: Optional[torch.Tensor] = None
     meta_group_stride: int = 0              # per-KV-head mode: one metadata row per group
     lse: Optional[torch.Tensor] = None      # f32 [n_layers][H][w] supplied row normalisers
+    attn_o: Optional[torch.Tensor] = None   # f32 [n_layers][H][w][d] window_attention output
+    attn_lse: Optional[torch.Tensor] = None  # f32 [n_layers][H][w] window_attention normalisers
 
     def to_c(self) -> CSeq:
         s = CSeq()
-        for name in ("k", "v", "q", "meta", "k_out", "v_out", "meta_out", "idx", "S", "score", "stats", "lse"):
+        for name in ("k", "v", "q", "meta", "k_out", "v_out", "meta_out", "idx", "S", "score", "stats", "lse",
+                     "attn_o", "attn_lse"):
             setattr(s, name, _ptr(getattr(self, name)))
         s.meta_layer_stride = self.meta_layer_stride
         s.meta_group_stride = self.meta_group_stride
@@ -362,6 +366,14 @@ def compact(st: State, layer: int, seqs: Sequence[Seq], ws: torch.Tensor, stream
 def step(st: State, seqs: Sequence[Seq], ws: torch.Tensor, stream=None) -> None:
     arr = _seq_array(seqs)
     _check(lib().starkv_step(st.handle, arr, len(seqs), ws.data_ptr(), ws.numel(), _stream(stream)))
+
+
+def window_attention(st: State, seqs: Sequence[Seq], ws: torch.Tensor, stream=None) -> None:
+    """Attention output (``attn_o``, optional) and normaliser (``attn_lse``) of
+    the window rows over the past keys, for every layer of every sequence."""
+    arr = _seq_array(seqs)
+    _check(lib().starkv_window_attention(st.handle, arr, len(seqs), ws.data_ptr(), ws.numel(),
+                                         _stream(stream)))
 
 
 def step_host(st: State, seqs: Sequence[Seq], ws: torch.Tensor, stream=None) -> None:

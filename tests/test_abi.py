@@ -50,7 +50,7 @@ def test_header_constants_match_binding():
     assert m and all(sk.stats_stride(g) == 8 + int(m.group(1)) * g for g in range(1, 9))
     m = re.search(r"STARKV_SELECT_GLOBAL = (\d+), STARKV_SELECT_PER_HEAD = (\d+)", text)
     assert m and (int(m.group(1)), int(m.group(2))) == (sk.SELECT_GLOBAL, sk.SELECT_PER_HEAD)
-    assert ctypes.sizeof(sk.CSeq) == 4 * 8 + 8 + 4 * 4 + 7 * 8 + 8 + 8
+    assert ctypes.sizeof(sk.CSeq) == 4 * 8 + 8 + 4 * 4 + 7 * 8 + 8 + 8 + 2 * 8
 
 
 def test_default_config_matches_paper_defaults(library):
