@@ -66,6 +66,21 @@ def work_per_step(wl, seqs, per_head=False):
                 step_bytes=k_bytes + s_bytes + gather)
 
 
+def with_attention(wl, work, n_seqs):
+    """The step's work when it also runs the window-attention producer (the
+    model's own attention of the window rows, whose normaliser the compression
+    then takes): V read once (G * d * 2 B per scored token and layer) and the
+    output written (H * w * d fp32 per layer and sequence) on top of K and Q,
+    and the P V flops (as many as Q K^T) on top of Q K^T."""
+    v_bytes = wl.n_kv_heads * wl.head_dim * 2.0 * work["tokens"]
+    o_bytes = wl.n_heads * wl.window * wl.head_dim * 4.0 * wl.n_layers * n_seqs
+    out = dict(work)
+    out["attn_bytes"] = work["k_bytes"] + v_bytes + o_bytes
+    out["step_bytes"] = work["step_bytes"] + v_bytes + o_bytes
+    out["step_flops"] = 2 * work["qk_flops"]
+    return out
+
+
 def kernel_work(kind, work, peaks):
     """(bound, algorithmic units per step, unit) of one kernel kind.  A scoring
     pass reads K once and does the Q K^T flops; its bound is whichever of the
@@ -79,6 +94,8 @@ def kernel_work(kind, work, peaks):
         return "tensor", work["qk_flops"] / 1e12, "TFLOP/s"
     if kind == "compact":
         return "hbm", work["gather_bytes"] / 1e9, "GB/s"
+    if kind == "attention":
+        return "hbm", work["attn_bytes"] / 1e9, "GB/s"
     return "hbm", work["s_bytes"] / 1e9, "GB/s"
 
 
@@ -111,7 +128,8 @@ def kernel_src_hash(kind, read=None):
     """Hash of the code (comments excluded) that a kernel is built from;
     ``read(name)`` returns a source file's text (default: the working tree)."""
     files = {"score_lse": "score.cu", "score_accum": "score.cu", "pool": "score.cu",
-             "calibrate": "select.cu", "compact": "compact.cu"}[kind]
+             "calibrate": "select.cu", "compact": "compact.cu", "attention": "attn.cu",
+             "attn_combine": "attn.cu"}[kind]
     read = read or (lambda f: (ROOT / "paper_2606_01790_gb300" / "csrc" / f).read_text())
     h = hashlib.sha256()
     for f in (files, "ptx.cuh", "common.cuh"):
@@ -329,24 +347,6 @@ def job_throughput(tokens_per_rank_step, world, steps, ms_max):
 
 # ----------------------------------------------------------------------------- GPU arm
 
-def window_lse_torch(si, wl, dev):
-    """[n_layers][H][w] natural-log log-sum-exp of each window row over the
-    past keys, in fp32 with torch (input preparation for --lse given)."""
-    import math
-    import torch
-    nl, H, G, w = si.k.shape[0], wl.n_heads, wl.n_kv_heads, wl.window
-    lp = si.L - w
-    out = torch.empty((nl, H, w), dtype=torch.float32, device=dev)
-    for l in range(nl):
-        q = si.q[l].to(dev).float()                      # [H][w][d]
-        k = si.k[l, :, :lp].to(dev).float()              # [G][lp][d]
-        for g in range(G):
-            hs = slice(g * (H // G), (g + 1) * (H // G))
-            z = torch.einsum("hid,td->hit", q[hs], k[g]) / math.sqrt(wl.head_dim)
-            out[l, hs] = torch.logsumexp(z, dim=-1)
-    return out
-
-
 class GpuBench:
     """Device set-up, inputs and the timed loops of the GPU arm."""
 
@@ -368,6 +368,19 @@ class GpuBench:
         __graft_entry__.build()
         self.wl = syn.WORKLOADS[args.workload]
         self.peaks = _peaks()
+        self.step_fn = sk.step
+
+    def use_attention(self):
+        """Every step first runs the window-attention producer, whose
+        normalisers the compression step then takes (its first scoring pass
+        skipped): the model's attention of the window rows plus the
+        compression, as App. A.3 accounts them."""
+        sk = self.sk
+
+        def step(st, seqs, ws):
+            sk.window_attention(st, seqs, ws)
+            sk.step(st, seqs, ws)
+        self.step_fn = step
 
     def config(self, n_seqs):
         sk, wl = self.sk, self.wl
@@ -414,13 +427,13 @@ class GpuBench:
         launches made in the timed region."""
         torch, sk = self.torch, self.sk
         for _ in range(warmup):
-            sk.step(st, seqs, ws)
+            self.step_fn(st, seqs, ws)
         torch.cuda.synchronize(self.dev)
         sk.check_device_error(st)
         t_soak = time.time()
         while time.time() - t_soak < soak_s:
             for _ in range(10):
-                sk.step(st, seqs, ws)
+                self.step_fn(st, seqs, ws)
             torch.cuda.synchronize(self.dev)
         sk.kernel_times(st)   # reset counters
         self.barrier()
@@ -428,7 +441,7 @@ class GpuBench:
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for _ in range(steps):
-            sk.step(st, seqs, ws)
+            self.step_fn(st, seqs, ws)
         e1.record(stream)
         self.barrier()
         ms = e0.elapsed_time(e1)
@@ -443,7 +456,7 @@ class GpuBench:
         torch, sk = self.torch, self.sk
         sk.set_timing(st, True)
         for _ in range(n):
-            sk.step(st, seqs, ws)
+            self.step_fn(st, seqs, ws)
         torch.cuda.synchronize(self.dev)
         sk.set_timing(st, False)
         return sk.kernel_times(st)
@@ -478,6 +491,40 @@ class GpuBench:
         sk.check_device_error(st)
         return e_ms / n, h2d, d2h
 
+    def e2e_attention(self, st, sis, P, n, devseqs, ws):
+        """The end-to-end step with the attention producer: K, V, Q and the
+        metadata copied from page-locked host buffers, the producer and the
+        step on the device buffers, the compacted cache and indices copied
+        back, all in the timed region: (ms per step, h2d bytes, d2h bytes)."""
+        torch, sk = self.torch, self.sk
+        hseqs = [self.make_seq(si, i, P, pin=True) for i, si in enumerate(sis)]
+        names_in, names_out = ("k", "v", "q", "meta"), ("k_out", "v_out", "meta_out", "idx")
+        h2d = sum(getattr(h, a).numel() * getattr(h, a).element_size() for h in hseqs for a in names_in)
+        d2h = sum(getattr(h, a).numel() * getattr(h, a).element_size() for h in hseqs for a in names_out)
+
+        def one():
+            for h, d in zip(hseqs, devseqs):
+                for a in names_in:
+                    getattr(d, a).copy_(getattr(h, a), non_blocking=True)
+            sk.window_attention(st, devseqs, ws)
+            sk.step(st, devseqs, ws)
+            for h, d in zip(hseqs, devseqs):
+                for a in names_out:
+                    getattr(h, a).copy_(getattr(d, a), non_blocking=True)
+        for _ in range(2):
+            one()
+        self.barrier()
+        stream = torch.cuda.current_stream(self.dev)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(n):
+            one()
+        b.record(stream)
+        self.barrier()
+        e_ms = max_over_ranks(a.elapsed_time(b), self.dist, self.dev)
+        sk.check_device_error(st)
+        return e_ms / n, h2d, d2h
+
     def roofline(self, kt, work, n_kt, workload):
         """The dominant kernel's achieved rate against its binding peak, and its
         share of the per-kernel pass."""
@@ -498,10 +545,10 @@ class GpuBench:
         return roof, kernels
 
     def step_roofline(self, work, ms_step):
-        us = max(work["step_bytes"] / (self.peaks["hbm"] * 1e9),
-                 work["qk_flops"] / (self.peaks["tc"] * 1e12)) * 1e6
+        flops = work.get("step_flops", work["qk_flops"])
+        us = max(work["step_bytes"] / (self.peaks["hbm"] * 1e9), flops / (self.peaks["tc"] * 1e12)) * 1e6
         return {"roofline_us": us, "measured_us": 1e3 * ms_step, "frac": us / (1e3 * ms_step),
-                "alg_bytes": work["step_bytes"], "alg_flops": work["qk_flops"], "peak_src": self.peaks["src"]}
+                "alg_bytes": work["step_bytes"], "alg_flops": flops, "peak_src": self.peaks["src"]}
 
 
 def gpu_arm(args):
@@ -514,13 +561,19 @@ def gpu_arm(args):
     st = sk.init_state(gb.config(len(sis)))
     P = sk.sel_rows(st.cfg)   # rows of idx / meta_out per layer
     seqs = [gb.make_seq(si, i, P) for i, si in enumerate(sis)]
-    if args.lse == "given":
-        # the softmax normaliser of each window row over the past keys, as the
-        # layer's prefill attention pass supplies it (input preparation, torch)
-        for s_, si in zip(seqs, sis):
-            s_.lse = window_lse_torch(si, wl, gb.dev)
-    ws = sk.workspace(st, seqs, device=gb.dev)
     work = work_per_step(wl, [dict(L=si.L, B=si.budget) for si in sis], per_head=P > 1)
+    if args.lse == "given":
+        # every step runs the window-attention producer (the model's own
+        # attention of the window rows, output and normalisers), and the
+        # compression takes its normalisers
+        for s_ in seqs:
+            s_.attn_o = torch.empty((wl.n_layers, wl.n_heads, wl.window, wl.head_dim), dtype=torch.float32,
+                                    device=gb.dev)
+            s_.attn_lse = torch.empty((wl.n_layers, wl.n_heads, wl.window), dtype=torch.float32, device=gb.dev)
+            s_.lse = s_.attn_lse
+        gb.use_attention()
+        work = with_attention(wl, work, len(seqs))
+    ws = sk.workspace(st, seqs, device=gb.dev)
 
     clocks = ClockSampler(gb.local)
     t0 = time.time()
@@ -537,7 +590,10 @@ def gpu_arm(args):
     e2e = None
     if not args.no_e2e:
         n_e2e = max(1, min(args.steps, 20))
-        e_ms, h2d, d2h = gb.e2e(st, sis, P, n_e2e, seqs)
+        if args.lse == "given":
+            e_ms, h2d, d2h = gb.e2e_attention(st, sis, P, n_e2e, seqs, ws)
+        else:
+            e_ms, h2d, d2h = gb.e2e(st, sis, P, n_e2e, seqs)
         e2e = {"value": job_throughput(work["tokens"], gb.world, 1, e_ms), "unit": UNIT,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "steps": n_e2e, "ms_per_step": e_ms}
 
@@ -551,8 +607,9 @@ def gpu_arm(args):
             "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": args.workload, "select_mode": args.select_mode,
-                       "lse": "supplied (prefill attention); first scoring pass skipped" if args.lse == "given"
-                       else "computed (both scoring passes)", "layers": wl.n_layers, "seqs_per_gpu": len(sis),
+                       "lse": "from the window-attention producer run in every step (the model's attention "
+                              "of the window rows: output and normalisers); first scoring pass skipped"
+                       if args.lse == "given" else "computed (both scoring passes)", "layers": wl.n_layers, "seqs_per_gpu": len(sis),
                        "L": [si.L for si in sis], "w": wl.window, "B": [si.budget for si in sis],
                        "budget_pct": args.budget_pct or None, "H": wl.n_heads, "G": wl.n_kv_heads,
                        "d": wl.head_dim,
@@ -674,8 +731,9 @@ def main():
     ap.add_argument("--select-mode", choices=["global", "per_head"], default="global",
                     help="global top-B per layer (the paper's) or one top-B per KV group")
     ap.add_argument("--lse", choices=["computed", "given"], default="computed",
-                    help="given: the window rows' softmax normalisers are inputs (from the prefill "
-                         "attention pass), so the first scoring pass is skipped")
+                    help="given: every step first runs the window-attention producer (the model's "
+                         "attention of the window rows) and the compression takes its normalisers, "
+                         "so the first scoring pass is skipped")
     ap.add_argument("--budget-pct", type=int, default=0,
                     help="budget as this percentage of the visual tokens (0: the workload's own)")
     ap.add_argument("--trajectory", action="store_true",

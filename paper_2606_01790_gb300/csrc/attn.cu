@@ -29,9 +29,10 @@
 // The row reference m is the first unit's maximum and moves only when a
 // unit's maximum exceeds it by more than 15 (fp16 holds P < 2^16); the move
 // rescales that row's O in TMEM after the previous unit's P V is done (rare).
-// Warp roles: warp 0 TMA producer (K and V through a three-stage ring, Q per
-// piece), warp 1 MMA issuer and TMEM owner, warps 4..11 softmax (warpgroup =
-// M tile), warps 12..15 V conversion.
+// Warp roles: warp 0 loads K (a three-stage ring, each stage free once S of
+// its unit is done) and Q per piece, warp 3 loads V (a three-stage ring, free
+// once the P V product is done), warp 1 issues S and owns TMEM, warp 2 issues
+// P V, warps 4..11 softmax (warpgroup = M tile), warps 12..15 V conversion.
 #include <algorithm>
 #include <utility>
 
@@ -45,10 +46,9 @@ namespace starkv {
 
 namespace {
 
-constexpr int kStages = 3;                        // K/V ring depth
+constexpr int kStages = 3;                        // depth of the K ring and of the V ring
 constexpr int kUnitBytes = kAttnUnitKeys * 256;   // 64 keys x 128 bf16: 16 KB (K or V)
 constexpr int kHalfBytes = kAttnUnitKeys * 128;   // one 64-column half of a unit: 8 KB
-constexpr int kStageBytes = 2 * kUnitBytes;       // K then V
 constexpr int kPTileBytes = 128 * 128;            // one M tile of P: 128 rows x 64 fp16
 constexpr int kTmemCols = 512;                    // O [0, 256), S stage t at 256 + 128 t
 constexpr int kSoftWarp0 = 4, kSoftWarps = 8;
@@ -63,7 +63,8 @@ __device__ __forceinline__ uint64_t drain_limit(uint64_t wait_ns) {
 }
 
 struct AttnCtl {
-  uint64_t kv_full[kStages], kv_empty[kStages], v_ready[kStages];
+  uint64_t k_full[kStages], k_empty[kStages];
+  uint64_t v_full[kStages], v_empty[kStages], v_ready[kStages];
   uint64_t s_full[2], s_empty[2];
   uint64_t p_full[2], p_empty[2];
   uint64_t q_full, q_empty, drain;
@@ -177,8 +178,9 @@ __host__ __device__ __forceinline__ int cta_of(int64_t f, int64_t T, int P) {
   return static_cast<int>(((f + 1) * P - 1) / T);
 }
 
-__device__ void producer_loop(const AttnParams& p, AttnCtl* ctl, uint8_t* sQ, uint8_t* sKV, int64_t fb,
-                              int64_t fe) {
+// K (and Q per piece) loader: a K stage is free once S of its unit is done,
+// so K runs ahead of the products.
+__device__ void k_loader(const AttnParams& p, AttnCtl* ctl, uint8_t* sQ, uint8_t* sK, int64_t fb, int64_t fe) {
   const uint64_t pol = policy_evict_first();   // K and V stream through L2 once
   const int qhalf = p.q_rows * 128;
   int stage = 0, phase = 0, pc = 0, last_q_pc = -1;
@@ -198,14 +200,11 @@ __device__ void producer_loop(const AttnParams& p, AttnCtl* ctl, uint8_t* sQ, ui
       last_q_pc = pc;
       ++pc;
     }
-    if (!mbar_wait(&ctl->kv_empty[stage], phase ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
-    mbar_arrive_expect_tx(&ctl->kv_full[stage], kStageBytes);
+    if (!mbar_wait(&ctl->k_empty[stage], phase ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
+    mbar_arrive_expect_tx(&ctl->k_full[stage], kUnitBytes);
     const int zk = (p.layer0 + c.l) * p.G + c.g, y = c.j * kAttnUnitKeys;
-    uint8_t* st = sKV + stage * kStageBytes;
-    for (int h = 0; h < 2; ++h) {
-      tma_load_3d_hint(st + h * kHalfBytes, &p.tmk[c.s], &ctl->kv_full[stage], h * 64, y, zk, pol);
-      tma_load_3d_hint(st + kUnitBytes + h * kHalfBytes, &p.tmv[c.s], &ctl->kv_full[stage], h * 64, y, zk, pol);
-    }
+    for (int h = 0; h < 2; ++h)
+      tma_load_3d_hint(sK + stage * kUnitBytes + h * kHalfBytes, &p.tmk[c.s], &ctl->k_full[stage], h * 64, y, zk, pol);
     last_ph[stage] = phase;
     if (++stage == kStages) {
       stage = 0;
@@ -214,56 +213,59 @@ __device__ void producer_loop(const AttnParams& p, AttnCtl* ctl, uint8_t* sQ, ui
   }
   if (ctl->abort) {   // every issued copy completes before the CTA can exit
     for (int i = 0; i < kStages; ++i)
-      if (last_ph[i] >= 0) mbar_wait(&ctl->kv_full[i], last_ph[i], drain_limit(p.wait_ns));
+      if (last_ph[i] >= 0) mbar_wait(&ctl->k_full[i], last_ph[i], drain_limit(p.wait_ns));
     if (last_q_pc >= 0) mbar_wait(&ctl->q_full, last_q_pc & 1, drain_limit(p.wait_ns));
   }
 }
 
-// Single MMA issuer: S(u) into S stage u & 1, then O += P(u - 1) V(u - 1)
-// once the softmax has written P(u - 1), so that the product of one unit runs
-// while the softmax of the next is computed.
-__device__ void mma_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sQ, const uint8_t* sKV,
-                         const uint8_t* sP, uint32_t tmem, int64_t fb, int64_t fe) {
+// V loader: a V stage is free once the P V product of its unit is done.
+__device__ void v_loader(const AttnParams& p, AttnCtl* ctl, uint8_t* sV, int64_t fb, int64_t fe) {
+  const uint64_t pol = policy_evict_first();
+  int stage = 0, phase = 0;
+  int last_ph[kStages];
+  for (int i = 0; i < kStages; ++i) last_ph[i] = -1;
+  UnitIter c;
+  for (c.init(p, fb, fe); c.valid(); c.next(p)) {
+    if (ctl->abort) break;
+    if (!mbar_wait(&ctl->v_empty[stage], phase ^ 1, p.wait_ns)) { fail(ctl, p.err); break; }
+    mbar_arrive_expect_tx(&ctl->v_full[stage], kUnitBytes);
+    const int zk = (p.layer0 + c.l) * p.G + c.g, y = c.j * kAttnUnitKeys;
+    for (int h = 0; h < 2; ++h)
+      tma_load_3d_hint(sV + stage * kUnitBytes + h * kHalfBytes, &p.tmv[c.s], &ctl->v_full[stage], h * 64, y, zk, pol);
+    last_ph[stage] = phase;
+    if (++stage == kStages) {
+      stage = 0;
+      phase ^= 1;
+    }
+  }
+  if (ctl->abort)
+    for (int i = 0; i < kStages; ++i)
+      if (last_ph[i] >= 0) mbar_wait(&ctl->v_full[i], last_ph[i], drain_limit(p.wait_ns));
+}
+
+// Two MMA issuers walk the same units: warp 1 issues S(u) into S stage u & 1
+// as soon as the stage is free and K(u) has landed, warp 2 issues
+// O += P(u) V(u) once the softmax has written P(u) and V(u) is fp16, so that
+// S of the next units runs ahead of the products.
+__device__ void mma_s_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sQ, const uint8_t* sK, uint32_t tmem,
+                           int64_t fb, int64_t fe) {
   const uint32_t idesc_s = idesc_bf16(128, kAttnUnitKeys);
-  const uint32_t idesc_o = idesc_f16_bmn(128, kHeadDim);
   const uint64_t dq0 = sdesc_k_sw128(smem_u32(sQ));
   const uint32_t qhalf16 = (p.q_rows * 128) >> 4;
   int stage = 0, kphase = 0, pc = 0;
-  bool pend = false, pend_first = false;
-  int pend_stage = 0, pend_vph = 0;
   int64_t ui = 0;
-  auto issue_pv = [&](int st, int vph, int64_t u, bool first_of_piece) -> bool {
-    const int b = static_cast<int>(u & 1);
-    if (!mbar_wait(&ctl->v_ready[st], vph, p.wait_ns)) return false;
-    if (!mbar_wait(&ctl->p_full[b], static_cast<uint32_t>((u >> 1) & 1), p.wait_ns)) return false;
-    tc_fence_after();
-    const uint64_t dv = sdesc_mn_sw128(smem_u32(sKV + st * kStageBytes + kUnitBytes), kHalfBytes, 1024);
-#pragma unroll
-    for (int mt = 0; mt < 2; ++mt) {
-      if (mt >= p.n_mtiles) break;
-      const uint64_t dp = sdesc_k_sw128(smem_u32(sP + (b * 2 + mt) * kPTileBytes));
-#pragma unroll
-      for (int kk = 0; kk < 4; ++kk)   // 16 keys per step: +32 B along the P row, +16 rows of V
-        mma_f16(tmem + mt * kHeadDim, dp + static_cast<uint64_t>(kk * 2), dv + static_cast<uint64_t>(kk * 128),
-                idesc_o, (!first_of_piece || kk > 0) ? 1u : 0u);
-    }
-    mma_commit(&ctl->kv_empty[st]);
-    mma_commit(&ctl->p_empty[b]);
-    return true;
-  };
   UnitIter c;
   for (c.init(p, fb, fe); c.valid(); c.next(p), ++ui) {
     if (ctl->abort) break;
-    const bool first = c.first(fb);
-    if (first) {
+    if (c.first(fb)) {
       if (!mbar_wait(&ctl->q_full, pc & 1, p.wait_ns)) { fail(ctl, p.err); break; }
       ++pc;
     }
     const int t = static_cast<int>(ui & 1);
-    if (!mbar_wait(&ctl->kv_full[stage], kphase, p.wait_ns)) { fail(ctl, p.err); break; }
+    if (!mbar_wait(&ctl->k_full[stage], kphase, p.wait_ns)) { fail(ctl, p.err); break; }
     if (!mbar_wait(&ctl->s_empty[t], static_cast<uint32_t>(((ui >> 1) & 1) ^ 1), p.wait_ns)) { fail(ctl, p.err); break; }
     tc_fence_after();
-    const uint64_t dk = sdesc_k_sw128(smem_u32(sKV + stage * kStageBytes));
+    const uint64_t dk = sdesc_k_sw128(smem_u32(sK + stage * kUnitBytes));
 #pragma unroll
     for (int mt = 0; mt < 2; ++mt) {
       if (mt >= p.n_mtiles) break;
@@ -278,19 +280,48 @@ __device__ void mma_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sQ, c
       }
     }
     mma_commit(&ctl->s_full[t]);
+    mma_commit(&ctl->k_empty[stage]);
     if (c.last()) mma_commit(&ctl->q_empty);
-    if (pend && !issue_pv(pend_stage, pend_vph, ui - 1, pend_first)) { fail(ctl, p.err); pend = false; break; }
-    pend = true;
-    pend_first = first;
-    pend_stage = stage;
-    pend_vph = kphase;
     if (++stage == kStages) {
       stage = 0;
       kphase ^= 1;
     }
   }
-  if (pend && !ctl->abort && !issue_pv(pend_stage, pend_vph, ui - 1, pend_first)) fail(ctl, p.err);
   // every MMA issued above must be complete before TMEM is released
+  mma_commit(&ctl->drain);
+  mbar_wait(&ctl->drain, 0, drain_limit(p.wait_ns));
+}
+
+__device__ void mma_pv_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sV, const uint8_t* sP, uint32_t tmem,
+                            int64_t fb, int64_t fe) {
+  const uint32_t idesc_o = idesc_f16_bmn(128, kHeadDim);
+  int stage = 0, kphase = 0;
+  int64_t ui = 0;
+  UnitIter c;
+  for (c.init(p, fb, fe); c.valid(); c.next(p), ++ui) {
+    if (ctl->abort) break;
+    const int b = static_cast<int>(ui & 1);
+    if (!mbar_wait(&ctl->v_ready[stage], kphase, p.wait_ns)) { fail(ctl, p.err); break; }
+    if (!mbar_wait(&ctl->p_full[b], static_cast<uint32_t>((ui >> 1) & 1), p.wait_ns)) { fail(ctl, p.err); break; }
+    tc_fence_after();
+    const bool first = c.first(fb);   // the piece's first product overwrites O
+    const uint64_t dv = sdesc_mn_sw128(smem_u32(sV + stage * kUnitBytes), kHalfBytes, 1024);
+#pragma unroll
+    for (int mt = 0; mt < 2; ++mt) {
+      if (mt >= p.n_mtiles) break;
+      const uint64_t dp = sdesc_k_sw128(smem_u32(sP + (b * 2 + mt) * kPTileBytes));
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)   // 16 keys per step: +32 B along the P row, +16 rows of V
+        mma_f16(tmem + mt * kHeadDim, dp + static_cast<uint64_t>(kk * 2), dv + static_cast<uint64_t>(kk * 128),
+                idesc_o, (!first || kk > 0) ? 1u : 0u);
+    }
+    mma_commit(&ctl->v_empty[stage]);
+    mma_commit(&ctl->p_empty[b]);
+    if (++stage == kStages) {
+      stage = 0;
+      kphase ^= 1;
+    }
+  }
   mma_commit(&ctl->drain);
   mbar_wait(&ctl->drain, 0, drain_limit(p.wait_ns));
 }
@@ -301,15 +332,18 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;                              // [2 halves][q_rows][128 B]
-  uint8_t* sKV = sQ + 2 * p.q_rows * 128;          // [kStages][K 16 KB | V 16 KB]
-  uint8_t* sP = sKV + kStages * kStageBytes;       // [2 buffers][2 M tiles][128 rows][128 B]
+  uint8_t* sK = sQ + 2 * p.q_rows * 128;           // [kStages][2 halves][64 keys][128 B]
+  uint8_t* sV = sK + kStages * kUnitBytes;         // [kStages][2 halves][64 keys][128 B]
+  uint8_t* sP = sV + kStages * kUnitBytes;         // [2 buffers][2 M tiles][128 rows][128 B]
   AttnCtl* ctl = reinterpret_cast<AttnCtl*>(sP + 4 * kPTileBytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < kStages; ++i) {
-      mbar_init(&ctl->kv_full[i], 1);
-      mbar_init(&ctl->kv_empty[i], 1);
+      mbar_init(&ctl->k_full[i], 1);
+      mbar_init(&ctl->k_empty[i], 1);
+      mbar_init(&ctl->v_full[i], 1);
+      mbar_init(&ctl->v_empty[i], 1);
       mbar_init(&ctl->v_ready[i], kConvWarps);
     }
     for (int i = 0; i < 2; ++i) {
@@ -320,7 +354,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
     }
     mbar_init(&ctl->q_full, 1);
     mbar_init(&ctl->q_empty, 1);
-    mbar_init(&ctl->drain, 1);
+    mbar_init(&ctl->drain, 2);   // one commit per MMA issuer
     ctl->abort = 0;
     fence_mbar_init();
   }
@@ -339,9 +373,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
   const int64_t fe = range_begin(T, blockIdx.x + 1, gridDim.x);
 
   if (warp == 0) {
-    if (lane == 0) producer_loop(p, ctl, sQ, sKV, fb, fe);
+    if (lane == 0) k_loader(p, ctl, sQ, sK, fb, fe);
+  } else if (warp == 3) {
+    if (lane == 0) v_loader(p, ctl, sV, fb, fe);
   } else if (warp == 1) {
-    if (lane == 0) mma_loop(p, ctl, sQ, sKV, sP, tmem, fb, fe);
+    if (lane == 0) mma_s_loop(p, ctl, sQ, sK, tmem, fb, fe);
+  } else if (warp == 2) {
+    if (lane == 0) mma_pv_loop(p, ctl, sV, sP, tmem, fb, fe);
   } else if (warp >= kSoftWarp0 && warp < kSoftWarp0 + kSoftWarps) {
     const int mt = (warp - kSoftWarp0) >> 2, quad = warp & 3;
     const int rho = quad * 32 + lane;                  // row within the M tile (TMEM lane)
@@ -483,11 +521,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
     int stage = 0, phase = 0;
     for (int64_t f = fb; f < fe; ++f) {
       if (ctl->abort) break;
-      if (!__all_sync(kFull, mbar_wait(&ctl->kv_full[stage], phase, p.wait_ns))) {
+      if (!__all_sync(kFull, mbar_wait(&ctl->v_full[stage], phase, p.wait_ns))) {
         fail(ctl, p.err);
         break;
       }
-      uint4* v4 = reinterpret_cast<uint4*>(sKV + stage * kStageBytes + kUnitBytes);
+      uint4* v4 = reinterpret_cast<uint4*>(sV + stage * kUnitBytes);
 #pragma unroll
       for (int i = 0; i < kUnitBytes / 16 / (32 * kConvWarps); ++i) {
         uint4 x = v4[ct + i * 32 * kConvWarps];
@@ -515,8 +553,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
 
 // Merges the pieces of each (seq, layer, group) row: M = max m, L = sum
 // 2^(m - M) l, O = sum 2^(m - M) O_piece / L, lse = (M + log2 L) ln 2.
-// grid: (rows of the launch, ceil(window rows / 32)); one warp per window row
-// at a time, four output columns per lane.
+// grid: (rows of the launch, ceil(window rows / 8)); one warp per window row,
+// four output columns per lane, every piece's loads issued before the sums.
+constexpr int kMaxPieces = 8;   // pieces merged per batch of loads
 __global__ void __launch_bounds__(256) k_attn_combine(const __grid_constant__ AttnParams p) {
   griddep_launch_dependents();
   griddep_wait();
@@ -525,6 +564,8 @@ __global__ void __launch_bounds__(256) k_attn_combine(const __grid_constant__ At
   const int s = R / per_seq, rem = R - s * per_seq, l = rem / p.G, g = rem - l * p.G;
   const AttnSeq& sq = p.seq[s];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.y * 8 + warp;
+  if (r >= p.rows) return;
   const int64_t row0 = (static_cast<int64_t>(p.layer0 + l) * p.G + g) * p.rows;   // flat (h, i) row of r = 0
   int c0 = 0, c1 = -1;
   if (sq.nu > 0) {
@@ -532,32 +573,49 @@ __global__ void __launch_bounds__(256) k_attn_combine(const __grid_constant__ At
     c0 = cta_of(f0, p.total_units, p.grid);
     c1 = cta_of(f0 + sq.nu - 1, p.total_units, p.grid);
   }
-  for (int r = blockIdx.y * 32 + warp; r < min(p.rows, blockIdx.y * 32 + 32); r += 8) {
-    float M = -INFINITY;
-    for (int c = c0; c <= c1; ++c) M = fmaxf(M, p.part_ml[(static_cast<int64_t>(R) + c) * kMaxRows + r].x);
-    float L = 0.f;
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int c = c0; c <= c1; ++c) {
-      const int64_t slot = static_cast<int64_t>(R) + c;
-      const float2 ml = p.part_ml[slot * kMaxRows + r];
-      const float wgt = exp2f(ml.x - M);
-      const float4 o = reinterpret_cast<const float4*>(p.part_o + (slot * kMaxRows + r) * kHeadDim)[lane];
-      L += wgt * ml.y;
-      acc.x += wgt * o.x;
-      acc.y += wgt * o.y;
-      acc.z += wgt * o.z;
-      acc.w += wgt * o.w;
+  float M = -INFINITY, L = 0.f;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int cb = c0; cb <= c1; cb += kMaxPieces) {
+    float2 ml[kMaxPieces];
+    float4 o[kMaxPieces];
+#pragma unroll
+    for (int k = 0; k < kMaxPieces; ++k) {
+      if (cb + k > c1) break;
+      const int64_t slot = static_cast<int64_t>(R) + cb + k;
+      ml[k] = p.part_ml[slot * kMaxRows + r];
+      o[k] = reinterpret_cast<const float4*>(p.part_o + (slot * kMaxRows + r) * kHeadDim)[lane];
     }
-    const float inv = L > 0.f ? 1.f / L : 0.f;
-    if (sq.o)
-      reinterpret_cast<float4*>(sq.o + (row0 + r) * kHeadDim)[lane] =
-          make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
-    if (lane == 0) sq.lse[row0 + r] = L > 0.f ? (M + log2f(L)) * 0.6931471805599453f : -INFINITY;
+    float bm = M;
+#pragma unroll
+    for (int k = 0; k < kMaxPieces; ++k)
+      if (cb + k <= c1) bm = fmaxf(bm, ml[k].x);
+    const float keep = M == -INFINITY ? 0.f : exp2f(M - bm);
+    L *= keep;
+    acc.x *= keep;
+    acc.y *= keep;
+    acc.z *= keep;
+    acc.w *= keep;
+#pragma unroll
+    for (int k = 0; k < kMaxPieces; ++k) {
+      if (cb + k > c1) break;
+      const float wgt = exp2f(ml[k].x - bm);
+      L += wgt * ml[k].y;
+      acc.x += wgt * o[k].x;
+      acc.y += wgt * o[k].y;
+      acc.z += wgt * o[k].z;
+      acc.w += wgt * o[k].w;
+    }
+    M = bm;
   }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  if (sq.o)
+    reinterpret_cast<float4*>(sq.o + (row0 + r) * kHeadDim)[lane] =
+        make_float4(acc.x * inv, acc.y * inv, acc.z * inv, acc.w * inv);
+  if (lane == 0) sq.lse[row0 + r] = L > 0.f ? (M + log2f(L)) * 0.6931471805599453f : -INFINITY;
 }
 
 size_t attn_smem_bytes(int q_rows) {
-  return 1024 + static_cast<size_t>(2 * q_rows * 128) + static_cast<size_t>(kStages) * kStageBytes +
+  return 1024 + static_cast<size_t>(2 * q_rows * 128) + 2 * static_cast<size_t>(kStages) * kUnitBytes +
          4 * static_cast<size_t>(kPTileBytes) + 256;
 }
 
@@ -592,7 +650,7 @@ cudaError_t attn_main_launch(const AttnParams& p, cudaStream_t stream) {
 
 cudaError_t attn_combine_launch(const AttnParams& p, cudaStream_t stream) {
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = pdl_config(attr, dim3(p.nseq * p.nlayers * p.G, (p.rows + 31) / 32), dim3(256), 0, stream);
+  cudaLaunchConfig_t cfg = pdl_config(attr, dim3(p.nseq * p.nlayers * p.G, (p.rows + 7) / 8), dim3(256), 0, stream);
   return cudaLaunchKernelEx(&cfg, k_attn_combine, p);
 }
 
