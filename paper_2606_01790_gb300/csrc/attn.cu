@@ -415,12 +415,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
       const int lim = p.seq[c.s].Lp - c.j * kAttnUnitKeys;   // valid keys of the unit (>= 1)
       float mx = 0.f;   // a warp without rows keeps a finite reference
       if (wactive) {
-        mx = -INFINITY;
+        // eight independent partial maxima (short dependency chains)
+        float pm[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) pm[k] = -INFINITY;
 #pragma unroll
         for (int q = 0; q < 4; ++q)
 #pragma unroll
           for (int i = 0; i < 16; ++i)
-            if (q * 16 + i < lim) mx = fmaxf(mx, __uint_as_float(z[q][i]));
+            if (q * 16 + i < lim) pm[i & 7] = fmaxf(pm[i & 7], __uint_as_float(z[q][i]));
+        mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])), fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
         mx *= c2;
       }
       float alpha = 1.f;
@@ -463,7 +467,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
       }
       if (wactive) {
         const float2 sc2 = make_float2(c2, c2), nm2 = make_float2(-m, -m);
-        float2 acc = make_float2(0.f, 0.f);
+        float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                         make_float2(0.f, 0.f)};   // four independent running sums
         uint8_t* prow = sP + (b * 2 + mt) * kPTileBytes + rho * 128;
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
@@ -474,14 +479,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
             const int k = q * 16 + i;
             const float p0 = (live && k < lim) ? ex2_approx(e.x) : 0.f;
             const float p1 = (live && k + 1 < lim) ? ex2_approx(e.y) : 0.f;
-            acc = fadd2(acc, make_float2(p0, p1));
+            acc[(i >> 1) & 3] = fadd2(acc[(i >> 1) & 3], make_float2(p0, p1));
             h[i >> 1] = pack_half2(p0, p1);
           }
           // keys 16q .. 16q + 15 are 16-byte chunks 2q and 2q + 1 of the row
           *reinterpret_cast<uint4*>(prow + (((2 * q) ^ (rho & 7)) * 16)) = make_uint4(h[0], h[1], h[2], h[3]);
           *reinterpret_cast<uint4*>(prow + (((2 * q + 1) ^ (rho & 7)) * 16)) = make_uint4(h[4], h[5], h[6], h[7]);
         }
-        l += acc.x + acc.y;
+        const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
+        const float2 a = fadd2(a01, a23);
+        l += a.x + a.y;
       }
       fence_proxy_async_smem();
       __syncwarp();
