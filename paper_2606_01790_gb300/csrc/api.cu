@@ -539,6 +539,7 @@ starkv_status run_attention(starkv_state* st, const starkv_seq* seqs, int nseq, 
     p.rows = (H / G) * w;
     p.n_mtiles = (p.rows + 127) / 128;
     p.q_rows = (p.rows + 15) & ~15;
+    p.kv_stages = attn_kv_stages(p.q_rows);
     p.scale2 = static_cast<float>(1.4426950408889634 / std::sqrt(static_cast<double>(kHeadDim)));
     int64_t units = 0;
     for (int i = i0; i < i1; ++i) {

@@ -20,19 +20,22 @@
 //                       (two S stages, so the MMA of unit u+1 runs under the
 //                       softmax of unit u);
 //   softmax             rows on TMEM lanes, one thread per row: p = exp2(S c - m),
-//                       l += p in fp32, P rounded to fp16 into shared memory
-//                       (128-byte swizzled K-major rows, two buffers);
-//   O += P V            M = 128, N = d = 128, K = 64 keys, fp16 -> fp32 in TMEM;
+//                       l += p in fp32, P rounded to fp16 and written over the
+//                       S columns it came from (two fp16 per 32-bit column);
+//   O += P V            M = 128, N = d = 128, K = 64 keys, fp16 -> fp32 in TMEM,
+//                       A = P read from tensor memory;
 //                       V arrives as bf16 and four warps convert it to fp16 in
 //                       place (exact for |v| < 65504), read as the transposed
 //                       (MN-major) operand.
 // The row reference m is the first unit's maximum and moves only when a
 // unit's maximum exceeds it by more than 15 (fp16 holds P < 2^16); the move
 // rescales that row's O in TMEM after the previous unit's P V is done (rare).
-// Warp roles: warp 0 loads K (a three-stage ring, each stage free once S of
-// its unit is done) and Q per piece, warp 3 loads V (a three-stage ring, free
-// once the P V product is done), warp 1 issues S and owns TMEM, warp 2 issues
-// P V, warps 4..11 softmax (warpgroup = M tile), warps 12..15 V conversion.
+// An S stage holds P until the P V product of its unit is done, which frees
+// it for S two units later.  Warp roles: warp 0 loads K (a four-stage ring,
+// each stage free once S of its unit is done) and Q per piece, warp 3 loads V
+// (a four-stage ring, free once the P V product is done), warp 1 issues S and
+// owns TMEM, warp 2 issues P V, warps 4..11 softmax (warpgroup = M tile),
+// warps 12..15 V conversion.
 #include <algorithm>
 #include <utility>
 
@@ -46,10 +49,9 @@ namespace starkv {
 
 namespace {
 
-constexpr int kStages = 3;                        // depth of the K ring and of the V ring
+constexpr int kStages = 4;                        // largest depth of the K ring and of the V ring
 constexpr int kUnitBytes = kAttnUnitKeys * 256;   // 64 keys x 128 bf16: 16 KB (K or V)
 constexpr int kHalfBytes = kAttnUnitKeys * 128;   // one 64-column half of a unit: 8 KB
-constexpr int kPTileBytes = 128 * 128;            // one M tile of P: 128 rows x 64 fp16
 constexpr int kTmemCols = 512;                    // O [0, 256), S stage t at 256 + 128 t
 constexpr int kSoftWarp0 = 4, kSoftWarps = 8;
 constexpr int kConvWarp0 = 12, kConvWarps = 4;
@@ -65,8 +67,8 @@ __device__ __forceinline__ uint64_t drain_limit(uint64_t wait_ns) {
 struct AttnCtl {
   uint64_t k_full[kStages], k_empty[kStages];
   uint64_t v_full[kStages], v_empty[kStages], v_ready[kStages];
-  uint64_t s_full[2], s_empty[2];
-  uint64_t p_full[2], p_empty[2];
+  uint64_t s_full[2], s_empty[2];   // s_empty: the stage's P V is done
+  uint64_t p_full[2];               // P of the stage written
   uint64_t q_full, q_empty, drain;
   uint32_t tmem_base;
   volatile int abort;
@@ -108,6 +110,26 @@ __device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_
       "setp.ne.b32 p, %4, 0;\n\t"
       "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
       "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// D[tmem] (+)= A[tmem] * B[smem]: A with M = 128 rows on TMEM lanes and its
+// K elements as fp16 pairs, lower index in the low half of each 32-bit column.
+__device__ __forceinline__ void mma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                           uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// 8 consecutive 32-bit columns of this warp's 32 TMEM lanes, stored.
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};\n" ::"r"(taddr),
+      "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
       : "memory");
 }
 
@@ -206,7 +228,7 @@ __device__ void k_loader(const AttnParams& p, AttnCtl* ctl, uint8_t* sQ, uint8_t
     for (int h = 0; h < 2; ++h)
       tma_load_3d_hint(sK + stage * kUnitBytes + h * kHalfBytes, &p.tmk[c.s], &ctl->k_full[stage], h * 64, y, zk, pol);
     last_ph[stage] = phase;
-    if (++stage == kStages) {
+    if (++stage == p.kv_stages) {
       stage = 0;
       phase ^= 1;
     }
@@ -233,7 +255,7 @@ __device__ void v_loader(const AttnParams& p, AttnCtl* ctl, uint8_t* sV, int64_t
     for (int h = 0; h < 2; ++h)
       tma_load_3d_hint(sV + stage * kUnitBytes + h * kHalfBytes, &p.tmv[c.s], &ctl->v_full[stage], h * 64, y, zk, pol);
     last_ph[stage] = phase;
-    if (++stage == kStages) {
+    if (++stage == p.kv_stages) {
       stage = 0;
       phase ^= 1;
     }
@@ -282,7 +304,7 @@ __device__ void mma_s_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sQ,
     mma_commit(&ctl->s_full[t]);
     mma_commit(&ctl->k_empty[stage]);
     if (c.last()) mma_commit(&ctl->q_empty);
-    if (++stage == kStages) {
+    if (++stage == p.kv_stages) {
       stage = 0;
       kphase ^= 1;
     }
@@ -292,32 +314,32 @@ __device__ void mma_s_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sQ,
   mbar_wait(&ctl->drain, 0, drain_limit(p.wait_ns));
 }
 
-__device__ void mma_pv_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sV, const uint8_t* sP, uint32_t tmem,
-                            int64_t fb, int64_t fe) {
+__device__ void mma_pv_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sV, uint32_t tmem, int64_t fb,
+                            int64_t fe) {
   const uint32_t idesc_o = idesc_f16_bmn(128, kHeadDim);
   int stage = 0, kphase = 0;
   int64_t ui = 0;
   UnitIter c;
   for (c.init(p, fb, fe); c.valid(); c.next(p), ++ui) {
     if (ctl->abort) break;
-    const int b = static_cast<int>(ui & 1);
+    const int t = static_cast<int>(ui & 1);
     if (!mbar_wait(&ctl->v_ready[stage], kphase, p.wait_ns)) { fail(ctl, p.err); break; }
-    if (!mbar_wait(&ctl->p_full[b], static_cast<uint32_t>((ui >> 1) & 1), p.wait_ns)) { fail(ctl, p.err); break; }
+    if (!mbar_wait(&ctl->p_full[t], static_cast<uint32_t>((ui >> 1) & 1), p.wait_ns)) { fail(ctl, p.err); break; }
     tc_fence_after();
     const bool first = c.first(fb);   // the piece's first product overwrites O
     const uint64_t dv = sdesc_mn_sw128(smem_u32(sV + stage * kUnitBytes), kHalfBytes, 1024);
 #pragma unroll
     for (int mt = 0; mt < 2; ++mt) {
       if (mt >= p.n_mtiles) break;
-      const uint64_t dp = sdesc_k_sw128(smem_u32(sP + (b * 2 + mt) * kPTileBytes));
+      const uint32_t ap = tmem + 256 + t * 128 + mt * kAttnUnitKeys;   // P of M tile mt over its S columns
 #pragma unroll
-      for (int kk = 0; kk < 4; ++kk)   // 16 keys per step: +32 B along the P row, +16 rows of V
-        mma_f16(tmem + mt * kHeadDim, dp + static_cast<uint64_t>(kk * 2), dv + static_cast<uint64_t>(kk * 128),
-                idesc_o, (!first || kk > 0) ? 1u : 0u);
+      for (int kk = 0; kk < 4; ++kk)   // 16 keys per step: +8 columns of P, +16 rows of V
+        mma_f16_ts(tmem + mt * kHeadDim, ap + kk * 8, dv + static_cast<uint64_t>(kk * 128), idesc_o,
+                   (!first || kk > 0) ? 1u : 0u);
     }
     mma_commit(&ctl->v_empty[stage]);
-    mma_commit(&ctl->p_empty[b]);
-    if (++stage == kStages) {
+    mma_commit(&ctl->s_empty[t]);   // S stage t (holding P) is free for S two units later
+    if (++stage == p.kv_stages) {
       stage = 0;
       kphase ^= 1;
     }
@@ -332,10 +354,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;                              // [2 halves][q_rows][128 B]
-  uint8_t* sK = sQ + 2 * p.q_rows * 128;           // [kStages][2 halves][64 keys][128 B]
-  uint8_t* sV = sK + kStages * kUnitBytes;         // [kStages][2 halves][64 keys][128 B]
-  uint8_t* sP = sV + kStages * kUnitBytes;         // [2 buffers][2 M tiles][128 rows][128 B]
-  AttnCtl* ctl = reinterpret_cast<AttnCtl*>(sP + 4 * kPTileBytes);
+  uint8_t* sK = sQ + 2 * p.q_rows * 128;           // [kv_stages][2 halves][64 keys][128 B]
+  uint8_t* sV = sK + p.kv_stages * kUnitBytes;     // [kv_stages][2 halves][64 keys][128 B]
+  AttnCtl* ctl = reinterpret_cast<AttnCtl*>(sV + p.kv_stages * kUnitBytes);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
@@ -348,9 +369,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&ctl->s_full[i], 1);
-      mbar_init(&ctl->s_empty[i], kSoftWarps);
+      mbar_init(&ctl->s_empty[i], 1);   // the P V issuer's commit
       mbar_init(&ctl->p_full[i], kSoftWarps);
-      mbar_init(&ctl->p_empty[i], 1);
     }
     mbar_init(&ctl->q_full, 1);
     mbar_init(&ctl->q_empty, 1);
@@ -379,7 +399,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
   } else if (warp == 1) {
     if (lane == 0) mma_s_loop(p, ctl, sQ, sK, tmem, fb, fe);
   } else if (warp == 2) {
-    if (lane == 0) mma_pv_loop(p, ctl, sV, sP, tmem, fb, fe);
+    if (lane == 0) mma_pv_loop(p, ctl, sV, tmem, fb, fe);
   } else if (warp >= kSoftWarp0 && warp < kSoftWarp0 + kSoftWarps) {
     const int mt = (warp - kSoftWarp0) >> 2, quad = warp & 3;
     const int rho = quad * 32 + lane;                  // row within the M tile (TMEM lane)
@@ -390,13 +410,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
     const uint32_t s_col0 = 256 + mt * kAttnUnitKeys, o_col = mt * kHeadDim;
     const float c2 = p.scale2;
     float m = -INFINITY, l = 0.f;
-    int fills0 = 0, fills1 = 0;   // fills of P buffers 0 and 1 so far
     int64_t ui = 0;
     UnitIter c;
     for (c.init(p, fb, fe); c.valid(); c.next(p), ++ui) {
       if (ctl->abort) break;
       const bool first = c.first(fb), last = c.last();
-      const int t = static_cast<int>(ui & 1), b = t;
+      const int t = static_cast<int>(ui & 1);
+      const uint32_t scol = s_col0 + t * 128;   // this unit's S, then P, columns
       if (!__all_sync(kFull, mbar_wait(&ctl->s_full[t], static_cast<uint32_t>((ui >> 1) & 1), p.wait_ns))) {
         fail(ctl, p.err);
         break;
@@ -405,13 +425,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
       uint32_t z[4][16];
       if (wactive) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q) tmem_ld16_async(lane_base + s_col0 + t * 128 + q * 16, z[q]);
+        for (int q = 0; q < 4; ++q) tmem_ld16_async(lane_base + scol + q * 16, z[q]);
 #pragma unroll
         for (int q = 0; q < 4; ++q) tmem_wait16(z[q]);
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl->s_empty[t]);
       const int lim = p.seq[c.s].Lp - c.j * kAttnUnitKeys;   // valid keys of the unit (>= 1)
       float mx = 0.f;   // a warp without rows keeps a finite reference
       if (wactive) {
@@ -438,9 +455,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
         m = mx;
       }
       if (wactive && __any_sync(kFull, move && live)) {
-        // the previous unit's P V must be done before this warp's O rows move
-        const int bp = b ^ 1;
-        if (!mbar_wait(&ctl->p_empty[bp], static_cast<uint32_t>(((bp ? fills1 : fills0) - 1) & 1), p.wait_ns)) {
+        // the previous unit's P V (committed to s_empty of its stage) must be
+        // done before this warp's O rows move
+        if (!mbar_wait(&ctl->s_empty[t ^ 1], static_cast<uint32_t>(((ui - 1) >> 1) & 1), p.wait_ns)) {
           fail(ctl, p.err);
           break;
         }
@@ -454,22 +471,13 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
           for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
           tmem_st16(lane_base + o_col + ch * 16, o);
         }
-        tmem_wait_st();
-        tc_fence_before();
       }
       l *= alpha;
-      // P into buffer b once the product of its previous fill is done
-      const int nfill = b ? fills1 : fills0;   // earlier fills of buffer b
-      if (nfill > 0 &&
-          !__all_sync(kFull, mbar_wait(&ctl->p_empty[b], static_cast<uint32_t>((nfill - 1) & 1), p.wait_ns))) {
-        fail(ctl, p.err);
-        break;
-      }
       if (wactive) {
+        // P over the first 32 of this unit's 64 S columns: keys 2j, 2j + 1 in column j
         const float2 sc2 = make_float2(c2, c2), nm2 = make_float2(-m, -m);
         float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                          make_float2(0.f, 0.f)};   // four independent running sums
-        uint8_t* prow = sP + (b * 2 + mt) * kPTileBytes + rho * 128;
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
           uint32_t h[8];
@@ -482,22 +490,20 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
             acc[(i >> 1) & 3] = fadd2(acc[(i >> 1) & 3], make_float2(p0, p1));
             h[i >> 1] = pack_half2(p0, p1);
           }
-          // keys 16q .. 16q + 15 are 16-byte chunks 2q and 2q + 1 of the row
-          *reinterpret_cast<uint4*>(prow + (((2 * q) ^ (rho & 7)) * 16)) = make_uint4(h[0], h[1], h[2], h[3]);
-          *reinterpret_cast<uint4*>(prow + (((2 * q + 1) ^ (rho & 7)) * 16)) = make_uint4(h[4], h[5], h[6], h[7]);
+          tmem_st8(lane_base + scol + q * 8, h);   // keys 16 q .. 16 q + 15: columns 8 q .. 8 q + 7
         }
         const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
         const float2 a = fadd2(a01, a23);
         l += a.x + a.y;
       }
-      fence_proxy_async_smem();
+      tmem_wait_st();
+      tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl->p_full[b]);
-      if (b) ++fills1; else ++fills0;
+      if (lane == 0) mbar_arrive(&ctl->p_full[t]);
       if (last) {
         // the piece's partial: (m, l) and the unnormalised O rows, once the
-        // product of this last unit (fill nfill of buffer b) is done
-        if (!__all_sync(kFull, mbar_wait(&ctl->p_empty[b], static_cast<uint32_t>(nfill & 1), p.wait_ns))) {
+        // product of this last unit is done
+        if (!__all_sync(kFull, mbar_wait(&ctl->s_empty[t], static_cast<uint32_t>((ui >> 1) & 1), p.wait_ns))) {
           fail(ctl, p.err);
           break;
         }
@@ -545,7 +551,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
       fence_proxy_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(&ctl->v_ready[stage]);
-      if (++stage == kStages) {
+      if (++stage == p.kv_stages) {
         stage = 0;
         phase ^= 1;
       }
@@ -621,9 +627,14 @@ __global__ void __launch_bounds__(256) k_attn_combine(const __grid_constant__ At
   if (lane == 0) sq.lse[row0 + r] = L > 0.f ? (M + log2f(L)) * 0.6931471805599453f : -INFINITY;
 }
 
-size_t attn_smem_bytes(int q_rows) {
-  return 1024 + static_cast<size_t>(2 * q_rows * 128) + 2 * static_cast<size_t>(kStages) * kUnitBytes +
-         4 * static_cast<size_t>(kPTileBytes) + 256;
+size_t attn_smem_bytes(int q_rows, int kv_stages) {
+  return 1024 + static_cast<size_t>(2 * q_rows * 128) + 2 * static_cast<size_t>(kv_stages) * kUnitBytes + 256;
+}
+
+int attn_kv_stages(int q_rows) {
+  int k = kStages;
+  while (k > 2 && attn_smem_bytes(q_rows, k) > kSmemLimit) --k;
+  return k;
 }
 
 cudaError_t attn_configure() {
@@ -651,7 +662,7 @@ cudaLaunchConfig_t pdl_config(cudaLaunchAttribute* attr, dim3 grid, dim3 block, 
 cudaError_t attn_main_launch(const AttnParams& p, cudaStream_t stream) {
   if (p.total_units <= 0) return cudaSuccess;
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = pdl_config(attr, dim3(p.grid), dim3(kAttnThreads), attn_smem_bytes(p.q_rows), stream);
+  cudaLaunchConfig_t cfg = pdl_config(attr, dim3(p.grid), dim3(kAttnThreads), attn_smem_bytes(p.q_rows, p.kv_stages), stream);
   return cudaLaunchKernelEx(&cfg, k_window_attn, p);
 }
 

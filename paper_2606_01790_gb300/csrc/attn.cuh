@@ -26,6 +26,7 @@ struct AttnParams {
   int rows;            // (H / G) * w window rows per group
   int n_mtiles;        // ceil(rows / 128)
   int q_rows;          // rows rounded up to 16 (shared-memory Q rows per half)
+  int kv_stages;       // depth of the K and V rings (attn_kv_stages)
   int grid;            // CTAs of the main kernel (defines the piece partition)
   int64_t total_units;
   float scale2;        // log2(e) / sqrt(d)
@@ -35,7 +36,9 @@ struct AttnParams {
   uint64_t wait_ns;
 };
 
-size_t attn_smem_bytes(int q_rows);
+size_t attn_smem_bytes(int q_rows, int kv_stages);
+// deepest K / V ring (at most 4) that fits the shared memory
+int attn_kv_stages(int q_rows);
 cudaError_t attn_configure();
 // Slots of piece partials a launch needs: one per (seq, layer, group) row plus
 // one per CTA of the main kernel.
