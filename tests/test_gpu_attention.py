@@ -178,6 +178,18 @@ def test_attention_at_other_shapes(shape):
     st.close()
 
 
+def test_attention_at_mha_head_granularity():
+    """G = H = 28 (each group's keys and values replicated for its query head):
+    32 rows per group, one M tile, 28 groups per layer."""
+    wl = syn.WORKLOADS["uitars_layer_mha"]
+    si = syn.make_sequence(wl)
+    st = sk.init_state(H.gpu_config(wl, H.hyper()))
+    ds = _attach(H.device_seq(si, wl), si, wl)
+    _run_attention(st, [ds])
+    check_layer(ds, si, wl, 0)
+    st.close()
+
+
 @pytest.mark.parametrize("name", ["tiny", "uitars_layer"])
 def test_step_fed_by_the_attention_pass_matches_oracle(name):
     """The compression step with lse = attn_lse: pass 1 skipped, the group
