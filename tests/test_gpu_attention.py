@@ -178,6 +178,18 @@ def test_attention_at_other_shapes(shape):
     st.close()
 
 
+def test_attention_on_a_56k_token_row():
+    """The long-cache shape (L_p = 56,096): about 880 units per row, so a
+    piece runs over hundreds of units and the references can move late."""
+    wl = syn.WORKLOADS["long_layer"]
+    si = syn.make_sequence(wl)
+    st = sk.init_state(H.gpu_config(wl, H.hyper()))
+    ds = _attach(H.device_seq(si, wl), si, wl)
+    _run_attention(st, [ds])
+    check_layer(ds, si, wl, 0)
+    st.close()
+
+
 def test_attention_at_mha_head_granularity():
     """G = H = 28 (each group's keys and values replicated for its query head):
     32 rows per group, one M tile, 28 groups per layer."""
