@@ -27,9 +27,11 @@
 //                       V arrives as bf16 and four warps convert it to fp16 in
 //                       place (exact for |v| < 65504), read as the transposed
 //                       (MN-major) operand.
-// The row reference m is the first unit's maximum and moves only when a
-// unit's maximum exceeds it by more than 15 (fp16 holds P < 2^16); the move
+// The row reference m is the piece's first unit's maximum and moves only when
+// a unit's maximum exceeds it by more than 15 (fp16 holds P < 2^16); the move
 // rescales that row's O in TMEM after the previous unit's P V is done (rare).
+// Later units take no maximum unless their sum of P exceeds 2^15: below that
+// no p can exceed 2^15, so no reference can have to move.
 // An S stage holds P until the P V product of its unit is done, which frees
 // it for S two units later.  Warp roles: warp 0 loads K (a four-stage ring,
 // each stage free once S of its unit is done) and Q per piece, warp 3 loads V
@@ -101,16 +103,6 @@ __host__ __device__ constexpr uint32_t idesc_f16_bmn(int M, int N) {
          | (1u << 16)                                // B major: MN
          | (static_cast<uint32_t>(N >> 3) << 17)
          | (static_cast<uint32_t>(M >> 4) << 24);
-}
-
-__device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                        uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
 }
 
 // D[tmem] (+)= A[tmem] * B[smem]: A with M = 128 rows on TMEM lanes and its
@@ -348,6 +340,209 @@ __device__ void mma_pv_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sV
   mbar_wait(&ctl->drain, 0, drain_limit(p.wait_ns));
 }
 
+// Maximum raw logit of a thread's row over the unit's first `lim` keys.
+__device__ __forceinline__ float unit_max(const uint32_t (&z)[4][16], int lim) {
+  float pm[8];   // eight independent partial maxima (short dependency chains)
+#pragma unroll
+  for (int k = 0; k < 8; ++k) pm[k] = -INFINITY;
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if (q * 16 + i < lim) pm[i & 7] = fmaxf(pm[i & 7], __uint_as_float(z[q][i]));
+  return fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])), fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+}
+
+// p = exp2(z c2 - m) of the unit's 64 keys (0 past `lim` and in a row that
+// is not live) as fp16 pairs h[q][j] = (p[16 q + 2 j], p[16 q + 2 j + 1]), the
+// lower key in the low half; returns the sum of the p.
+__device__ __forceinline__ float exp_pack_p(const uint32_t (&z)[4][16], int lim, bool live, float c2, float m,
+                                            uint32_t (&h)[4][8]) {
+  const float2 sc2 = make_float2(c2, c2), nm2 = make_float2(-m, -m);
+  float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                   make_float2(0.f, 0.f)};   // four independent running sums
+#pragma unroll
+  for (int q = 0; q < 4; ++q)
+#pragma unroll
+    for (int i = 0; i < 16; i += 2) {
+      const float2 e = ffma2(make_float2(__uint_as_float(z[q][i]), __uint_as_float(z[q][i + 1])), sc2, nm2);
+      const int k = q * 16 + i;
+      const float p0 = (live && k < lim) ? ex2_approx(e.x) : 0.f;
+      const float p1 = (live && k + 1 < lim) ? ex2_approx(e.y) : 0.f;
+      acc[(i >> 1) & 3] = fadd2(acc[(i >> 1) & 3], make_float2(p0, p1));
+      h[q][i >> 1] = pack_half2(p0, p1);
+    }
+  const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
+  const float2 a = fadd2(a01, a23);
+  return a.x + a.y;
+}
+
+// The unit's 64 S columns of this warp's lanes from `scol`, waited for.
+__device__ __forceinline__ void load_s(uint32_t scol, uint32_t (&z)[4][16]) {
+#pragma unroll
+  for (int q = 0; q < 4; ++q) tmem_ld16_async(scol + q * 16, z[q]);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) tmem_wait16(z[q]);
+}
+
+// Rescales this warp's O rows by alpha (1 in lanes whose reference stays).
+__device__ __forceinline__ void rescale_o(uint32_t o_addr, float alpha) {
+#pragma unroll 1
+  for (int ch = 0; ch < kHeadDim / 16; ++ch) {
+    uint32_t o[16];
+    tmem_ld16_async(o_addr + ch * 16, o);
+    tmem_wait16(o);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
+    tmem_st16(o_addr + ch * 16, o);
+  }
+}
+
+// One unit of a softmax warp (warp-uniform `wactive`; TMEM loads and stores
+// are warp-collective): S at `scol` becomes P over its first 32 columns, and
+// the reference m and sum l of the thread's row advance.  `fresh`: the
+// piece's first unit, whose maximum sets the reference.  P is computed with
+// the current reference; every p is below 2^15 unless the unit's sum exceeds
+// it, and only then is the maximum taken (S is still in place, P is stored
+// last): lanes where it lies more than 15 above the reference move it and
+// rescale their O rows (at o_addr, once the product of the previous unit,
+// phase `prev_par` of `prev_bar`, is done), and P is redone.  Returns false
+// when that wait ran out.
+__device__ __forceinline__ bool softmax_unit(const AttnParams& p, bool wactive, bool live, bool fresh, int lim,
+                                             uint32_t scol, uint32_t o_addr, uint64_t* prev_bar, uint32_t prev_par,
+                                             float& m, float& l) {
+  const float c2 = p.scale2;
+  if (fresh) l = 0.f;
+  if (!wactive) {
+    if (fresh) m = 0.f;   // a warp without rows keeps a finite reference
+    return true;
+  }
+  uint32_t z[4][16];
+  uint32_t h[4][8];
+  load_s(scol, z);
+  if (fresh) m = unit_max(z, lim) * c2;
+  float us = exp_pack_p(z, lim, live, c2, m, h);
+  if (__any_sync(kFull, live && us > 32768.f)) {   // rare
+    load_s(scol, z);   // z again, so that it need not live across the first pass
+    const float mx = unit_max(z, lim) * c2;
+    const bool move = live && mx > m + kMoveThreshold;
+    if (__any_sync(kFull, move)) {
+      const float alpha = move ? ex2_approx(m - mx) : 1.f;
+      if (move) m = mx;
+      if (!__all_sync(kFull, mbar_wait(prev_bar, prev_par, p.wait_ns))) return false;
+      tc_fence_after();
+      rescale_o(o_addr, alpha);
+      l *= alpha;
+    }
+    // P again in every lane (the same values where the reference stayed), so
+    // that the first h need not live across the reload either
+    us = exp_pack_p(z, lim, live, c2, m, h);
+  }
+#pragma unroll
+  for (int q = 0; q < 4; ++q) tmem_st8(scol + q * 8, h[q]);   // keys 16 q ..: columns 8 q ..
+  l += us;
+  return true;
+}
+
+// Softmax warps: one thread per window row of M tile `mt` (TMEM lane
+// quad * 32 + lane).  NS S stages, unit u in stage u mod NS; the S (then P)
+// columns of stage t start at s_col0 + t s_stride and O at o_col.  A piece's
+// partial goes to slot row + slot0.
+template <int NS>
+__device__ void softmax_loop(const AttnParams& p, AttnCtl* ctl, uint32_t tmem, int mt, int quad, int lane,
+                             uint32_t s_col0, uint32_t s_stride, uint32_t o_col, int slot0, int64_t fb, int64_t fe) {
+  const int rho = quad * 32 + lane;   // row within the M tile (TMEM lane)
+  const int r = mt * 128 + rho;       // window row within the group
+  const bool wactive = mt < p.n_mtiles && mt * 128 + quad * 32 < p.rows;
+  const bool live = r < p.rows;
+  const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+  float m = -INFINITY, l = 0.f;
+  uint32_t ui = 0;
+  UnitIter c;
+  for (c.init(p, fb, fe); c.valid(); c.next(p), ++ui) {
+    if (ctl->abort) break;
+    const bool first = c.first(fb), last = c.last();
+    const int t = static_cast<int>(ui % NS);
+    const uint32_t par = (ui / NS) & 1u;
+    const uint32_t scol = s_col0 + t * s_stride;   // this unit's S, then P, columns
+    if (!__all_sync(kFull, mbar_wait(&ctl->s_full[t], par, p.wait_ns))) {
+      fail(ctl, p.err);
+      break;
+    }
+    tc_fence_after();
+    const int lim = p.seq[c.s].Lp - c.j * kAttnUnitKeys;   // valid keys of the unit (>= 1)
+    const uint32_t up = ui - 1;   // the previous unit (a piece's first unit never moves)
+    if (!softmax_unit(p, wactive, live, first, lim, lane_base + scol, lane_base + o_col, &ctl->s_empty[up % NS],
+                             (up / NS) & 1u, m, l)) {
+      fail(ctl, p.err);
+      break;
+    }
+    tmem_wait_st();
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&ctl->p_full[t]);
+    if (last) {
+      // the piece's partial: (m, l) and the unnormalised O rows, once the
+      // product of this last unit is done
+      if (!__all_sync(kFull, mbar_wait(&ctl->s_empty[t], par, p.wait_ns))) {
+        fail(ctl, p.err);
+        break;
+      }
+      tc_fence_after();
+      const int64_t slot = static_cast<int64_t>(c.row(p)) + slot0;
+      if (wactive) {
+        float* dst = p.part_o + (slot * kMaxRows + r) * kHeadDim;
+#pragma unroll 1
+        for (int ch = 0; ch < kHeadDim / 16; ++ch) {
+          uint32_t o[16];
+          tmem_ld16_async(lane_base + o_col + ch * 16, o);
+          tmem_wait16(o);
+          if (live)
+#pragma unroll
+            for (int i = 0; i < 16; i += 4)
+              *reinterpret_cast<float4*>(dst + ch * 16 + i) =
+                  make_float4(__uint_as_float(o[i]), __uint_as_float(o[i + 1]), __uint_as_float(o[i + 2]),
+                              __uint_as_float(o[i + 3]));
+        }
+        if (live) p.part_ml[slot * kMaxRows + r] = make_float2(m, l);
+      }
+      tc_fence_before();
+    }
+  }
+}
+
+// V conversion warps (NW of them, thread ct of 32 NW): V of every unit to
+// fp16 in place, then released to the P V product.
+template <int NW>
+__device__ void convert_loop(const AttnParams& p, AttnCtl* ctl, uint8_t* sV, int kv_stages, int ct, int lane, int64_t fb,
+                             int64_t fe) {
+  int stage = 0, phase = 0;
+  for (int64_t f = fb; f < fe; ++f) {
+    if (ctl->abort) break;
+    if (!__all_sync(kFull, mbar_wait(&ctl->v_full[stage], phase, p.wait_ns))) {
+      fail(ctl, p.err);
+      break;
+    }
+    uint4* v4 = reinterpret_cast<uint4*>(sV + stage * kUnitBytes);
+#pragma unroll
+    for (int i = 0; i < kUnitBytes / 16 / (32 * NW); ++i) {
+      uint4 x = v4[ct + i * 32 * NW];
+      x.x = bf16x2_to_f16x2(x.x);
+      x.y = bf16x2_to_f16x2(x.y);
+      x.z = bf16x2_to_f16x2(x.z);
+      x.w = bf16x2_to_f16x2(x.w);
+      v4[ct + i * 32 * NW] = x;
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&ctl->v_ready[stage]);
+    if (++stage == kv_stages) {
+      stage = 0;
+      phase ^= 1;
+    }
+  }
+}
+
 }  // namespace
 
 __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_constant__ AttnParams p) {
@@ -401,161 +596,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
   } else if (warp == 2) {
     if (lane == 0) mma_pv_loop(p, ctl, sV, tmem, fb, fe);
   } else if (warp >= kSoftWarp0 && warp < kSoftWarp0 + kSoftWarps) {
-    const int mt = (warp - kSoftWarp0) >> 2, quad = warp & 3;
-    const int rho = quad * 32 + lane;                  // row within the M tile (TMEM lane)
-    const int r = mt * 128 + rho;                      // window row within the group
-    const bool wactive = mt < p.n_mtiles && mt * 128 + quad * 32 < p.rows;
-    const bool live = r < p.rows;
-    const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
-    const uint32_t s_col0 = 256 + mt * kAttnUnitKeys, o_col = mt * kHeadDim;
-    const float c2 = p.scale2;
-    float m = -INFINITY, l = 0.f;
-    int64_t ui = 0;
-    UnitIter c;
-    for (c.init(p, fb, fe); c.valid(); c.next(p), ++ui) {
-      if (ctl->abort) break;
-      const bool first = c.first(fb), last = c.last();
-      const int t = static_cast<int>(ui & 1);
-      const uint32_t scol = s_col0 + t * 128;   // this unit's S, then P, columns
-      if (!__all_sync(kFull, mbar_wait(&ctl->s_full[t], static_cast<uint32_t>((ui >> 1) & 1), p.wait_ns))) {
-        fail(ctl, p.err);
-        break;
-      }
-      tc_fence_after();
-      uint32_t z[4][16];
-      if (wactive) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) tmem_ld16_async(lane_base + scol + q * 16, z[q]);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) tmem_wait16(z[q]);
-      }
-      const int lim = p.seq[c.s].Lp - c.j * kAttnUnitKeys;   // valid keys of the unit (>= 1)
-      float mx = 0.f;   // a warp without rows keeps a finite reference
-      if (wactive) {
-        // eight independent partial maxima (short dependency chains)
-        float pm[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) pm[k] = -INFINITY;
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-#pragma unroll
-          for (int i = 0; i < 16; ++i)
-            if (q * 16 + i < lim) pm[i & 7] = fmaxf(pm[i & 7], __uint_as_float(z[q][i]));
-        mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])), fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
-        mx *= c2;
-      }
-      float alpha = 1.f;
-      bool move = false;
-      if (first) {
-        m = mx;
-        l = 0.f;
-      } else if (mx > m + kMoveThreshold) {
-        move = true;
-        alpha = ex2_approx(m - mx);
-        m = mx;
-      }
-      if (wactive && __any_sync(kFull, move && live)) {
-        // the previous unit's P V (committed to s_empty of its stage) must be
-        // done before this warp's O rows move
-        if (!mbar_wait(&ctl->s_empty[t ^ 1], static_cast<uint32_t>(((ui - 1) >> 1) & 1), p.wait_ns)) {
-          fail(ctl, p.err);
-          break;
-        }
-        tc_fence_after();
-#pragma unroll 1
-        for (int ch = 0; ch < kHeadDim / 16; ++ch) {
-          uint32_t o[16];
-          tmem_ld16_async(lane_base + o_col + ch * 16, o);
-          tmem_wait16(o);
-#pragma unroll
-          for (int i = 0; i < 16; ++i) o[i] = __float_as_uint(__uint_as_float(o[i]) * alpha);
-          tmem_st16(lane_base + o_col + ch * 16, o);
-        }
-      }
-      l *= alpha;
-      if (wactive) {
-        // P over the first 32 of this unit's 64 S columns: keys 2j, 2j + 1 in column j
-        const float2 sc2 = make_float2(c2, c2), nm2 = make_float2(-m, -m);
-        float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
-                         make_float2(0.f, 0.f)};   // four independent running sums
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          uint32_t h[8];
-#pragma unroll
-          for (int i = 0; i < 16; i += 2) {
-            const float2 e = ffma2(make_float2(__uint_as_float(z[q][i]), __uint_as_float(z[q][i + 1])), sc2, nm2);
-            const int k = q * 16 + i;
-            const float p0 = (live && k < lim) ? ex2_approx(e.x) : 0.f;
-            const float p1 = (live && k + 1 < lim) ? ex2_approx(e.y) : 0.f;
-            acc[(i >> 1) & 3] = fadd2(acc[(i >> 1) & 3], make_float2(p0, p1));
-            h[i >> 1] = pack_half2(p0, p1);
-          }
-          tmem_st8(lane_base + scol + q * 8, h);   // keys 16 q .. 16 q + 15: columns 8 q .. 8 q + 7
-        }
-        const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
-        const float2 a = fadd2(a01, a23);
-        l += a.x + a.y;
-      }
-      tmem_wait_st();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl->p_full[t]);
-      if (last) {
-        // the piece's partial: (m, l) and the unnormalised O rows, once the
-        // product of this last unit is done
-        if (!__all_sync(kFull, mbar_wait(&ctl->s_empty[t], static_cast<uint32_t>((ui >> 1) & 1), p.wait_ns))) {
-          fail(ctl, p.err);
-          break;
-        }
-        tc_fence_after();
-        const int64_t slot = static_cast<int64_t>(c.row(p)) + blockIdx.x;
-        if (wactive) {
-          float* dst = p.part_o + (slot * kMaxRows + r) * kHeadDim;
-#pragma unroll 1
-          for (int ch = 0; ch < kHeadDim / 16; ++ch) {
-            uint32_t o[16];
-            tmem_ld16_async(lane_base + o_col + ch * 16, o);
-            tmem_wait16(o);
-            if (live)
-#pragma unroll
-              for (int i = 0; i < 16; i += 4)
-                *reinterpret_cast<float4*>(dst + ch * 16 + i) =
-                    make_float4(__uint_as_float(o[i]), __uint_as_float(o[i + 1]), __uint_as_float(o[i + 2]),
-                                __uint_as_float(o[i + 3]));
-          }
-          if (live) p.part_ml[slot * kMaxRows + r] = make_float2(m, l);
-        }
-        tc_fence_before();
-      }
-    }
+    const int mt = (warp - kSoftWarp0) >> 2;
+    softmax_loop<2>(p, ctl, tmem, mt, warp & 3, lane, 256 + mt * kAttnUnitKeys, 128, mt * kHeadDim, blockIdx.x, fb, fe);
   } else if (warp >= kConvWarp0) {
-    // V of every unit to fp16 in place, then released to the P V product
-    const int ct = threadIdx.x - 32 * kConvWarp0;
-    int stage = 0, phase = 0;
-    for (int64_t f = fb; f < fe; ++f) {
-      if (ctl->abort) break;
-      if (!__all_sync(kFull, mbar_wait(&ctl->v_full[stage], phase, p.wait_ns))) {
-        fail(ctl, p.err);
-        break;
-      }
-      uint4* v4 = reinterpret_cast<uint4*>(sV + stage * kUnitBytes);
-#pragma unroll
-      for (int i = 0; i < kUnitBytes / 16 / (32 * kConvWarps); ++i) {
-        uint4 x = v4[ct + i * 32 * kConvWarps];
-        x.x = bf16x2_to_f16x2(x.x);
-        x.y = bf16x2_to_f16x2(x.y);
-        x.z = bf16x2_to_f16x2(x.z);
-        x.w = bf16x2_to_f16x2(x.w);
-        v4[ct + i * 32 * kConvWarps] = x;
-      }
-      fence_proxy_async_smem();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&ctl->v_ready[stage]);
-      if (++stage == p.kv_stages) {
-        stage = 0;
-        phase ^= 1;
-      }
-    }
+    convert_loop<kConvWarps>(p, ctl, sV, p.kv_stages, threadIdx.x - 32 * kConvWarp0, lane, fb, fe);
   }
   __syncthreads();
   if (warp == 1) {
