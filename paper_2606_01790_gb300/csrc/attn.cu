@@ -353,6 +353,20 @@ __device__ __forceinline__ float unit_max(const uint32_t (&z)[4][16], int lim) {
   return fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])), fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
 }
 
+// exp2 and pack of one 16-key chunk (keys k0 .. k0 + 15)
+__device__ __forceinline__ void exp_pack_chunk(const uint32_t (&z)[16], int k0, int lim, bool live, float2 sc2,
+                                               float2 nm2, float2 (&acc)[4], uint32_t (&h)[8]) {
+#pragma unroll
+  for (int i = 0; i < 16; i += 2) {
+    const float2 e = ffma2(make_float2(__uint_as_float(z[i]), __uint_as_float(z[i + 1])), sc2, nm2);
+    const int k = k0 + i;
+    const float p0 = (live && k < lim) ? ex2_approx(e.x) : 0.f;
+    const float p1 = (live && k + 1 < lim) ? ex2_approx(e.y) : 0.f;
+    acc[(i >> 1) & 3] = fadd2(acc[(i >> 1) & 3], make_float2(p0, p1));
+    h[i >> 1] = pack_half2(p0, p1);
+  }
+}
+
 // p = exp2(z c2 - m) of the unit's 64 keys (0 past `lim` and in a row that
 // is not live) as fp16 pairs h[q][j] = (p[16 q + 2 j], p[16 q + 2 j + 1]), the
 // lower key in the low half; returns the sum of the p.
@@ -362,16 +376,33 @@ __device__ __forceinline__ float exp_pack_p(const uint32_t (&z)[4][16], int lim,
   float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
                    make_float2(0.f, 0.f)};   // four independent running sums
 #pragma unroll
-  for (int q = 0; q < 4; ++q)
-#pragma unroll
-    for (int i = 0; i < 16; i += 2) {
-      const float2 e = ffma2(make_float2(__uint_as_float(z[q][i]), __uint_as_float(z[q][i + 1])), sc2, nm2);
-      const int k = q * 16 + i;
-      const float p0 = (live && k < lim) ? ex2_approx(e.x) : 0.f;
-      const float p1 = (live && k + 1 < lim) ? ex2_approx(e.y) : 0.f;
-      acc[(i >> 1) & 3] = fadd2(acc[(i >> 1) & 3], make_float2(p0, p1));
-      h[q][i >> 1] = pack_half2(p0, p1);
-    }
+  for (int q = 0; q < 4; ++q) exp_pack_chunk(z[q], 16 * q, lim, live, sc2, nm2, acc, h[q]);
+  const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
+  const float2 a = fadd2(a01, a23);
+  return a.x + a.y;
+}
+
+// exp_pack_p reading S itself from `scol` in two halves, the second half's
+// loads in flight under the first half's arithmetic (measured faster than
+// waiting for all four loads first, and than one 16-column load ahead)
+__device__ __forceinline__ float exp_pack_p_streamed(uint32_t scol, int lim, bool live, float c2, float m,
+                                                     uint32_t (&h)[4][8]) {
+  const float2 sc2 = make_float2(c2, c2), nm2 = make_float2(-m, -m);
+  float2 acc[4] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f), make_float2(0.f, 0.f),
+                   make_float2(0.f, 0.f)};   // four independent running sums
+  uint32_t a0[16], a1[16], b0[16], b1[16];
+  tmem_ld16_async(scol, a0);
+  tmem_ld16_async(scol + 16, a1);
+  tmem_wait16(a0);
+  tmem_wait16(a1);
+  tmem_ld16_async(scol + 32, b0);
+  tmem_ld16_async(scol + 48, b1);
+  exp_pack_chunk(a0, 0, lim, live, sc2, nm2, acc, h[0]);
+  exp_pack_chunk(a1, 16, lim, live, sc2, nm2, acc, h[1]);
+  tmem_wait16(b0);
+  tmem_wait16(b1);
+  exp_pack_chunk(b0, 32, lim, live, sc2, nm2, acc, h[2]);
+  exp_pack_chunk(b1, 48, lim, live, sc2, nm2, acc, h[3]);
   const float2 a01 = fadd2(acc[0], acc[1]), a23 = fadd2(acc[2], acc[3]);
   const float2 a = fadd2(a01, a23);
   return a.x + a.y;
@@ -419,9 +450,14 @@ __device__ __forceinline__ bool softmax_unit(const AttnParams& p, bool wactive, 
   }
   uint32_t z[4][16];
   uint32_t h[4][8];
-  load_s(scol, z);
-  if (fresh) m = unit_max(z, lim) * c2;
-  float us = exp_pack_p(z, lim, live, c2, m, h);
+  float us;
+  if (fresh) {
+    load_s(scol, z);
+    m = unit_max(z, lim) * c2;
+    us = exp_pack_p(z, lim, live, c2, m, h);
+  } else {
+    us = exp_pack_p_streamed(scol, lim, live, c2, m, h);
+  }
   if (__any_sync(kFull, live && us > 32768.f)) {   // rare
     load_s(scol, z);   // z again, so that it need not live across the first pass
     const float mx = unit_max(z, lim) * c2;
