@@ -202,6 +202,35 @@ def test_attention_at_mha_head_granularity():
     st.close()
 
 
+@pytest.mark.parametrize("lift", [10.0, 20.0], ids=["sum_over_guard", "reference_moves"])
+def test_attention_units_far_above_the_reference(lift):
+    """Alternate 64-key units whose logits sit `lift` log2 units above the
+    others (every window row, every group).  lift 10: a unit's 64 p reach
+    about 2^16 in sum although none exceeds 2^15, so the softmax takes the
+    unit maximum and keeps its reference (no move); lift 20: p would reach
+    2^20, so rows move their reference in the middle of a piece and rescale O.
+    Both against the fp64 oracle at the usual bounds."""
+    wl = syn.WORKLOADS["uitars_layer"]
+    si = syn.make_sequence(wl)
+    d, lp = wl.head_dim, si.L - wl.window
+    g = torch.Generator().manual_seed(7)
+    beta = 8.0
+    gamma = lift / (beta / math.sqrt(d) * math.log2(math.e))   # q.k / sqrt(d) = lift / log2(e)
+    q = 0.05 * torch.randn(si.q.shape, generator=g)
+    q[..., 0] = beta
+    k = si.k.float().clone()
+    k[..., :lp, :] = 0.05 * torch.randn(k[..., :lp, :].shape, generator=g)
+    units = torch.arange(lp) // 64
+    k[..., :lp, 0] = torch.where(units % 2 == 1, torch.tensor(gamma), torch.tensor(0.0))
+    si.q = q.to(torch.bfloat16)
+    si.k = k.to(torch.bfloat16)
+    st = sk.init_state(H.gpu_config(wl, H.hyper()))
+    ds = _attach(H.device_seq(si, wl), si, wl)
+    _run_attention(st, [ds])
+    check_layer(ds, si, wl, 0)
+    st.close()
+
+
 @pytest.mark.parametrize("name", ["tiny", "uitars_layer"])
 def test_step_fed_by_the_attention_pass_matches_oracle(name):
     """The compression step with lse = attn_lse: pass 1 skipped, the group
