@@ -648,8 +648,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
 // 2^(m - M) l, O = sum 2^(m - M) O_piece / L, lse = (M + log2 L) ln 2.
 // grid: (rows of the launch, ceil(window rows / 8)); one warp per window row,
 // four output columns per lane, every piece's loads issued before the sums.
-constexpr int kMaxPieces = 8;   // pieces merged per batch of loads
-__global__ void __launch_bounds__(256) k_attn_combine(const __grid_constant__ AttnParams p) {
+// Four pieces per batch of loads and six 256-thread blocks per SM (at most 40
+// registers): more rows' loads in flight than eight pieces at three blocks.
+constexpr int kMaxPieces = 4;   // pieces merged per batch of loads
+__global__ void __launch_bounds__(256, 6) k_attn_combine(const __grid_constant__ AttnParams p) {
   griddep_launch_dependents();
   griddep_wait();
   const int R = blockIdx.x;
