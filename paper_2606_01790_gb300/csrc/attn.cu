@@ -19,9 +19,11 @@
 //   S = Q K^T           M = 128 rows, N = 64 keys, K = d, bf16 -> fp32 in TMEM
 //                       (two S stages, so the MMA of unit u+1 runs under the
 //                       softmax of unit u);
-//   softmax             rows on TMEM lanes, one thread per row: p = exp2(S c - m),
-//                       l += p in fp32, P rounded to fp16 and written over the
-//                       S columns it came from (two fp16 per 32-bit column);
+//   softmax             rows on TMEM lanes, one thread per row: S read in two
+//                       halves (the second half's loads under the first half's
+//                       arithmetic), p = exp2(S c - m), l += p in fp32, P
+//                       rounded to fp16 and written over the first 32 of the
+//                       unit's 64 S columns (two fp16 per 32-bit column);
 //   O += P V            M = 128, N = d = 128, K = 64 keys, fp16 -> fp32 in TMEM,
 //                       A = P read from tensor memory;
 //                       V arrives as bf16 and four warps convert it to fp16 in
@@ -480,11 +482,13 @@ __device__ __forceinline__ bool softmax_unit(const AttnParams& p, bool wactive, 
   return true;
 }
 
+constexpr int kSStages = 2;   // S stages in tensor memory
+
 // Softmax warps: one thread per window row of M tile `mt` (TMEM lane
-// quad * 32 + lane).  NS S stages, unit u in stage u mod NS; the S (then P)
+// quad * 32 + lane).  Unit u sits in S stage u mod kSStages; the S (then P)
 // columns of stage t start at s_col0 + t s_stride and O at o_col.  A piece's
 // partial goes to slot row + slot0.
-template <int NS>
+
 __device__ void softmax_loop(const AttnParams& p, AttnCtl* ctl, uint32_t tmem, int mt, int quad, int lane,
                              uint32_t s_col0, uint32_t s_stride, uint32_t o_col, int slot0, int64_t fb, int64_t fe) {
   const int rho = quad * 32 + lane;   // row within the M tile (TMEM lane)
@@ -498,8 +502,8 @@ __device__ void softmax_loop(const AttnParams& p, AttnCtl* ctl, uint32_t tmem, i
   for (c.init(p, fb, fe); c.valid(); c.next(p), ++ui) {
     if (ctl->abort) break;
     const bool first = c.first(fb), last = c.last();
-    const int t = static_cast<int>(ui % NS);
-    const uint32_t par = (ui / NS) & 1u;
+    const int t = static_cast<int>(ui % kSStages);
+    const uint32_t par = (ui / kSStages) & 1u;
     const uint32_t scol = s_col0 + t * s_stride;   // this unit's S, then P, columns
     if (!__all_sync(kFull, mbar_wait(&ctl->s_full[t], par, p.wait_ns))) {
       fail(ctl, p.err);
@@ -508,8 +512,8 @@ __device__ void softmax_loop(const AttnParams& p, AttnCtl* ctl, uint32_t tmem, i
     tc_fence_after();
     const int lim = p.seq[c.s].Lp - c.j * kAttnUnitKeys;   // valid keys of the unit (>= 1)
     const uint32_t up = ui - 1;   // the previous unit (a piece's first unit never moves)
-    if (!softmax_unit(p, wactive, live, first, lim, lane_base + scol, lane_base + o_col, &ctl->s_empty[up % NS],
-                             (up / NS) & 1u, m, l)) {
+    if (!softmax_unit(p, wactive, live, first, lim, lane_base + scol, lane_base + o_col,
+                      &ctl->s_empty[up % kSStages], (up / kSStages) & 1u, m, l)) {
       fail(ctl, p.err);
       break;
     }
@@ -633,7 +637,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
     if (lane == 0) mma_pv_loop(p, ctl, sV, tmem, fb, fe);
   } else if (warp >= kSoftWarp0 && warp < kSoftWarp0 + kSoftWarps) {
     const int mt = (warp - kSoftWarp0) >> 2;
-    softmax_loop<2>(p, ctl, tmem, mt, warp & 3, lane, 256 + mt * kAttnUnitKeys, 128, mt * kHeadDim, blockIdx.x, fb, fe);
+    softmax_loop(p, ctl, tmem, mt, warp & 3, lane, 256 + mt * kAttnUnitKeys, 128, mt * kHeadDim, blockIdx.x, fb, fe);
   } else if (warp >= kConvWarp0) {
     convert_loop<kConvWarps>(p, ctl, sV, p.kv_stages, threadIdx.x - 32 * kConvWarp0, lane, fb, fe);
   }
