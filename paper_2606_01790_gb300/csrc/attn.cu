@@ -71,14 +71,16 @@ __device__ __forceinline__ uint64_t drain_limit(uint64_t wait_ns) {
 struct AttnCtl {
   uint64_t k_full[kStages], k_empty[kStages];
   uint64_t v_full[kStages], v_empty[kStages], v_ready[kStages];
-  uint64_t s_full[2], s_empty[2];   // s_empty: the stage's P V is done
-  uint64_t p_full[2];               // P of the stage written
+  uint64_t s_full[2][2];   // [stage][M tile]: S of that M tile is in the stage
+  uint64_t s_empty[2];      // the stage's P V products are done
+  uint64_t p_full[2][2];    // [stage][M tile]: P of that M tile is written
   uint64_t q_full, q_empty, drain;
   uint32_t tmem_base;
   volatile int abort;
 };
 
-static_assert(sizeof(AttnCtl) <= 256, "the control block has 256 bytes");
+constexpr int kCtlBytes = 512;
+static_assert(sizeof(AttnCtl) <= kCtlBytes, "the control block fits its bytes");
 
 __device__ __forceinline__ void fail(AttnCtl* ctl, uint32_t* err) {
   ctl->abort = 1;
@@ -294,8 +296,8 @@ __device__ void mma_s_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sQ,
         const uint32_t qoff16 = (kk >> 2) * qhalf16 + (kk & 3) * 2;
         mma_bf16(tmem + 256 + t * 128 + mt * kAttnUnitKeys, dq + qoff16, dk + koff16, idesc_s, kk > 0);
       }
+      mma_commit(&ctl->s_full[t][mt]);   // that M tile's softmax starts without waiting for the next
     }
-    mma_commit(&ctl->s_full[t]);
     mma_commit(&ctl->k_empty[stage]);
     if (c.last()) mma_commit(&ctl->q_empty);
     if (++stage == p.kv_stages) {
@@ -318,18 +320,27 @@ __device__ void mma_pv_loop(const AttnParams& p, AttnCtl* ctl, const uint8_t* sV
     if (ctl->abort) break;
     const int t = static_cast<int>(ui & 1);
     if (!mbar_wait(&ctl->v_ready[stage], kphase, p.wait_ns)) { fail(ctl, p.err); break; }
-    if (!mbar_wait(&ctl->p_full[t], static_cast<uint32_t>((ui >> 1) & 1), p.wait_ns)) { fail(ctl, p.err); break; }
-    tc_fence_after();
     const bool first = c.first(fb);   // the piece's first product overwrites O
     const uint64_t dv = sdesc_mn_sw128(smem_u32(sV + stage * kUnitBytes), kHalfBytes, 1024);
+    bool ok = true;
 #pragma unroll
     for (int mt = 0; mt < 2; ++mt) {
       if (mt >= p.n_mtiles) break;
+      // each M tile's product as soon as its P is written
+      if (!mbar_wait(&ctl->p_full[t][mt], static_cast<uint32_t>((ui >> 1) & 1), p.wait_ns)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
       const uint32_t ap = tmem + 256 + t * 128 + mt * kAttnUnitKeys;   // P of M tile mt over its S columns
 #pragma unroll
       for (int kk = 0; kk < 4; ++kk)   // 16 keys per step: +8 columns of P, +16 rows of V
         mma_f16_ts(tmem + mt * kHeadDim, ap + kk * 8, dv + static_cast<uint64_t>(kk * 128), idesc_o,
                    (!first || kk > 0) ? 1u : 0u);
+    }
+    if (!ok) {
+      fail(ctl, p.err);
+      break;
     }
     mma_commit(&ctl->v_empty[stage]);
     mma_commit(&ctl->s_empty[t]);   // S stage t (holding P) is free for S two units later
@@ -493,7 +504,8 @@ __device__ void softmax_loop(const AttnParams& p, AttnCtl* ctl, uint32_t tmem, i
                              uint32_t s_col0, uint32_t s_stride, uint32_t o_col, int slot0, int64_t fb, int64_t fe) {
   const int rho = quad * 32 + lane;   // row within the M tile (TMEM lane)
   const int r = mt * 128 + rho;       // window row within the group
-  const bool wactive = mt < p.n_mtiles && mt * 128 + quad * 32 < p.rows;
+  if (mt >= p.n_mtiles) return;   // no S is computed for this M tile, no P awaited from it
+  const bool wactive = mt * 128 + quad * 32 < p.rows;
   const bool live = r < p.rows;
   const uint32_t lane_base = tmem + (static_cast<uint32_t>(quad * 32) << 16);
   float m = -INFINITY, l = 0.f;
@@ -505,7 +517,7 @@ __device__ void softmax_loop(const AttnParams& p, AttnCtl* ctl, uint32_t tmem, i
     const int t = static_cast<int>(ui % kSStages);
     const uint32_t par = (ui / kSStages) & 1u;
     const uint32_t scol = s_col0 + t * s_stride;   // this unit's S, then P, columns
-    if (!__all_sync(kFull, mbar_wait(&ctl->s_full[t], par, p.wait_ns))) {
+    if (!__all_sync(kFull, mbar_wait(&ctl->s_full[t][mt], par, p.wait_ns))) {
       fail(ctl, p.err);
       break;
     }
@@ -520,7 +532,7 @@ __device__ void softmax_loop(const AttnParams& p, AttnCtl* ctl, uint32_t tmem, i
     tmem_wait_st();
     tc_fence_before();
     __syncwarp();
-    if (lane == 0) mbar_arrive(&ctl->p_full[t]);
+    if (lane == 0) mbar_arrive(&ctl->p_full[t][mt]);
     if (last) {
       // the piece's partial: (m, l) and the unnormalised O rows, once the
       // product of this last unit is done
@@ -603,9 +615,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_window_attn(const __grid_co
       mbar_init(&ctl->v_ready[i], kConvWarps);
     }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&ctl->s_full[i], 1);
+      for (int m = 0; m < 2; ++m) {
+        mbar_init(&ctl->s_full[i][m], 1);
+        mbar_init(&ctl->p_full[i][m], kSoftWarps / 2);   // the four warps of the M tile
+      }
       mbar_init(&ctl->s_empty[i], 1);   // the P V issuer's commit
-      mbar_init(&ctl->p_full[i], kSoftWarps);
     }
     mbar_init(&ctl->q_full, 1);
     mbar_init(&ctl->q_empty, 1);
@@ -714,7 +728,7 @@ __global__ void __launch_bounds__(256, 6) k_attn_combine(const __grid_constant__
 }
 
 size_t attn_smem_bytes(int q_rows, int kv_stages) {
-  return 1024 + static_cast<size_t>(2 * q_rows * 128) + 2 * static_cast<size_t>(kv_stages) * kUnitBytes + 256;
+  return 1024 + static_cast<size_t>(2 * q_rows * 128) + 2 * static_cast<size_t>(kv_stages) * kUnitBytes + kCtlBytes;
 }
 
 int attn_kv_stages(int q_rows) {
