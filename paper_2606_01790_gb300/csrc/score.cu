@@ -122,7 +122,7 @@ struct TileIter {
 struct SmemCtl {
   uint64_t k_full[kMaxStages];
   uint64_t k_empty[kMaxStages];
-  uint64_t t_full[2];
+  uint64_t t_full[2][2];   // [accumulator stage][M tile]: that M tile's tile product is done
   uint64_t t_empty[2];
   uint64_t q_full;
   uint64_t q_empty;
@@ -149,7 +149,7 @@ __device__ __forceinline__ void ctl_init(SmemCtl* ctl, int kstages) {
     mbar_init(&ctl->k_empty[i], 1);
   }
   for (int i = 0; i < 2; ++i) {
-    mbar_init(&ctl->t_full[i], 1);
+    for (int m = 0; m < 2; ++m) mbar_init(&ctl->t_full[i][m], 1);
     mbar_init(&ctl->t_empty[i], kEpiWarps);   // one arrival per epilogue warp
   }
   mbar_init(&ctl->q_full, 1);
@@ -268,6 +268,7 @@ __device__ void mma_loop(const ScoreParams& p, SmemCtl* ctl, const uint8_t* sQ, 
             const uint32_t qoff16 = (kk >> 2) * qhalf16 + (kk & 3) * 2;
             mma_bf16(d, dq + qoff16, dk + koff16, idesc, kk > 0);
           }
+          mma_commit(&ctl->t_full[who][mt]);   // that M tile's epilogue starts without waiting for the next
         }
       } else {
 #pragma unroll
@@ -277,9 +278,9 @@ __device__ void mma_loop(const ScoreParams& p, SmemCtl* ctl, const uint8_t* sQ, 
           mma_bf16(d0, dk + koff16, dq0 + qoff16, idesc, kk > 0);
         }
         mma_bf16(d0, dax, dbx, idesc, 1);
+        mma_commit(&ctl->t_full[who][0]);
       }
       mma_commit(&ctl->k_empty[stage]);
-      mma_commit(&ctl->t_full[who]);
       ++own;
       stage += 2;
       if (stage >= p.kstages) {
@@ -495,7 +496,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_lse(const __grid_con
       }
       const int ts = jt & 1;
       if (!dead) {
-        if (!__all_sync(kFull, mbar_wait(&ctl->t_full[ts], (jt >> 1) & 1, p.wait_ns))) {
+        if (!__all_sync(kFull, mbar_wait(&ctl->t_full[ts][mt], (jt >> 1) & 1, p.wait_ns))) {
           fail(ctl, p.err);
           dead = true;
         } else {
@@ -636,7 +637,7 @@ __global__ void __launch_bounds__(kScoreThreads, 1) k_score_accum(const __grid_c
       }
       const int ts = jt & 1;
       if (!dead) {
-        if (!__all_sync(kFull, mbar_wait(&ctl->t_full[ts], (jt >> 1) & 1, p.wait_ns))) {
+        if (!__all_sync(kFull, mbar_wait(&ctl->t_full[ts][0], (jt >> 1) & 1, p.wait_ns))) {
           fail(ctl, p.err);
           dead = true;
         } else {
