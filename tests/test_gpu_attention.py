@@ -202,28 +202,38 @@ def test_attention_at_mha_head_granularity():
     st.close()
 
 
-@pytest.mark.parametrize("lift", [10.0, 20.0], ids=["sum_over_guard", "reference_moves"])
-def test_attention_units_far_above_the_reference(lift):
-    """Alternate 64-key units whose logits sit `lift` log2 units above the
-    others (every window row, every group).  lift 10: a unit's 64 p reach
-    about 2^16 in sum although none exceeds 2^15, so the softmax takes the
-    unit maximum and keeps its reference (no move); lift 20: p would reach
-    2^20, so rows move their reference in the middle of a piece and rescale O.
-    Both against the fp64 oracle at the usual bounds."""
-    wl = syn.WORKLOADS["uitars_layer"]
-    si = syn.make_sequence(wl)
+def _lifted_keys(si, wl, lift_of_key, seed=7):
+    """Queries along one axis and past keys whose logit along it is
+    lift_of_key(t) log2 units, the other dimensions small noise."""
     d, lp = wl.head_dim, si.L - wl.window
-    g = torch.Generator().manual_seed(7)
+    g = torch.Generator().manual_seed(seed)
     beta = 8.0
-    gamma = lift / (beta / math.sqrt(d) * math.log2(math.e))   # q.k / sqrt(d) = lift / log2(e)
     q = 0.05 * torch.randn(si.q.shape, generator=g)
     q[..., 0] = beta
     k = si.k.float().clone()
     k[..., :lp, :] = 0.05 * torch.randn(k[..., :lp, :].shape, generator=g)
-    units = torch.arange(lp) // 64
-    k[..., :lp, 0] = torch.where(units % 2 == 1, torch.tensor(gamma), torch.tensor(0.0))
+    lift = torch.tensor([lift_of_key(t) for t in range(lp)], dtype=torch.float32)
+    k[..., :lp, 0] = lift / (beta / math.sqrt(d) * math.log2(math.e))   # q.k / sqrt(d) = lift / log2(e)
     si.q = q.to(torch.bfloat16)
     si.k = k.to(torch.bfloat16)
+
+
+@pytest.mark.parametrize("pattern", ["sum_over_guard", "reference_moves"])
+def test_attention_keys_far_above_the_reference(pattern):
+    """Logits that force the softmax off its fast path, against the fp64
+    oracle at the usual bounds.  sum_over_guard: every other 128-key block 10
+    log2 units up, so that after a low block the 64 p of a half sum to about
+    2^16 although none exceeds 2^15: the maximum is taken and the reference
+    stays.  reference_moves: a sawtooth rising 20 log2 units every 64 keys
+    (eight steps, then down again), so that references move in the middle of
+    pieces, in the first half of a unit (O and the row sum rescaled) and in
+    the second (the first half's stored P rescaled too)."""
+    wl = syn.WORKLOADS["uitars_layer"]
+    si = syn.make_sequence(wl)
+    if pattern == "sum_over_guard":
+        _lifted_keys(si, wl, lambda t: 10.0 * ((t // 128) % 2))
+    else:
+        _lifted_keys(si, wl, lambda t: 20.0 * ((t // 64) % 8))
     st = sk.init_state(H.gpu_config(wl, H.hyper()))
     ds = _attach(H.device_seq(si, wl), si, wl)
     _run_attention(st, [ds])
