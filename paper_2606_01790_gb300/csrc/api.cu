@@ -895,9 +895,17 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
   }
   // layers are independent: the step runs in chunks of layers so that the
   // upload of chunk i+1 and the download of chunk i-1 overlap the compute of
-  // chunk i (the host link carries both directions at once)
-  const int chunk = std::min(NL, 4);
-  const int nchunk = (NL + chunk - 1) / chunk;
+  // chunk i (the host link carries both directions at once).  Chunks of four
+  // layers, the last ones halving (4 layers as 2 + 1 + 1): what follows the
+  // last upload (that chunk's compute and download) is then one layer's
+  std::vector<int> chunk_l0;
+  for (int l0 = 0; l0 < NL;) {
+    const int rem = NL - l0;
+    chunk_l0.push_back(l0);
+    l0 += rem > 4 ? 4 : (rem + 1) / 2;
+  }
+  chunk_l0.push_back(NL);
+  const int nchunk = static_cast<int>(chunk_l0.size()) - 1;
   const size_t n_ev = 2 + 2 * static_cast<size_t>(nchunk);
   while (st->pipe_ev.size() < n_ev) {
     cudaEvent_t e = nullptr;
@@ -961,7 +969,7 @@ starkv_status starkv_step_host(starkv_state* st, const starkv_seq* seqs, int32_t
                            cudaMemcpyDeviceToHost, st->pipe_out);
   };
   for (int k = 0; k < nchunk; ++k) {
-    const int l0 = k * chunk, nl = std::min(chunk, NL - l0);
+    const int l0 = chunk_l0[k], nl = chunk_l0[k + 1] - l0;
     for (int i = 0; i < nseq; ++i) {
       const starkv_seq& h = seqs[i];
       const starkv_seq& d = dev[i];
