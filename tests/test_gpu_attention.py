@@ -241,6 +241,27 @@ def test_attention_keys_far_above_the_reference(pattern):
     st.close()
 
 
+def test_attention_on_sixteen_ragged_sequences():
+    """Config 5's batch (16 sequences of 1-12 screenshots and 128-1,024 text
+    tokens) in one launch over 28 layers: every sequence's output against the
+    oracle on one layer, rotating over the stack, and its normaliser on two
+    more."""
+    wl = syn.WORKLOADS["ragged"]
+    sis = [syn.make_sequence(wl, seq=i) for i in range(wl.n_seqs)]
+    st = sk.init_state(H.gpu_config(wl, H.hyper(), max_seqs=wl.n_seqs))
+    dss = [_attach(H.device_seq(si, wl, slot=i), si, wl) for i, si in enumerate(sis)]
+    kt = _run_attention(st, dss)
+    assert kt["attention"][0] == 1   # one launch for the whole batch
+    for i, (si, ds) in enumerate(zip(sis, dss)):
+        layer = (11 * i) % wl.n_layers
+        check_layer(ds, si, wl, layer)
+        for extra in ((layer + 9) % wl.n_layers, (layer + 19) % wl.n_layers):
+            ref = O.window_lse(si.q[extra].double().numpy(), si.k[extra].double().numpy(), wl.window)
+            np.testing.assert_allclose(ds.seq.attn_lse[extra].double().cpu().numpy(), ref, rtol=LSE_REL,
+                                       atol=LSE_TOL)
+    st.close()
+
+
 @pytest.mark.parametrize("name", ["tiny", "uitars_layer"])
 def test_step_fed_by_the_attention_pass_matches_oracle(name):
     """The compression step with lse = attn_lse: pass 1 skipped, the group
