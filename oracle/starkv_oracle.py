@@ -53,9 +53,10 @@ parameter with the stated default):
   factor per row, so in this mode the MI prior scales the scores without
   changing any set; only D changes the ranking.
 
-Parity of the absolute values of MI, w and phi on realistic inputs is
-unpinned beyond the closed forms and library cross-checks in the tests: the
-paper prints no worked example, and these values depend on the readings above.
+MI, MI_bar and w of a layer are pinned end to end against scikit-learn and
+scipy on small layers, and phi against scipy's cosine; that these are the
+paper's values rests on the readings above, which the paper fixes with no
+worked example (parity unpinned in that sense only).
 """
 from __future__ import annotations
 

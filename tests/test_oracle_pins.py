@@ -646,6 +646,37 @@ def test_mi_over_the_newest_frame_vs_sklearn():
     assert not np.allclose(full["mi"], o["mi"])   # the span matters
 
 
+def test_mi_prior_of_a_layer_end_to_end_vs_sklearn_and_scipy():
+    """The default span: MI_g of every group over all visual tokens of the
+    layer (equal-frequency rank bins of the pooled score, scipy ordinal ranks;
+    patch cells on the M x M grid) against scikit-learn's mutual_info_score,
+    the prior w = softmax(min-max(MI_bar) / tau) against scipy's softmax, and
+    the EMA carried into a second step with new scores."""
+    metrics = pytest.importorskip("sklearn.metrics")
+    K, M, R, C = 4, 2, 4, 5
+    p = O.Params(n_warmup=0, n_ramp=0, pool_kernel=3, mi_bins=K, mi_grid=M, tau=0.7, rho_mi=0.8)
+    st = O.LayerState.fresh(3, R, C)
+    mi_bar = None
+    for step, seed in enumerate((71, 72)):
+        q, k, meta, F_ = _small_case(seed, G=3, shots=3, n_text=20)
+        is_vis, frame, row, col = meta
+        s = O.score_layer(q, k, q.shape[1], p)
+        lp = s.shape[1]
+        o = O.select_layer(s, *meta, F_, 9, R, C, st, p)
+        sel = is_vis[:lp] != 0
+        cells = (row[:lp][sel] * M // R) * M + (col[:lp][sel] * M // C)
+        mi = np.empty(3)
+        for g in range(3):
+            v = s[g][sel]
+            bins = (scipy.stats.rankdata(v, method="ordinal").astype(np.int64) - 1) * K // v.size
+            mi[g] = metrics.mutual_info_score(bins, cells)
+        np.testing.assert_allclose(o["mi"], mi, rtol=0, atol=1e-12)
+        mi_bar = mi.copy() if step == 0 else p.rho_mi * mi_bar + (1 - p.rho_mi) * mi
+        np.testing.assert_allclose(o["mi_bar"], mi_bar, rtol=0, atol=1e-12)
+        m = (mi_bar - mi_bar.min()) / (mi_bar.max() - mi_bar.min() + p.eps)
+        np.testing.assert_allclose(o["w"], scipy.special.softmax(m / p.tau), rtol=0, atol=1e-12)
+
+
 def test_mha_granularity_by_replicated_kv_keeps_s_bar():
     """The paper's MHA-head ablation on a GQA model: every group's keys
     replicated for each of its query heads (G' = H).  Each head's row of S is
