@@ -263,13 +263,18 @@ def run_oracle_subprocess(workload, budget_s=15.0, max_layers=28, repeat=0, sele
     return d
 
 
+def seconds_text(t):
+    """A duration in s, or in ms below one second."""
+    return f"{t:.1f} s" if t >= 1.0 else f"{1e3 * t:.1f} ms"
+
+
 def oracle_sample(d, what):
     """Words for a timed oracle sample, with the whole-step extrapolation."""
     per_layer = d["seconds"] / max(1, d["calls"])
     return (f"{what}: {d['calls']} layer compressions of sequence 0 (layers "
             f"{min(d['layers'])}..{max(d['layers'])} cycled, step 0 of the workload), {d['tokens']} "
             f"tokens scored in {d['seconds']:.1f} s, numpy BLAS on {d['cores']} thread(s); a whole "
-            f"{d['n_layers']}-layer step extrapolates to {d['n_layers'] * per_layer:.1f} s at this rate")
+            f"{d['n_layers']}-layer step extrapolates to {seconds_text(d['n_layers'] * per_layer)} at this rate")
 
 
 def cpu_baselines(args):
@@ -304,7 +309,7 @@ def reference_arm(args):
     sample = (f"one layer compression per step (layer = step mod {wl.n_layers}, sequence 0, step 0 of the "
               f"workload; L_past = {d['l_past']} tokens scored per step), numpy BLAS on {d['cores']} "
               f"threads; a whole {wl.n_layers}-layer step extrapolates to "
-              f"{wl.n_layers * total / len(times):.1f} s at this rate")
+              f"{seconds_text(wl.n_layers * total / len(times))} at this rate")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,

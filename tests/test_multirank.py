@@ -62,6 +62,31 @@ def test_reference_arm_prints_on_rank_zero_only():
     assert r.stdout.strip() == ""
 
 
+def test_reference_arm_line_keeps_the_contract():
+    """The reference arm (the fp64 oracle on the host cores) on the tiny
+    workload: one JSON line with the contract's keys, the metric's unit and
+    direction, a cpu_baseline describing the run and an e2e object that moves
+    no bytes over the host link."""
+    env = dict(os.environ)
+    for v in ("RANK", "WORLD_SIZE", "LOCAL_RANK"):
+        env.pop(v, None)
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload", "tiny",
+                        "--steps", "1", "--warmup", "0"], env=env, capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr
+    lines = [l for l in r.stdout.splitlines() if l.strip()]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better",
+                "scaling", "vs_baseline", "dtype", "data", "config", "cpu_baseline", "e2e"):
+        assert key in d, key
+    assert d["impl"] == "reference" and d["unit"] == "tokens/s" and d["higher_is_better"] is True
+    assert d["value"] > 0 and d["ms_per_step"] > 0 and d["steps"] == 1
+    assert d["config"]["workload"] == "tiny"
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+
+
 def test_recorded_traffic_follows_the_kernel_code_not_its_comments():
     """The DRAM bytes a committed ncu capture recorded are reported only for
     the code they were measured on: the key ignores comments and layout, and
